@@ -1,0 +1,263 @@
+"""ctypes wrapper of the CPU oracle (test infrastructure only).
+
+Only the tests, the smoke check and the benchmark's CPU-baseline leg load this
+module.  It compiles ``trimmoe_oracle.cpp`` with gcc (``-ffp-contract=off``,
+OpenMP) into ``oracle/_build/liboracle.so`` and exposes numpy-level helpers.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+SRC = os.path.join(HERE, "trimmoe_oracle.cpp")
+BUILD_DIR = os.path.join(HERE, "_build")
+LIB_PATH = os.path.join(BUILD_DIR, "liboracle.so")
+
+A_EXEC, A_SKIP, A_EXIT, A_DEAD = 0, 1, 2, 3
+
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    os.makedirs(BUILD_DIR, exist_ok=True)
+    if force or not os.path.exists(LIB_PATH) or os.path.getmtime(LIB_PATH) < os.path.getmtime(SRC):
+        tmp = LIB_PATH + f".{os.getpid()}.tmp"
+        cmd = ["g++", "-O2", "-std=c++17", "-fPIC", "-shared", "-ffp-contract=off", "-fno-fast-math",
+               "-fopenmp", "-o", tmp, SRC]
+        subprocess.check_call(cmd)
+        os.replace(tmp, LIB_PATH)
+    return LIB_PATH
+
+
+class OrModel(C.Structure):
+    _fields_ = [(n, C.c_int) for n in
+                ("N", "d", "E", "k", "F", "F_sh", "C", "M", "H", "act", "renorm_topk", "n_sub")] + \
+               [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref", "phi_beta")] + [
+        ("place", C.c_void_p), ("sim", C.c_void_p), ("sub_thresh", C.c_void_p),
+        ("trans", C.c_void_p), ("comp", C.c_void_p), ("P", C.c_void_p), ("theta", C.c_void_p),
+        ("lambda_", C.c_void_p), ("eps", C.c_void_p)]
+
+
+class OrLayerWeights(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in
+                ("W_r", "b_r", "W_x_prev", "b_x_prev", "W13", "W2", "W13_sh", "W2_sh")]
+
+
+class OrTokens(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in
+                ("s", "Dhat", "Dbar", "pJ", "alive", "last_exec", "xi_last", "exit_layer")]
+
+
+class OrLayerOut(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in
+                ("topk_idx", "topk_g", "I", "xi", "action", "exp_sel", "srv_sel", "perm",
+                 "group_off", "near", "Gamma", "tot_exec", "tot_skip")]
+
+
+class OrDecision(C.Structure):
+    _fields_ = [("topk", C.c_int * 16), ("g", C.c_float * 16)] + \
+               [(n, C.c_float) for n in ("I", "xi", "Gamma", "tot_exec", "tot_skip", "Lambda")] + \
+               [(n, C.c_int) for n in ("action", "skip_ok", "exit_ok")] + \
+               [("exp_sel", C.c_int * 16), ("srv_sel", C.c_int * 16), ("Q_sel", C.c_float * 16),
+                ("f_sel", C.c_float * 16), ("Dhat_new", C.c_float), ("s_new", C.c_int), ("near", C.c_int)]
+
+
+def lib():
+    global _lib
+    with _lock:
+        if _lib is None:
+            L = C.CDLL(build())
+            vp, i, f = C.c_void_p, C.c_int, C.c_float
+            L.or_router.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp]
+            L.or_exit_conf.argtypes = [vp, vp, vp, vp, vp]
+            L.or_exit_conf.restype = f
+            L.or_sub_loss.argtypes = [vp, i, i, i]
+            L.or_sub_loss.restype = f
+            L.or_candidates.argtypes = [vp, i, i, vp, vp, vp, i]
+            L.or_candidates.restype = i
+            L.or_exec_cost.argtypes = [vp, i, i, i, f, f]
+            L.or_exec_cost.restype = f
+            L.or_lookahead_table.argtypes = [vp, i, f, f, vp]
+            L.or_phi_naive.argtypes = [vp, i, i, i, i, f, f]
+            L.or_phi_naive.restype = f
+            L.or_decide_given.argtypes = [vp, i, vp, vp, f, f, i, f, f, f, i, vp]
+            L.or_decide_token.argtypes = [vp, vp, i, vp, i, f, f, f, i, vp, vp]
+            L.or_ffn_row.argtypes = [i, i, i, vp, vp, vp, vp]
+            L.or_layer_step.argtypes = [vp, vp, i, i, vp, vp, vp, vp, i]
+            L.or_layer_step.restype = i
+            L.or_forward.argtypes = [vp, vp, i, vp, vp, i]
+            L.or_forward.restype = i
+            L.or_max_threads.restype = i
+            _lib = L
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data
+
+
+class OracleModel:
+    """Holds the numpy arrays alive and the ctypes model struct."""
+
+    def __init__(self, cfg, tables, small, experts=None):
+        self.cfg = cfg
+        self.keep = {}
+        def keep(name, a, dt):
+            a = np.ascontiguousarray(a, dtype=dt)
+            self.keep[name] = a
+            return a
+        t = tables
+        self.m = OrModel(
+            N=cfg.N, d=cfg.d, E=cfg.E, k=cfg.k, F=cfg.F, F_sh=cfg.F_sh, C=cfg.C, M=cfg.M, H=cfg.H,
+            act=cfg.act, renorm_topk=cfg.renorm_topk, n_sub=cfg.n_sub,
+            omega_T=cfg.omega_T, omega_D=cfg.omega_D, d_ref=t["d_ref"], phi_beta=cfg.phi_beta,
+            place=_p(keep("place", t["place"], np.uint16)), sim=_p(keep("sim", t["sim"], np.float32)),
+            sub_thresh=_p(keep("sub_thresh", t["sub_thresh"], np.float32)),
+            trans=_p(keep("trans", t["trans"], np.float32)), comp=_p(keep("comp", t["comp"], np.float32)),
+            P=_p(keep("P", t["P"] if t["P"].size else np.zeros((1, cfg.E, cfg.E)), np.float32)),
+            theta=_p(keep("theta", t["theta"], np.float32)), lambda_=_p(keep("lam", t["lam"], np.float32)),
+            eps=_p(keep("eps", t["eps"], np.float32)))
+        self.small = {k: np.ascontiguousarray(v) for k, v in small.items()}
+        self.experts = experts   # dict of numpy arrays (bf16 bits) per layer or full, or None
+
+    def layer_weights(self, l, experts_l=None):
+        """experts_l: dict with W13, W2 (and W13_sh, W2_sh) for layer l (uint16 arrays)."""
+        s = self.small
+        if experts_l is None:
+            e = self.experts or {}
+            experts_l = {k: e[k][l] for k in e}
+        ex = {k: np.ascontiguousarray(v, dtype=np.uint16) for k, v in experts_l.items()}
+        br = np.ascontiguousarray(s["b_r"][l], dtype=np.float32)
+        wr = np.ascontiguousarray(s["W_r"][l], dtype=np.uint16)
+        wx = np.ascontiguousarray(s["W_x"][l - 1], dtype=np.uint16) if l > 0 else None
+        bx = np.ascontiguousarray(s["b_x"][l - 1], dtype=np.float32) if l > 0 else None
+        lw = OrLayerWeights(W_r=_p(wr), b_r=_p(br), W_x_prev=_p(wx), b_x_prev=_p(bx),
+                            W13=_p(ex.get("W13")), W2=_p(ex.get("W2")),
+                            W13_sh=_p(ex.get("W13_sh")), W2_sh=_p(ex.get("W2_sh")))
+        lw._keep = (wr, br, wx, bx, ex)
+        return lw
+
+
+def tokens_struct(tok):
+    arrs = {
+        "s": np.ascontiguousarray(tok["s"], dtype=np.uint8),
+        "Dhat": np.ascontiguousarray(tok["Dhat"], dtype=np.float32),
+        "Dbar": np.ascontiguousarray(tok["Dbar"], dtype=np.float32),
+        "pJ": np.ascontiguousarray(tok["pJ"], dtype=np.float32),
+        "alive": np.ascontiguousarray(tok["alive"], dtype=np.uint8),
+        "last_exec": np.ascontiguousarray(tok["last_exec"], dtype=np.uint8),
+        "xi_last": np.ascontiguousarray(tok["xi_last"], dtype=np.float32),
+        "exit_layer": np.ascontiguousarray(tok["exit_layer"], dtype=np.int16),
+    }
+    st = OrTokens(**{k: _p(v) for k, v in arrs.items()})
+    return st, arrs
+
+
+def alloc_layer_out(T, cfg):
+    K, E = cfg.k, cfg.E
+    o = dict(
+        topk_idx=np.zeros(T * K, np.int32), topk_g=np.zeros(T * K, np.float32),
+        I=np.zeros(T, np.float32), xi=np.zeros(T, np.float32), action=np.zeros(T, np.uint8),
+        exp_sel=np.zeros(T * K, np.uint8), srv_sel=np.zeros(T * K, np.uint8),
+        perm=np.full(T * K + T, -1, np.int32), group_off=np.zeros(E + 2, np.int32),
+        near=np.zeros(T, np.uint8), Gamma=np.zeros(T, np.float32), tot_exec=np.zeros(T, np.float32),
+        tot_skip=np.zeros(T, np.float32))
+    return OrLayerOut(**{k: _p(v) for k, v in o.items()}), o
+
+
+def layer_step(om: OracleModel, l, h, tok, experts_l=None, row_mask=None, nthreads=0):
+    """Run one layer; returns (h_out, tokens_out, outputs). Inputs are not modified."""
+    T = h.shape[0]
+    h = np.array(h, dtype=np.uint16, copy=True, order="C")
+    st, arrs = tokens_struct({k: np.array(v, copy=True) for k, v in tok.items()})
+    out_s, out = alloc_layer_out(T, om.cfg)
+    lw = om.layer_weights(l, experts_l)
+    rm = None if row_mask is None else np.ascontiguousarray(row_mask, dtype=np.uint8)
+    rc = lib().or_layer_step(C.byref(om.m), C.byref(lw), l, T, _p(h), C.byref(st), C.byref(out_s),
+                             _p(rm), nthreads)
+    if rc:
+        raise RuntimeError(f"or_layer_step failed: {rc}")
+    return h, arrs, out
+
+
+def forward(om: OracleModel, h, tok, nthreads=0):
+    T = h.shape[0]
+    h = np.array(h, dtype=np.uint16, copy=True, order="C")
+    st, arrs = tokens_struct({k: np.array(v, copy=True) for k, v in tok.items()})
+    lws = (OrLayerWeights * om.cfg.N)()
+    keep = []
+    for l in range(om.cfg.N):
+        lw = om.layer_weights(l)
+        keep.append(lw)
+        lws[l] = lw
+    rc = lib().or_forward(C.byref(om.m), lws, T, _p(h), C.byref(st), nthreads)
+    if rc:
+        raise RuntimeError(f"or_forward failed: {rc}")
+    return h, arrs
+
+
+def router(om: OracleModel, l, h_row):
+    cfg = om.cfg
+    z = np.zeros(cfg.E, np.float32); p = np.zeros(cfg.E, np.float32)
+    topk = np.zeros(16, np.int32); g = np.zeros(16, np.float32); I = np.zeros(1, np.float32)
+    wr = np.ascontiguousarray(om.small["W_r"][l], dtype=np.uint16)
+    br = np.ascontiguousarray(om.small["b_r"][l], dtype=np.float32)
+    hr = np.ascontiguousarray(h_row, dtype=np.uint16)
+    lib().or_router(C.byref(om.m), _p(wr), _p(br), _p(hr), _p(z), _p(p), _p(topk), _p(g), _p(I))
+    return z, p, topk[:cfg.k].copy(), g[:cfg.k].copy(), float(I[0])
+
+
+def exit_conf(om: OracleModel, W_x_l, b_x_l, h_row):
+    wx = np.ascontiguousarray(W_x_l, dtype=np.uint16)
+    bx = np.ascontiguousarray(b_x_l, dtype=np.float32)
+    hr = np.ascontiguousarray(h_row, dtype=np.uint16)
+    return float(lib().or_exit_conf(C.byref(om.m), _p(wx), _p(bx), _p(hr), None))
+
+
+def candidates(om: OracleModel, l, r):
+    cap = om.cfg.M * om.cfg.E
+    cm = np.zeros(cap, np.int32); ck = np.zeros(cap, np.int32); cQ = np.zeros(cap, np.float32)
+    n = lib().or_candidates(C.byref(om.m), l, r, _p(cm), _p(ck), _p(cQ), cap)
+    return [(int(cm[i]), int(ck[i]), float(cQ[i])) for i in range(n)]
+
+
+def exec_cost(om, l, s, m, Q, Dbar):
+    return float(lib().or_exec_cost(C.byref(om.m), l, s, m, C.c_float(Q), C.c_float(Dbar)))
+
+
+def lookahead_table(om, l, R, Dbar):
+    out = np.zeros(om.cfg.M * om.cfg.E, np.float32)
+    lib().or_lookahead_table(C.byref(om.m), l, C.c_float(R), C.c_float(Dbar), _p(out))
+    return out.reshape(om.cfg.M, om.cfg.E)
+
+
+def phi_naive(om, l, h, m, k, R, Dbar):
+    return float(lib().or_phi_naive(C.byref(om.m), l, h, m, k, C.c_float(R), C.c_float(Dbar)))
+
+
+def decide_given(om, l, topk, g, I, xi, s, Dhat, Dbar, pJ, last_exec):
+    tk = np.zeros(16, np.int32); tk[:len(topk)] = topk
+    gg = np.zeros(16, np.float32); gg[:len(g)] = g
+    D = OrDecision()
+    lib().or_decide_given(C.byref(om.m), l, _p(tk), _p(gg), C.c_float(I), C.c_float(xi), s,
+                          C.c_float(Dhat), C.c_float(Dbar), C.c_float(pJ), last_exec, C.byref(D))
+    return D
+
+
+def ffn_row(d, F, act, W13_e, W2_e, x):
+    y = np.zeros(d, np.uint16)
+    w13 = np.ascontiguousarray(W13_e, dtype=np.uint16)
+    w2 = np.ascontiguousarray(W2_e, dtype=np.uint16)
+    xx = np.ascontiguousarray(x, dtype=np.uint16)
+    lib().or_ffn_row(d, F, act, _p(w13), _p(w2), _p(xx), _p(y))
+    return y
+
+
+def max_threads():
+    return int(lib().or_max_threads())
