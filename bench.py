@@ -1,0 +1,353 @@
+"""Benchmark: tokens/s of one adaptive-depth MoE forward on GB300, and % of roofline.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config mixtral] [--impl ours|reference]
+
+A step is one full forward (all layers: decide, compact, gather, grouped FFN,
+combine) over T tokens of the seeded synthetic workload, starting from the
+same initial hidden states and token state each step (a 134 MB device copy
+that is part of the step).  Inputs are larger than L2 (Mixtral-shaped: 90 GB
+of expert weights, 134 MB of hidden states), so no L2 flush is needed.
+
+Under torchrun each rank runs an independent replica on its own GPU (weak
+scaling: the token batches are independent and the method has no exchange
+step); rank 0 prints one JSON line with the max time over ranks.
+
+--impl reference times the CPU oracle on the host cores on a bounded sample
+of the same workload (S tokens through L layers, scaled to tokens/s of a full
+forward).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "tokens/s per adaptive-depth MoE forward on 1 GB300; % of roofline"
+UNIT = "tokens/s"
+
+# Oracle sample per configuration: (tokens, layers) -- about 10-30 s on 16 cores.
+CPU_SAMPLE = {"switch_tiny": (64, 4), "switch": (512, 12), "qwen": (256, 2), "mixtral": (128, 2),
+              "mixtral_decode": (128, 2)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return rank, world, local
+
+
+def init_dist(world):
+    if world <= 1:
+        return None
+    import torch.distributed as dist
+    dist.init_process_group("gloo")
+    return dist
+
+
+def max_over_ranks(dist, v: float) -> float:
+    if dist is None:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            j = json.load(fh)
+        return dict(hbm=j["hbm_gbs"], bf16=j["bf16_tflops"], bf16_sus=j["bf16_tflops_sustained"],
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        with open(self.path) as fh:
+            for line in fh:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return float("nan")
+        sm = [num(r[1]) for r in rows]
+        mx = [num(r[2]) for r in rows]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for n, v in zip(names, r[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        loaded = [s for s in sm if not math.isnan(s)]
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": len(rows)}
+
+
+def make_workload(cfg, device):
+    from paper_2608_00573_gb300 import workload as W
+    small = W.make_small_weights(cfg)
+    tables = W.make_tables(cfg, small["W_r"])
+    experts = W.make_expert_weights_device(cfg, device=device)
+    tok = W.make_tokens(cfg)
+    return small, tables, experts, tok
+
+
+def cpu_baseline(cfg, small, tables, experts, tok, n_tok, n_layers, steps=1):
+    """Time the oracle (all host cores) on n_tok tokens through layers 0..n_layers-1."""
+    import numpy as np
+    import torch
+    from oracle import oracle as O
+    O.build()
+    om = O.OracleModel(cfg, tables, small, None)
+    n_layers = min(n_layers, cfg.N)
+    ex_l = []
+    for l in range(n_layers):
+        d = {}
+        for k, v in experts.items():
+            if v is None:
+                continue
+            x = v[l]
+            if hasattr(x, "detach"):
+                x = x.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+            d[k] = np.ascontiguousarray(x)
+        ex_l.append(d)
+    sub = {k: np.ascontiguousarray(v[:n_tok]) for k, v in tok.items()}
+    threads = O.max_threads()
+    times = []
+    for _ in range(steps):
+        h = sub["h"].copy()
+        st = {k: v.copy() for k, v in sub.items() if k != "h"}
+        t0 = time.perf_counter()
+        for l in range(n_layers):
+            h, st, _ = O.layer_step(om, l, h, st, experts_l=ex_l[l], nthreads=threads)
+        times.append(time.perf_counter() - t0)
+    per_forward = [t * cfg.N / n_layers for t in times]
+    vals = [n_tok / t for t in per_forward]
+    return vals, threads, f"{n_tok} tokens x layers 0..{n_layers - 1} of the {cfg.name} workload, " \
+                          f"time scaled by {cfg.N}/{n_layers} to a full forward"
+
+
+def run_reference(args):
+    rank, world, local = dist_env()
+    if rank != 0:
+        return
+    import torch
+    from paper_2608_00573_gb300 import workload as W
+    cfg = W.CONFIGS[args.config]
+    device = "cuda" if torch.cuda.is_available() else "cpu"
+    small, tables, experts, tok = make_workload(cfg, device)
+    n_tok, n_layers = CPU_SAMPLE.get(cfg.name, (64, 2))
+    vals, threads, sample = cpu_baseline(cfg, small, tables, experts, tok, n_tok, n_layers,
+                                         steps=args.warmup + args.steps)
+    vals = vals[args.warmup:]
+    v = statistics.median(vals)
+    ms = cfg.T / v * 1e3
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "impl": "reference", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "T": cfg.T, "N": cfg.N, "d": cfg.d, "E": cfg.E, "k": cfg.k,
+                       "F": cfg.F, "F_sh": cfg.F_sh, "H": cfg.H, "budget": cfg.budget},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    from paper_2608_00573_gb300 import binding as B
+    from paper_2608_00573_gb300 import workload as W
+
+    rank, world, local = dist_env()
+    dist = init_dist(world)
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    B.lib()
+    cfg = W.CONFIGS[args.config]
+    T = cfg.T
+    small, tables, experts, tok = make_workload(cfg, device)
+    eng = B.Engine(cfg, tables, small, experts, T_max=T, device=device, profile=True)
+    tok0 = eng.tokens_to_device(tok)
+    work = {k: v.clone() for k, v in tok0.items()}
+    stream = torch.cuda.current_stream(device)
+
+    def step():
+        for k in work:
+            work[k].copy_(tok0[k], non_blocking=True)
+        eng.forward(work, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    st0 = eng.stats()
+    if st0["status"] != 0:
+        raise RuntimeError(f"warm-up failed: {st0}")
+    eng.reset_stats()
+    clocks = ClockSampler(local)
+    barrier(dist)
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier(dist)
+    ms_total = ev0.elapsed_time(ev1)
+    clk = clocks.stop()
+    st = eng.stats()
+    if st["status"] != 0 or st["device_error"]:
+        raise RuntimeError(f"timed run failed: {st}")
+    ms_step = max_over_ranks(dist, ms_total / args.steps)
+    value = T * world / (ms_step / 1e3)
+
+    # End to end through the public host-buffer entry point (pinned host memory).
+    host = {k: v.cpu().pin_memory() for k, v in tok0.items()}
+    host_src = {k: v.clone().pin_memory() for k, v in host.items()}
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    for _ in range(1):
+        eng.forward_host(host, stream=stream)
+    barrier(dist)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for k in host:
+            host[k].copy_(host_src[k])
+        eng.forward_host(host, stream=stream)
+    e2e_s = max_over_ranks(dist, (time.perf_counter() - t0) / args.steps)
+    e2e = {"value": T * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": h2d}
+
+    # Roofline of the dominant kernel (grouped FFN GEMM) from events recorded
+    # around each launch on the launching stream during the timed region.
+    peaks = load_peaks()
+    kinds = {"grouped_gemm_gate_up": (st["ms_gemm_up"], st["flops_gemm_up"], st["n_gemm_up"]),
+             "grouped_gemm_down": (st["ms_gemm_down"], st["flops_gemm_down"], st["n_gemm_down"])}
+    dom = max(kinds, key=lambda k: kinds[k][0])
+    ms_k, fl_k, n_k = kinds[dom]
+    achieved = fl_k / (ms_k / 1e3) / 1e12 if ms_k > 0 else 0.0
+    traffic = None
+    tp = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tp):
+        with open(tp) as fh:
+            tj = json.load(fh)
+        ent = tj.get(cfg.name, {}).get(dom)
+        if ent and ent.get("kernel_rev") == KERNEL_REV:
+            traffic = ent.get("bytes_per_launch")
+    roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peaks["bf16_sus"],
+            "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sus"], "traffic": traffic,
+            "peak_source": f"{peaks['source']} bf16 sustained",
+            "flops_per_launch": fl_k / max(n_k, 1), "ms_per_launch": ms_k / max(n_k, 1)}
+    # Whole-forward roofline: executed GEMM FLOPs at the bf16 peak vs bytes at HBM.
+    per_fwd_flops = st["gemm_flops"] / args.steps
+    fwd_roof_ms = per_fwd_flops / (peaks["bf16_sus"] * 1e12) * 1e3
+    kernel_ms = {k: st[f"ms_{k}"] / args.steps for k in
+                 ("decide", "compact", "gather", "gemm_up", "gemm_down", "combine")}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name, "T": T, "N": cfg.N, "d": cfg.d, "E": cfg.E, "k": cfg.k, "F": cfg.F,
+                   "F_sh": cfg.F_sh, "H": cfg.H, "budget": cfg.budget, "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (expert weights and hidden states)"},
+        "roofline": roof,
+        "forward_roofline": {"gemm_flops_per_forward": per_fwd_flops, "roofline_ms": fwd_roof_ms,
+                             "frac": fwd_roof_ms / ms_step},
+        "kernel_ms_per_step": kernel_ms,
+        "decisions": {"layer_tokens": st["layer_tokens"] // args.steps,
+                      "skip_share": st["skipped"] / max(st["layer_tokens"], 1),
+                      "exit_share_of_tokens": st["exited"] / args.steps / T,
+                      "remote_share_of_pairs": (st["pairs_remote_exact"] + st["pairs_remote_sub"]) /
+                      max(st["pairs_local_exact"] + st["pairs_local_sub"] + st["pairs_remote_exact"] +
+                          st["pairs_remote_sub"], 1)},
+        "e2e": e2e,
+        "gpu_launches": st["launches"],
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_tok, n_layers = CPU_SAMPLE.get(cfg.name, (64, 2))
+        vals, threads, sample = cpu_baseline(cfg, small, tables, experts, tok, n_tok, n_layers)
+        line["cpu_baseline"] = {"value": vals[0], "unit": UNIT, "cores": threads, "kind": "oracle",
+                                "sample": sample}
+    eng.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+# Revision tag of the timed GEMM kernel; a stored ncu traffic figure is used
+# only when it was taken on this revision.
+KERNEL_REV = "gemm-v1"
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--config", default="mixtral")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,222 @@
+/*
+ * trimmoe.h -- C ABI of the GB300 (sm_103a) adaptive-depth MoE layer step.
+ *
+ * The library implements the per-token, per-layer online decision of the
+ * paper's Sec. V (Algorithm 2 / Table II) together with the MoE computation it
+ * gates: router and importance (Eq. 4), exit-head confidence (Eq. 7-9), skip
+ * test (Eq. 5, 34, 35), substitute-or-fetch with server choice and look-ahead
+ * (Eq. 30-31, 38-40), state updates (Eq. 41-42), compaction of the executed
+ * (token, expert) pairs, grouped expert FFN and the gate-weighted combine.
+ * The M edge servers of Sec. III-A are simulated by the placement and cost
+ * tables only.
+ *
+ * Conventions for every call:
+ *  - Functions never abort or throw; they return a trimmoe_status and
+ *    trimmoe_last_error() gives a one-line reason for the handle's last error.
+ *  - "device" pointers are CUDA device memory owned by the caller; they must
+ *    stay valid until the work queued on the stream has finished.  "host"
+ *    tables are copied during trimmoe_create and may be freed afterwards.
+ *  - bf16 values are IEEE bfloat16 bit patterns (uint16).  All arrays are
+ *    dense, row-major, with the shapes given in brackets.
+ *  - Layers, experts, servers and tokens are 0-based.
+ *  - Calls are asynchronous on the given stream (a cudaStream_t passed as
+ *    void*, NULL = legacy default stream) except trimmoe_stats and
+ *    trimmoe_forward_host, which synchronise.  A handle must not be used by
+ *    two streams or two host threads at the same time: its workspaces are
+ *    shared by all its calls.
+ */
+#ifndef TRIMMOE_H
+#define TRIMMOE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    TRIMMOE_OK = 0,
+    TRIMMOE_ERR_ARG = -1,            /* null / misaligned pointer, bad size or layer */
+    TRIMMOE_ERR_UNSUPPORTED = -2,    /* dimensions this build does not handle */
+    TRIMMOE_ERR_OOM = -3,            /* device allocation failed */
+    TRIMMOE_ERR_CUDA = -4,           /* a CUDA runtime/driver call failed */
+    TRIMMOE_ERR_COVERAGE = -5,       /* an expert has no server (violates Eq. 2) */
+    TRIMMOE_ERR_DEVICE_TIMEOUT = -6  /* a kernel gave up waiting and flagged it */
+} trimmoe_status;
+
+typedef struct trimmoe* trimmoe_handle;
+
+/* Actions written to trimmoe_layer_out.action (Sec. V-A). */
+enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
+
+/* Model and policy hyper-parameters.
+ *  N layers; d = d_model; E routed experts; k = top-k; F = routed expert d_ff;
+ *  F_sh = shared-expert d_ff (0 = none; always SwiGLU, always local, Sec. III-B);
+ *  C exit-head classes (1 = sigmoid head of Sec. IV-A, >1 = max softmax prob);
+ *  M servers (<= 16); H look-ahead horizon (Eq. 39, 1 = myopic);
+ *  act: 0 ReLU, 1 SwiGLU; renorm_topk: combine weights renormalised over the
+ *  top-k (the importance I of Eq. 4 always uses the raw softmax gates);
+ *  n_sub: substitutes per target (|R_{l,r}| <= n_sub, Sec. III-A);
+ *  T_max: largest token count of a call (sizes the workspaces);
+ *  omega_T, omega_D: weights of Eq. (21)/(31); d_ref_ms: d^ref of Eq. (31);
+ *  phi_beta: Q = phi_beta * (1 - Sim)/2 (Eq. 3 with a linear phi);
+ *  profile: 1 = record CUDA events around each kernel launch (trimmoe_stats
+ *  then reports per-kernel device time).
+ * Supported: d % 256 == 0; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
+ * F_sh % 128 == 0; E <= 128; k <= min(E, 8); C <= 256; M*E <= 1024; H <= 6;
+ * n_sub <= 3. */
+typedef struct {
+    int N, d, E, k, F, F_sh, C, M, H;
+    int act;
+    int renorm_topk;
+    int n_sub;
+    int T_max;
+    float omega_T, omega_D, d_ref_ms, phi_beta;
+    int profile;
+} trimmoe_config;
+
+/* Weights (device, bf16 except the biases, borrowed; 16-byte aligned).
+ *  W_r  [N][E][d], b_r fp32 [N][E]        router (Sec. III-B)
+ *  W_x  [N][C][d], b_x fp32 [N][C]        exit heads h_l (Eq. 7)
+ *  W13  [N][E][n13*F][d]   n13 = 2 (SwiGLU) or 1 (ReLU).  SwiGLU rows are
+ *       interleaved in blocks of 128: rows [256b, 256b+128) are gate rows
+ *       128b..128b+127 and rows [256b+128, 256b+256) the matching up rows.
+ *  W2   [N][E][d][F]
+ *  W13_sh [N][2*F_sh][d] (same interleave), W2_sh [N][d][F_sh]; NULL if F_sh == 0. */
+typedef struct {
+    const void* W_r;
+    const float* b_r;
+    const void* W_x;
+    const float* b_x;
+    const void* W13;
+    const void* W2;
+    const void* W13_sh;
+    const void* W2_sh;
+} trimmoe_weights;
+
+/* The paper's input tables (host, copied at create).
+ *  place [N][E]    bit m set iff expert k of layer l is deployed on server m,
+ *                  x_{m,l,k} of Eq. (1)-(2); every entry must be non-zero.
+ *  sim   [N][E][E] Sim_l(r, k) of Eq. (3); R_{l,r} = the n_sub experts k != r of
+ *                  highest Sim_l(r, k) with Sim >= sub_thresh[l] (ties: lower k).
+ *  sub_thresh [N]
+ *  trans_ms [M][M] z_l/B + tau between servers (Eq. 14); the diagonal is unused.
+ *  comp_ms  [N][M] c_l / F_m (Eq. 15).
+ *  P     [N-1][E][E] P_l(k -> k') (Eq. 38); rows sum to 1.  May be NULL if N == 1.
+ *  theta [N] importance thresholds (Eq. 24); lambda [N] Lambda = lambda_l * I
+ *  (Eq. 5); eps [N] per-layer skip tolerance (Eq. 25), used by the look-ahead. */
+typedef struct {
+    const uint16_t* place;
+    const float* sim;
+    const float* sub_thresh;
+    const float* trans_ms;
+    const float* comp_ms;
+    const float* P;
+    const float* theta;
+    const float* lambda;
+    const float* eps;
+} trimmoe_tables;
+
+/* Per-token state (device, borrowed, length >= T; updated in place).
+ *  hidden bf16 [T][d] hidden states h, read and written in place;
+ *  s current server (Eq. 29); Dhat accumulated degradation (Eq. 41-42);
+ *  Dbar per-token budget (Eq. 33); pJ confidence requirement (Eq. 8);
+ *  alive y (Eq. 6); last_exec 1 iff the previous layer executed (Eq. 9);
+ *  xi_last last exit confidence evaluated; exit_layer first layer that did not
+ *  run (N when the token ran every layer). */
+typedef struct {
+    void* hidden;
+    uint8_t* s;
+    float* Dhat;
+    float* Dbar;
+    float* pJ;
+    uint8_t* alive;
+    uint8_t* last_exec;
+    float* xi_last;
+    int16_t* exit_layer;
+} trimmoe_tokens;
+
+/* Optional per-layer outputs of trimmoe_layer_step (device; any may be NULL).
+ *  topk_idx int32 [T][k] (-1 for dead tokens); topk_g fp32 [T][k] softmax gates;
+ *  I fp32 [T]; xi fp32 [T] (-1 where not evaluated); action uint8 [T];
+ *  exp_sel, srv_sel uint8 [T][k] executed expert and server (255 unless EXEC);
+ *  perm int32 [T*k + T]: the executed pairs t*k+j ordered by (expert, t, j),
+ *  then the tokens that run the shared expert (executed or skipped) by t;
+ *  group_off int32 [E+2]: pairs of expert e are perm[group_off[e] ..
+ *  group_off[e+1]), shared rows perm[group_off[E] .. group_off[E+1]). */
+typedef struct {
+    int32_t* topk_idx;
+    float* topk_g;
+    float* I;
+    float* xi;
+    uint8_t* action;
+    uint8_t* exp_sel;
+    uint8_t* srv_sel;
+    int32_t* perm;
+    int32_t* group_off;
+} trimmoe_layer_out;
+
+/* Counters accumulated since create / the last reset (Fig. 5(b) categories). */
+typedef struct {
+    uint64_t layer_tokens;        /* live (token, layer) decisions */
+    uint64_t exec_tokens;         /* token-layers executed */
+    uint64_t skipped;             /* token-layers skipped */
+    uint64_t exited;              /* exits */
+    uint64_t pairs_local_exact;   /* executed (token, slot) pairs by kind */
+    uint64_t pairs_local_sub;
+    uint64_t pairs_remote_exact;
+    uint64_t pairs_remote_sub;
+    uint64_t shared_rows;         /* rows through the shared expert */
+    double delay_ms;              /* sum of d(m, k) of Eq. (30) over executed pairs */
+    double remote_hops;           /* executed pairs on a server other than s */
+    float max_budget_ratio;       /* max Dhat / Dbar seen after a decision */
+    int device_error;             /* non-zero if a kernel flagged a timeout */
+    uint64_t launches;            /* kernels launched by the library */
+    uint64_t layer_calls;         /* layers processed */
+    double gemm_flops;            /* 2*M*N*K of the grouped FFN GEMMs that ran */
+    /* Device time per kernel family in ms (profile != 0 only). */
+    double ms_decide, ms_compact, ms_gather, ms_gemm_up, ms_gemm_down, ms_combine;
+    uint64_t n_gemm_up, n_gemm_down;
+    double flops_gemm_up, flops_gemm_down;
+} trimmoe_stats_t;
+
+/* Validate, copy the tables, derive the candidate lists V_{l,r} and losses Q,
+ * allocate the workspaces for T_max tokens, and build the TMA descriptors.
+ * Errors: ARG (null or misaligned pointer, non-stochastic P), UNSUPPORTED
+ * (dimensions), COVERAGE (Eq. 2), OOM, CUDA.  *out is NULL on error. */
+trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmoe_weights* w,
+                              const trimmoe_tables* tab, trimmoe_handle* out);
+
+/* One MoE layer over tokens [0, T) (Alg. 2, lines 6-25, plus the gated FFN and
+ * combine).  Dead tokens are untouched.  0 <= layer < N, 0 <= T <= T_max.
+ * out may be NULL.  Asynchronous on stream. */
+trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T, trimmoe_tokens* tok,
+                                  trimmoe_layer_out* out, void* stream);
+
+/* Layers 0..N-1 in order (Alg. 2, lines 5-26).  Asynchronous on stream. */
+trimmoe_status trimmoe_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream);
+
+/* trimmoe_forward on HOST buffers: copies hidden and the token state to device
+ * buffers owned by the handle, runs the forward, copies them back and
+ * synchronises the stream.  Pointers in tok are host pointers (pinned memory
+ * gives the fastest copies). */
+trimmoe_status trimmoe_forward_host(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream);
+
+/* Synchronise the handle's last stream and read the counters.  Returns
+ * DEVICE_TIMEOUT if a kernel flagged one (the flag stays set until reset). */
+trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out);
+
+/* Zero the counters and the device error flag (synchronises). */
+trimmoe_status trimmoe_reset_stats(trimmoe_handle h);
+
+/* Last error message of the handle ("" if none); NULL handle: last create error. */
+const char* trimmoe_last_error(trimmoe_handle h);
+
+/* Free the handle and its workspaces (synchronises first).  NULL is a no-op. */
+void trimmoe_destroy(trimmoe_handle h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TRIMMOE_H */

@@ -1,0 +1,159 @@
+// Kernel (b): compaction of the executed (token, slot) pairs by expert and of
+// the tokens that run the shared expert, then a gather of their hidden rows.
+//
+// The order is a stable counting sort: pairs of expert e are laid out in
+// increasing (t, j), experts in increasing e, and the shared-expert rows
+// (tokens executed or skipped at this layer) follow in increasing t.  Alg. 2
+// (Sec. V-E) removes exited tokens from the active set; only the survivors'
+// pairs reach the expert FFN.
+//
+// Three passes over chunks of kChunk tokens: per-chunk bucket counts, one
+// scan over chunks and buckets, and a scatter in which one warp walks its
+// chunk in order and ranks equal buckets with __match_any_sync.
+#include "internal.cuh"
+
+namespace tmoe {
+
+namespace {
+
+constexpr int kChunk = 256;
+
+__global__ void __launch_bounds__(kChunk) count_kernel(const CompactParams p) {
+    __shared__ int cnt[kMaxE + 1];
+    const int nb = p.E + 1;
+    for (int i = threadIdx.x; i < nb; i += blockDim.x) cnt[i] = 0;
+    __syncthreads();
+    const int t = blockIdx.x * kChunk + threadIdx.x;
+    if (t < p.T) {
+        const int a = p.action[t];
+        if (a == 0)
+            for (int j = 0; j < p.k; ++j) atomicAdd(&cnt[p.exp_sel[t * p.k + j]], 1);
+        if (p.has_shared && (a == 0 || a == 1)) atomicAdd(&cnt[p.E], 1);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nb; i += blockDim.x) p.blk_counts[blockIdx.x * nb + i] = cnt[i];
+}
+
+// One block: per bucket, exclusive prefix over chunks; then bucket offsets.
+__global__ void __launch_bounds__(256) scan_kernel(const CompactParams p) {
+    __shared__ int total[kMaxE + 1];
+    const int nb = p.E + 1;
+    for (int e = threadIdx.x; e < nb; e += blockDim.x) {
+        int run = 0;
+        for (int b = 0; b < p.nblk; ++b) {
+            const int c = p.blk_counts[b * nb + e];
+            p.blk_base[b * nb + e] = run;
+            run += c;
+        }
+        total[e] = run;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int acc = 0;
+        for (int e = 0; e < nb; ++e) {
+            p.goff[e] = acc;
+            acc += total[e];
+        }
+        p.goff[nb] = acc;
+        atomicAdd(&p.ctr->pairs_total, (unsigned long long)(acc - total[p.E]));
+        atomicAdd(&p.ctr->shared_rows, (unsigned long long)total[p.E]);
+    }
+}
+
+// One warp per chunk walks the chunk's pairs in (t, j) order, 32 at a time.
+__global__ void __launch_bounds__(32) scatter_kernel(const CompactParams p) {
+    __shared__ int run[kMaxE + 1];
+    const int lane = threadIdx.x;
+    const int nb = p.E + 1;
+    for (int e = lane; e < nb; e += 32) run[e] = p.goff[e] + p.blk_base[blockIdx.x * nb + e];
+    __syncwarp();
+    const int t0 = blockIdx.x * kChunk;
+    const int tn = min(kChunk, p.T - t0);
+    const unsigned lt_mask = (1u << lane) - 1u;
+    // Routed pairs.
+    const int npairs = tn * p.k;
+    for (int q0 = 0; q0 < npairs; q0 += 32) {
+        const int q = q0 + lane;
+        int key = -1, code = -1;
+        if (q < npairs) {
+            const int t = t0 + q / p.k;
+            const int j = q - (q / p.k) * p.k;
+            code = t * p.k + j;
+            if (p.action[t] == 0) key = p.exp_sel[code];
+            else p.pos_pair[code] = -1;
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, key);
+        if (key >= 0) {
+            const int rank = __popc(peers & lt_mask);
+            const int pos = run[key] + rank;
+            p.perm[pos] = code;
+            p.pos_pair[code] = pos;
+        }
+        __syncwarp();
+        if (key >= 0 && (peers & lt_mask) == 0) run[key] += __popc(peers);
+        __syncwarp();
+    }
+    // Shared-expert rows: executed or skipped tokens, by t.
+    if (p.has_shared) {
+        for (int q0 = 0; q0 < tn; q0 += 32) {
+            const int q = q0 + lane;
+            bool take = false;
+            int t = t0 + q;
+            if (q < tn) {
+                const int a = p.action[t];
+                take = (a == 0 || a == 1);
+                if (!take) p.pos_sh[t] = -1;
+            }
+            const unsigned ball = __ballot_sync(0xffffffffu, take);
+            if (take) {
+                const int pos = run[p.E] + __popc(ball & lt_mask);
+                p.perm[pos] = t;
+                p.pos_sh[t] = pos - p.goff[p.E];
+            }
+            __syncwarp();
+            if (lane == 0) run[p.E] += __popc(ball);
+            __syncwarp();
+        }
+    }
+}
+
+// Xp[row] = h[token of row] for every compacted row; one warp per row.
+__global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__ perm,
+                                                     const int32_t* __restrict__ goff, int E, int k,
+                                                     int d, const __nv_bfloat16* __restrict__ h,
+                                                     __nv_bfloat16* __restrict__ Xp) {
+    const int nrows = goff[E + 1];
+    const int routed = goff[E];
+    const int lane = threadIdx.x & 31;
+    const int nchunk = d >> 3;
+    for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < nrows;
+         r += (gridDim.x * blockDim.x) >> 5) {
+        const int code = perm[r];
+        const int t = r < routed ? code / k : code;
+        const uint4* src = reinterpret_cast<const uint4*>(h + (size_t)t * d);
+        uint4* dst = reinterpret_cast<uint4*>(Xp + (size_t)r * d);
+        for (int c = lane; c < nchunk; c += 32) dst[c] = src[c];
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_compact(const CompactParams& p, cudaStream_t st) {
+    if (p.T <= 0) return cudaSuccess;
+    count_kernel<<<p.nblk, kChunk, 0, st>>>(p);
+    scan_kernel<<<1, 256, 0, st>>>(p);
+    scatter_kernel<<<p.nblk, 32, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
+                          const __nv_bfloat16* h, __nv_bfloat16* Xp, int max_rows, int num_sms,
+                          cudaStream_t st) {
+    if (max_rows <= 0) return cudaSuccess;
+    int blocks = (max_rows + 7) / 8;
+    blocks = blocks < num_sms * 8 ? blocks : num_sms * 8;
+    gather_kernel<<<blocks, 256, 0, st>>>(perm, goff, E, k, d, h, Xp);
+    return cudaGetLastError();
+}
+
+}  // namespace tmoe

@@ -1,0 +1,398 @@
+// Kernel (a): fused router + exit head + skip test + substitute-or-fetch with
+// server argmin and look-ahead + state update, one warp per live token.
+//
+// Paper: Sec. V, Algorithm 2 lines 7-23.  Router and importance: Eq. (4);
+// exit confidence: Eq. (7)-(9); skip admission: Eq. (5), (34), (35); per-step
+// cost: Eq. (30)-(32); look-ahead cost-to-go: Eq. (38)-(39); choice: Eq. (40);
+// updates: Eq. (41)-(42).
+//
+// Every decision quantity after the dot products is fp32 with one fixed
+// operation order written with explicit round-to-nearest intrinsics (no fused
+// multiply-add), so that the integer outcomes are reproducible bit for bit.
+// Dot products accumulate in fp32 across lanes.
+#include <float.h>
+
+#include "internal.cuh"
+
+namespace tmoe {
+
+namespace {
+
+constexpr int kWarps = 4;
+#define kInf __int_as_float(0x7f800000)
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ float warp_min(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// (value, index) argmin over the warp; ties go to the lower index.
+__device__ __forceinline__ void warp_argmin(float& v, int& i) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        float ov = __shfl_xor_sync(0xffffffffu, v, o);
+        int oi = __shfl_xor_sync(0xffffffffu, i, o);
+        if (ov < v || (ov == v && oi < i)) { v = ov; i = oi; }
+    }
+}
+// (value, index) argmax; ties go to the lower index.
+__device__ __forceinline__ void warp_argmax(float& v, int& i) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        float ov = __shfl_xor_sync(0xffffffffu, v, o);
+        int oi = __shfl_xor_sync(0xffffffffu, i, o);
+        if (ov > v || (ov == v && oi < i)) { v = ov; i = oi; }
+    }
+}
+
+__device__ __forceinline__ float dot8(const float (&h)[8], uint4 w) {
+    float a = 0.f;
+    a = fmaf(h[0], bf16_lo(w.x), a);
+    a = fmaf(h[1], bf16_hi(w.x), a);
+    a = fmaf(h[2], bf16_lo(w.y), a);
+    a = fmaf(h[3], bf16_hi(w.y), a);
+    a = fmaf(h[4], bf16_lo(w.z), a);
+    a = fmaf(h[5], bf16_hi(w.z), a);
+    a = fmaf(h[6], bf16_lo(w.w), a);
+    a = fmaf(h[7], bf16_hi(w.w), a);
+    return a;
+}
+
+// out[r] = dot(h_row, W[r]) + b[r] for r < R; lanes split d in 16-byte chunks.
+__device__ void warp_gemv(const uint4* __restrict__ hrow, const __nv_bfloat16* __restrict__ W,
+                          const float* __restrict__ b, int R, int d, int lane, float* out) {
+    const int nchunk = d >> 3;
+    for (int r0 = 0; r0 < R; r0 += 8) {
+        const int nr = min(8, R - r0);
+        float acc[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+        for (int c = lane; c < nchunk; c += 32) {
+            const uint4 hv = hrow[c];
+            const float hf[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
+                                 bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                if (i < nr) {
+                    const uint4 wv = __ldg(reinterpret_cast<const uint4*>(W + (size_t)(r0 + i) * d) + c);
+                    acc[i] += dot8(hf, wv);
+                }
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = warp_sum(acc[i]);
+        if (lane == 0)
+            for (int i = 0; i < nr; ++i) out[r0 + i] = __fadd_rn(acc[i], b[r0 + i]);
+    }
+    __syncwarp();
+}
+
+// Per-step delay (Eq. 30) and execute cost (Eq. 31) from server s to m.
+__device__ __forceinline__ float exec_cost(const DecideParams& p, int l, int s, int m, float Q,
+                                           float Dbar) {
+    const float tr = (m != s) ? p.tab.trans[s * p.M + m] : 0.f;
+    const float dly = __fadd_rn(tr, p.tab.comp[l * p.M + m]);
+    float c = __fmul_rn(p.omega_T, __fdiv_rn(dly, p.d_ref));
+    if (Q > 0.f) c = __fadd_rn(c, __fmul_rn(p.omega_D, __fdiv_rn(Q, Dbar)));
+    return c;
+}
+
+struct WarpCounters {
+    unsigned long long layer_tokens, exec_tokens, skipped, exited;
+    unsigned long long le, ls, re, rs, hops;
+    double delay;
+    float max_ratio;
+};
+
+__global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams p) {
+    extern __shared__ float smem[];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int E = p.E, M = p.M, C = p.C, K = p.k, l = p.layer;
+    const int ME = M * E;
+    // Per-warp scratch: logits z[E], probabilities pr[E], head logits x[C],
+    // look-ahead tables V[M*E] and Phi[M*E].
+    float* zs = smem + (size_t)warp * (2 * E + C + 2 * ME);
+    float* ps = zs + E;
+    float* xs = ps + E;
+    float* bufV = xs + C;
+    float* bufPhi = bufV + ME;
+
+    __shared__ unsigned long long blk_cnt[9];
+    __shared__ double blk_delay;
+    __shared__ unsigned int blk_ratio;
+    if (threadIdx.x < 9) blk_cnt[threadIdx.x] = 0ull;
+    if (threadIdx.x == 0) { blk_delay = 0.0; blk_ratio = 0u; }
+    __syncthreads();
+
+    WarpCounters wc = {};
+    const int nwarps = gridDim.x * kWarps;
+    for (int t = blockIdx.x * kWarps + warp; t < p.T; t += nwarps) {
+        if (!p.alive[t]) {
+            if (lane == 0) {
+                p.action[t] = 3;
+                p.I_out[t] = 0.f;
+                p.xi_out[t] = -1.f;
+            }
+            if (lane < K) {
+                p.topk_idx[t * K + lane] = -1;
+                p.topk_g[t * K + lane] = 0.f;
+                p.exp_sel[t * K + lane] = 0xFF;
+                p.srv_sel[t * K + lane] = 0xFF;
+            }
+            continue;
+        }
+        const int s = p.s[t];
+        const float Dhat = p.Dhat[t];
+        const float Dbar = p.Dbar[t];
+        const float pJ = p.pJ[t];
+        const int last_exec = p.last_exec[t];
+        const uint4* hrow = reinterpret_cast<const uint4*>(p.h + (size_t)t * p.d);
+
+        // Router logits, softmax (Eq. 4) and top-k by logit.
+        warp_gemv(hrow, p.W_r, p.b_r, E, p.d, lane, zs);
+        float zmax = -FLT_MAX;
+        for (int e = lane; e < E; e += 32) zmax = fmaxf(zmax, zs[e]);
+        zmax = warp_max(zmax);
+        float S = 0.f;
+        for (int e = lane; e < E; e += 32) {
+            const float ex = expf(zs[e] - zmax);
+            ps[e] = ex;
+            S += ex;
+        }
+        S = warp_sum(S);
+        __syncwarp();
+        for (int e = lane; e < E; e += 32) ps[e] = __fdiv_rn(ps[e], S);
+        __syncwarp();
+        int topk[kMaxK];
+        float g[kMaxK];
+        unsigned used = 0u;   // bit i: expert lane + 32 i taken
+        for (int j = 0; j < K; ++j) {
+            float bz = -FLT_MAX;
+            int be = 0x7fffffff;
+            for (int i = 0, e = lane; e < E; ++i, e += 32)
+                if (!((used >> i) & 1u) && (zs[e] > bz || (zs[e] == bz && e < be))) { bz = zs[e]; be = e; }
+            warp_argmax(bz, be);
+            topk[j] = be;
+            if ((be & 31) == lane) used |= 1u << (be >> 5);
+        }
+        float I = 0.f;
+        for (int j = 0; j < K; ++j) { g[j] = ps[topk[j]]; I = __fadd_rn(I, g[j]); }
+
+        // Exit confidence of the previous layer's head (Eq. 7), exit gate (Eq. 8-9).
+        float xi = -1.f;
+        const bool have_xi = (l > 0) && last_exec && (p.W_x != nullptr);
+        if (have_xi) {
+            warp_gemv(hrow, p.W_x, p.b_x, C, p.d, lane, xs);
+            if (C == 1) {
+                xi = __fdiv_rn(1.f, __fadd_rn(1.f, expf(-xs[0])));
+            } else {
+                float xm = -FLT_MAX;
+                for (int c = lane; c < C; c += 32) xm = fmaxf(xm, xs[c]);
+                xm = warp_max(xm);
+                float Sx = 0.f;
+                for (int c = lane; c < C; c += 32) Sx += expf(xs[c] - xm);
+                Sx = warp_sum(Sx);
+                xi = __fdiv_rn(1.f, Sx);
+            }
+        }
+        const bool exit_ok = have_xi && (xi >= pJ);
+
+        // Transmission necessity (Eq. 35) over the budget-feasible candidates (Eq. 34).
+        float Gamma = 0.f;
+        for (int j = 0; j < K; ++j) {
+            const int base = (l * E + topk[j]) * kMaxCand;
+            const int n = p.tab.ncand[l * E + topk[j]];
+            float gmin = kInf;
+            for (int c = lane; c < n; c += 32) {
+                const float Q = p.tab.cand_Q[base + c];
+                if (__fadd_rn(Dhat, Q) <= Dbar) {
+                    const int m = p.tab.cand_m[base + c];
+                    gmin = fminf(gmin, (m != s) ? p.tab.trans[s * M + m] : 0.f);
+                }
+            }
+            Gamma = __fadd_rn(Gamma, warp_min(gmin));
+        }
+        const float Lambda = __fmul_rn(p.tab.lambda[l], I);
+        const bool skip_ok = (Gamma > 0.f) && (I <= p.tab.theta[l]) && (__fadd_rn(Dhat, Lambda) <= Dbar);
+
+        // Look-ahead Phi^{(H-1)}_l over all (m, k), bottom-up (Eq. 39).
+        const float R = __fsub_rn(Dbar, Dhat);
+        const int top = min(p.H - 1, p.N - 1 - l);
+        bool have_phi = false;
+        for (int jj = top; jj >= 1; --jj) {
+            const int lp = l + jj;
+            const float eps = p.tab.eps[lp];
+            for (int idx = lane; idx < ME; idx += 32) {
+                const int m = idx / E, kp = idx - (idx / E) * E;
+                const int base = (lp * E + kp) * kMaxCand;
+                const int n = p.tab.ncand[lp * E + kp];
+                float best = kInf;
+                bool local = false;
+                for (int c = 0; c < n; ++c) {
+                    const float Q = p.tab.cand_Q[base + c];
+                    if (!(Q <= R)) continue;
+                    const int mm = p.tab.cand_m[base + c];
+                    float v = exec_cost(p, lp, m, mm, Q, Dbar);
+                    if (have_phi) v = __fadd_rn(v, bufPhi[mm * E + p.tab.cand_k[base + c]]);
+                    best = fminf(best, v);
+                    local |= (mm == m);
+                }
+                if (!local && eps <= R) {
+                    float v = __fmul_rn(p.omega_D, __fdiv_rn(eps, Dbar));
+                    if (have_phi) v = __fadd_rn(v, bufPhi[m * E + kp]);
+                    best = fminf(best, v);
+                }
+                bufV[idx] = best;
+            }
+            __syncwarp();
+            const float* Pl = p.tab.P + (size_t)(lp - 1) * E * E;
+            for (int idx = lane; idx < ME; idx += 32) {
+                const int m = idx / E, k = idx - (idx / E) * E;
+                const float* Prow = Pl + k * E;
+                const float* Vrow = bufV + m * E;
+                float acc = 0.f;
+                for (int kp = 0; kp < E; ++kp) acc = __fadd_rn(acc, __fmul_rn(__ldg(Prow + kp), Vrow[kp]));
+                bufPhi[idx] = acc;
+            }
+            __syncwarp();
+            have_phi = true;
+        }
+
+        // Execute plan: slot 0 by f + Phi, later slots by f (Eq. 40), budget by Eq. (34).
+        int esel[kMaxK], msel[kMaxK];
+        float Drun = Dhat, tot = 0.f;
+        for (int j = 0; j < K; ++j) {
+            const int base = (l * E + topk[j]) * kMaxCand;
+            const int n = p.tab.ncand[l * E + topk[j]];
+            float bv = kInf, bf = 0.f;
+            int bi = 0x7fffffff;
+            for (int c = lane; c < n; c += 32) {
+                const float Q = p.tab.cand_Q[base + c];
+                if (!(__fadd_rn(Dhat, Q) <= Dbar)) continue;
+                if (!(__fadd_rn(Drun, Q) <= Dbar)) continue;
+                const int m = p.tab.cand_m[base + c];
+                const float f = exec_cost(p, l, s, m, Q, Dbar);
+                float v = f;
+                if (j == 0) v = __fadd_rn(f, have_phi ? bufPhi[m * E + p.tab.cand_k[base + c]] : 0.f);
+                if (v < bv) { bv = v; bi = c; bf = f; }
+            }
+            warp_argmin(bv, bi);
+            bf = __shfl_sync(0xffffffffu, bf, bi & 31);
+            esel[j] = p.tab.cand_k[base + bi];
+            msel[j] = p.tab.cand_m[base + bi];
+            Drun = __fadd_rn(Drun, p.tab.cand_Q[base + bi]);
+            tot = (j == 0) ? bv : __fadd_rn(tot, bv);
+        }
+        const float tot_exec = tot;
+        float tot_skip = kInf;
+        if (skip_ok)
+            tot_skip = __fadd_rn(__fmul_rn(p.omega_D, __fdiv_rn(Lambda, Dbar)),
+                                 have_phi ? bufPhi[s * E + topk[0]] : 0.f);
+        int action = 0;
+        float best = tot_exec;
+        if (skip_ok && tot_skip < tot_exec) { action = 1; best = tot_skip; }
+        if (exit_ok && best > 0.f) action = 2;
+
+        // Outputs and state update (Eq. 41, 42, exit).
+        if (lane < K) {
+            p.topk_idx[t * K + lane] = topk[lane];
+            p.topk_g[t * K + lane] = g[lane];
+            p.exp_sel[t * K + lane] = action == 0 ? (uint8_t)esel[lane] : 0xFF;
+            p.srv_sel[t * K + lane] = action == 0 ? (uint8_t)msel[lane] : 0xFF;
+        }
+        if (lane == 0) {
+            p.action[t] = (uint8_t)action;
+            p.I_out[t] = I;
+            p.xi_out[t] = xi;
+            if (xi >= 0.f) p.xi_last[t] = xi;
+            float Dnew = Dhat;
+            if (action == 0) {
+                p.s[t] = (uint8_t)msel[0];
+                Dnew = Drun;
+                p.Dhat[t] = Dnew;
+                p.last_exec[t] = 1;
+                for (int j = 0; j < K; ++j) {
+                    const bool remote = msel[j] != s;
+                    const bool sub = esel[j] != topk[j];
+                    if (remote) { if (sub) ++wc.rs; else ++wc.re; ++wc.hops; }
+                    else { if (sub) ++wc.ls; else ++wc.le; }
+                    const float tr = remote ? p.tab.trans[s * M + msel[j]] : 0.f;
+                    wc.delay += (double)(tr + p.tab.comp[l * M + msel[j]]);
+                }
+                ++wc.exec_tokens;
+            } else if (action == 1) {
+                Dnew = __fadd_rn(Dhat, Lambda);
+                p.Dhat[t] = Dnew;
+                p.last_exec[t] = 0;
+                ++wc.skipped;
+            } else {
+                p.alive[t] = 0;
+                p.exit_layer[t] = (int16_t)l;
+                ++wc.exited;
+            }
+            ++wc.layer_tokens;
+            if (Dbar > 0.f && Dbar < FLT_MAX) wc.max_ratio = fmaxf(wc.max_ratio, Dnew / Dbar);
+        }
+        __syncwarp();
+    }
+    if (lane == 0) {
+        atomicAdd(&blk_cnt[0], wc.layer_tokens);
+        atomicAdd(&blk_cnt[1], wc.exec_tokens);
+        atomicAdd(&blk_cnt[2], wc.skipped);
+        atomicAdd(&blk_cnt[3], wc.exited);
+        atomicAdd(&blk_cnt[4], wc.le);
+        atomicAdd(&blk_cnt[5], wc.ls);
+        atomicAdd(&blk_cnt[6], wc.re);
+        atomicAdd(&blk_cnt[7], wc.rs);
+        atomicAdd(&blk_cnt[8], wc.hops);
+        atomicAdd(&blk_delay, wc.delay);
+        atomicMax(&blk_ratio, __float_as_uint(fmaxf(wc.max_ratio, 0.f)));
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && blk_cnt[0]) {
+        DevCounters* c = p.ctr;
+        atomicAdd(&c->layer_tokens, blk_cnt[0]);
+        atomicAdd(&c->exec_tokens, blk_cnt[1]);
+        atomicAdd(&c->skipped, blk_cnt[2]);
+        atomicAdd(&c->exited, blk_cnt[3]);
+        atomicAdd(&c->pairs_local_exact, blk_cnt[4]);
+        atomicAdd(&c->pairs_local_sub, blk_cnt[5]);
+        atomicAdd(&c->pairs_remote_exact, blk_cnt[6]);
+        atomicAdd(&c->pairs_remote_sub, blk_cnt[7]);
+        atomicAdd(&c->remote_hops, blk_cnt[8]);
+        atomicAdd(&c->delay_ms, blk_delay);
+        atomicMax(&c->max_budget_ratio_bits, blk_ratio);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
+    if (p.T <= 0) return cudaSuccess;
+    const size_t per_warp = (size_t)(2 * p.E + p.C + 2 * p.M * p.E) * sizeof(float);
+    const size_t smem = per_warp * kWarps;
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(decide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             96 * 1024);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    int blocks = (p.T + kWarps - 1) / kWarps;
+    blocks = blocks < num_sms * 16 ? blocks : num_sms * 16;
+    decide_kernel<<<blocks, kWarps * 32, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace tmoe

@@ -1,0 +1,295 @@
+// Kernel (c): grouped expert-FFN GEMM on the 5th-generation tensor cores.
+//
+// For every group g (an expert, or the shared expert) with rows
+// [goff[g], goff[g+1]) of the compacted activations A (bf16, K contiguous) and
+// that group's weights B (bf16 [N][K], K contiguous):
+//     out[row, :] = epilogue(A[row, :] . B^T)
+// with epilogue = store (down projection), SwiGLU over the interleaved
+// gate/up columns (W13 of a SwiGLU expert) or ReLU (W1 of a ReLU expert).
+// This is the only dense contraction of the layer step (the expert FFN of the
+// executed layers, Sec. III-B/C, Alg. 2 line 17).
+//
+// Design (one CTA per SM, persistent, 192 threads):
+//   warp 0      TMA producer (one lane); also owns the TMEM allocation
+//   warp 1      MMA issuer (one lane): tcgen05.mma.cta_group::1.kind::f16,
+//               M = 128, N = 256, K = 16 per instruction, fp32 accumulators in
+//               TMEM, two 256-column accumulators so the epilogue of one tile
+//               overlaps the main loop of the next
+//   warps 2-5   epilogue: tcgen05.ld 32 rows x 32 columns per warp, fused
+//               activation, bf16 stores
+// Operand tiles (A 128x64, B 256x64 per stage, 4 stages) arrive by TMA with
+// 128-byte swizzle.  Tiles are ordered expert-major, then output-column tile,
+// then row tile, so concurrent CTAs share one weight tile through L2.
+// Every mbarrier wait is bounded (2 s); on expiry the kernel records an error
+// word, stops issuing work, frees its TMEM and returns.
+#include "internal.cuh"
+
+namespace tmoe {
+
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int kThreads = 192;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr int kMaxGroups = kMaxE + 1;
+
+struct __align__(8) GemmSmemTail {
+    uint64_t full[STAGES];
+    uint64_t empty[STAGES];
+    uint64_t tfull[2];
+    uint64_t tempty[2];
+    uint32_t tmem_base;
+    int abort_flag;
+    int total_tiles;
+    int tile_start[kMaxGroups + 1];
+    int gstart[kMaxGroups];
+    int gcnt[kMaxGroups];
+};
+
+constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + sizeof(GemmSmemTail);
+
+struct Tile {
+    int rows, a_row, out_row, b_row, nt;
+};
+
+__device__ __forceinline__ Tile map_tile(const GemmSmemTail* tl, int t, int ngroups, int n_tiles_n,
+                                         int base0, int a_rebase, int out_rebase, int b_rows_per_group) {
+    int lo = 0, hi = ngroups - 1;
+    while (lo < hi) {                      // largest g with tile_start[g] <= t
+        const int mid = (lo + hi + 1) >> 1;
+        if (tl->tile_start[mid] <= t) lo = mid; else hi = mid - 1;
+    }
+    const int g = lo;
+    const int cnt = tl->gcnt[g];
+    const int mtc = (cnt + BM - 1) / BM;
+    const int u = t - tl->tile_start[g];
+    const int nt = u / mtc;
+    const int mt = u - nt * mtc;
+    Tile r;
+    r.rows = min(BM, cnt - mt * BM);
+    r.a_row = tl->gstart[g] - (a_rebase ? base0 : 0) + mt * BM;
+    r.out_row = tl->gstart[g] - (out_rebase ? base0 : 0) + mt * BM;
+    r.b_row = g * b_rows_per_group + nt * BN;
+    r.nt = nt;
+    return r;
+}
+
+__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float (&v)[32]) {
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 u;
+        u.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
+        u.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
+        u.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
+        u.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
+        d4[q] = u;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
+                    int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
+                    __nv_bfloat16* __restrict__ out, int ldo, int* err) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
+    uint8_t* smem = smem_raw + pad;
+    const uint32_t sA = smem_u32(smem);
+    const uint32_t sB = sA + STAGES * A_BYTES;
+    GemmSmemTail* tl = reinterpret_cast<GemmSmemTail*>(smem + (size_t)STAGES * STAGE_BYTES);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    // Tile table from the device-side group offsets.
+    if (threadIdx.x == 0) {
+        const int base0 = goff[first_group];
+        int acc = 0;
+        for (int g = 0; g < ngroups; ++g) {
+            const int st = goff[first_group + g];
+            const int cnt = goff[first_group + g + 1] - st;
+            tl->gstart[g] = st;
+            tl->gcnt[g] = cnt;
+            tl->tile_start[g] = acc;
+            acc += ((cnt + BM - 1) / BM) * n_tiles_n;
+        }
+        tl->tile_start[ngroups] = acc;
+        tl->total_tiles = acc;
+        tl->abort_flag = 0;
+        (void)base0;
+    }
+    __syncthreads();
+    const int total = tl->total_tiles;
+    if ((int)blockIdx.x >= total) return;
+    const int base0 = tl->gstart[0];
+    const int nkb = K / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_u32(&tl->full[s]), 1);
+            mbar_init(smem_u32(&tl->empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&tl->tfull[b]), 1);
+            mbar_init(smem_u32(&tl->tempty[b]), 4);
+        }
+        fence_barrier_init();
+        prefetch_tmap(&tmA);
+        prefetch_tmap(&tmB);
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&tl->tmem_base), TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = tl->tmem_base;
+    volatile int* abort_flag = &tl->abort_flag;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------------------------------------------- producer
+            int it = 0;
+            for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
+                const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
+                                         b_rows_per_group);
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % STAGES;
+                    const uint32_t ph = (it / STAGES) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&tl->empty[s]), ph ^ 1, abort_flag, err,
+                                           ERR_TIMEOUT_PRODUCER))
+                        break;
+                    const uint32_t fb = smem_u32(&tl->full[s]);
+                    mbar_arrive_expect_tx(fb, STAGE_BYTES);
+                    tma_load_2d(sA + s * A_BYTES, &tmA, kb * BK, ti.a_row, fb);
+                    tma_load_2d(sB + s * B_BYTES, &tmB, kb * BK, ti.b_row, fb);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---------------------------------------------------- MMA issuer
+            constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+            int it = 0, tl_i = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++tl_i) {
+                const int buf = tl_i & 1;
+                const uint32_t aph = (tl_i >> 1) & 1;
+                if (!mbar_wait_bounded(smem_u32(&tl->tempty[buf]), aph ^ 1, abort_flag, err,
+                                       ERR_TIMEOUT_MMA)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % STAGES;
+                    const uint32_t ph = (it / STAGES) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&tl->full[s]), ph, abort_flag, err, ERR_TIMEOUT_MMA)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = sA + s * A_BYTES;
+                    const uint32_t b0 = sB + s * B_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        tc_mma_bf16(d_tmem, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + kk * 32),
+                                    idesc, (kb | kk) != 0 ? 1u : 0u);
+                    tc_commit(smem_u32(&tl->empty[s]));
+                }
+                if (!ok) break;
+                tc_commit(smem_u32(&tl->tfull[buf]));
+            }
+        }
+    } else {
+        // -------------------------------------------------------- epilogue
+        const int q = warp & 3;                 // TMEM lane quarter of this warp
+        const int row = q * 32 + lane;
+        int tl_i = 0;
+        for (int t = blockIdx.x; t < total; t += gridDim.x, ++tl_i) {
+            const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
+                                     b_rows_per_group);
+            const int buf = tl_i & 1;
+            const uint32_t aph = (tl_i >> 1) & 1;
+            int ok = 1;
+            if (lane == 0)
+                ok = mbar_wait_bounded(smem_u32(&tl->tfull[buf]), aph, abort_flag, err, ERR_TIMEOUT_EPI);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            tc_fence_after();
+            const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
+            const bool valid = row < ti.rows;
+            __nv_bfloat16* orow = out + (size_t)(ti.out_row + (valid ? row : 0)) * ldo;
+            if (epi_mode == EPI_SWIGLU) {
+#pragma unroll 1
+                for (int c = 0; c < BN / 2; c += 32) {
+                    uint32_t gr[32], ur[32];
+                    tmem_ld_32x32(tb + c, gr);
+                    tmem_ld_32x32(tb + BN / 2 + c, ur);
+                    tmem_ld_wait();
+                    if (valid) {
+                        float v[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const float gt = __uint_as_float(gr[i]);
+                            const float up = __uint_as_float(ur[i]);
+                            v[i] = gt / (1.f + __expf(-gt)) * up;
+                        }
+                        store_row32(orow + ti.nt * (BN / 2) + c, v);
+                    }
+                }
+            } else {
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32(tb + c, r);
+                    tmem_ld_wait();
+                    if (valid) {
+                        float v[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const float x = __uint_as_float(r[i]);
+                            v[i] = epi_mode == EPI_RELU ? fmaxf(x, 0.f) : x;
+                        }
+                        store_row32(orow + ti.nt * BN + c, v);
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&tl->tempty[buf]));
+        }
+    }
+
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem_base, TMEM_COLS);
+    }
+}
+
+}  // namespace
+
+size_t grouped_gemm_smem_bytes() { return kSmemBytes; }
+
+cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kSmemBytes);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    if (g.ngroups <= 0 || g.ngroups > kMaxGroups || g.K % BK != 0) return cudaErrorInvalidValue;
+    grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
+        *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
+        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err);
+    return cudaGetLastError();
+}
+
+}  // namespace tmoe

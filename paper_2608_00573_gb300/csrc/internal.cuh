@@ -1,0 +1,282 @@
+// Internal declarations of the sm_103a TrimMoE library: the handle, kernel
+// parameter blocks, launchers and the inline-PTX helpers (mbarrier, TMA,
+// tcgen05) the kernels share.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/trimmoe.h"
+
+namespace tmoe {
+
+constexpr int kMaxE = 128;
+constexpr int kMaxK = 8;
+constexpr int kMaxM = 16;
+constexpr int kMaxH = 6;
+constexpr int kMaxC = 256;
+constexpr int kMaxCand = 64;        // (1 + n_sub) * M with n_sub <= 3, M <= 16
+constexpr int kMaxME = 1024;        // look-ahead table entries per token
+constexpr int kGateUp = 128;        // W13 gate/up row interleave
+
+// Device error codes (first one wins).
+enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3 };
+
+// Device-side counters (trimmoe_stats_t is assembled from these).
+struct DevCounters {
+    unsigned long long layer_tokens, exec_tokens, skipped, exited;
+    unsigned long long pairs_local_exact, pairs_local_sub, pairs_remote_exact, pairs_remote_sub;
+    unsigned long long shared_rows, remote_hops, pairs_total;
+    double delay_ms;
+    unsigned int max_budget_ratio_bits;   // non-negative float bits, atomicMax-able
+};
+
+// Per-layer decision tables on the device (built at create).
+struct DevTables {
+    const uint8_t* cand_m;   // [N][E][kMaxCand] server of candidate
+    const uint8_t* cand_k;   // [N][E][kMaxCand] expert of candidate
+    const float* cand_Q;     // [N][E][kMaxCand] substitution loss Q_l(r, k)
+    const int* ncand;        // [N][E]
+    const float* trans;      // [M][M]
+    const float* comp;       // [N][M]
+    const float* P;          // [N-1][E][E]
+    const float* theta;      // [N]
+    const float* lambda;     // [N]
+    const float* eps;        // [N]
+};
+
+struct DecideParams {
+    int layer, T, N, d, E, k, C, M, H;
+    float omega_T, omega_D, d_ref;
+    const __nv_bfloat16* h;
+    const __nv_bfloat16* W_r;   // [E][d] of this layer
+    const float* b_r;
+    const __nv_bfloat16* W_x;   // [C][d] head of layer-1, NULL at layer 0
+    const float* b_x;
+    uint8_t* s;
+    float* Dhat;
+    const float* Dbar;
+    const float* pJ;
+    uint8_t* alive;
+    uint8_t* last_exec;
+    float* xi_last;
+    int16_t* exit_layer;
+    int32_t* topk_idx;
+    float* topk_g;
+    float* I_out;
+    float* xi_out;
+    uint8_t* action;
+    uint8_t* exp_sel;
+    uint8_t* srv_sel;
+    DevTables tab;
+    DevCounters* ctr;
+};
+
+struct CompactParams {
+    int T, k, E, has_shared, nblk;
+    const uint8_t* action;
+    const uint8_t* exp_sel;
+    int32_t* blk_counts;   // [nblk][E+1]
+    int32_t* blk_base;     // [nblk][E+1]
+    int32_t* goff;         // [E+2]
+    int32_t* perm;         // [T*k + T]
+    int32_t* pos_pair;     // [T*k]
+    int32_t* pos_sh;       // [T]
+    DevCounters* ctr;
+};
+
+struct GemmLaunch {
+    const CUtensorMap* tmA;
+    const CUtensorMap* tmB;
+    const int* goff;
+    int first_group, ngroups, a_rebase, out_rebase;
+    int K, n_tiles_n, b_rows_per_group, epi_mode;
+    __nv_bfloat16* out;
+    int ldo;
+    int* err;
+};
+
+enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2 };
+
+struct CombineParams {
+    int T, d, k, renorm, has_shared;
+    __nv_bfloat16* h;
+    const uint8_t* action;
+    const float* topk_g;
+    const int32_t* pos_pair;
+    const int32_t* pos_sh;
+    const __nv_bfloat16* Y;
+    const __nv_bfloat16* Ysh;
+};
+
+// Launchers (one translation unit each).
+cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
+cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);
+cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
+                          const __nv_bfloat16* h, __nv_bfloat16* Xp, int max_rows, int num_sms,
+                          cudaStream_t st);
+cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st);
+size_t grouped_gemm_smem_bytes();
+cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
+
+// ------------------------------------------------------------------ PTX
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait: gives up after kTimeoutNs, raising the CTA abort flag and the
+// device error word; also returns early once another role has aborted.
+constexpr uint64_t kTimeoutNs = 2000000000ull;
+
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  volatile int* abort_flag, int* err, int code) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (globaltimer_ns() - t0 > kTimeoutNs) {
+            *abort_flag = 1;
+            atomicCAS(err, 0, code);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (bf16 in, fp32 accumulate).
+__device__ __forceinline__ void tc_mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive (once) on an mbarrier when all previously issued MMAs have completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+// 32 lanes x 32 consecutive 32-bit columns from TMEM into registers.
+__device__ __forceinline__ void tmem_ld_32x32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand tile written by TMA with
+// 128-byte swizzle (rows of 64 bf16, 8-row atoms 1024 bytes apart).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
+    uint64_t desc = 0;
+    desc |= (uint64_t)((addr & 0x3FFFFu) >> 4);        // start address
+    desc |= (uint64_t)(16u >> 4) << 16;                 // leading byte offset (unused here)
+    desc |= (uint64_t)(1024u >> 4) << 32;               // stride byte offset: 8 rows
+    desc |= (uint64_t)1 << 46;                          // descriptor version
+    desc |= (uint64_t)2 << 61;                          // 128-byte swizzle
+    return desc;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+    return (1u << 4)                       // D format f32
+           | (1u << 7)                     // A format bf16
+           | (1u << 10)                    // B format bf16
+           | ((uint32_t)(N >> 3) << 17)    // N / 8
+           | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+}  // namespace tmoe

@@ -1,0 +1,693 @@
+// Host runtime of the C ABI declared in include/trimmoe.h: validation, the
+// candidate lists V_{l,r} with their losses Q (Eq. 3), workspaces, TMA
+// descriptors, and the per-layer launch sequence
+//   decide -> compact -> gather -> FFN gate/up -> FFN down -> combine
+// (Alg. 2 lines 6-25 plus the MoE computation they gate).
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "internal.cuh"
+
+using namespace tmoe;
+
+namespace {
+
+std::mutex g_err_mu;
+std::string g_create_error;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*,
+                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2-D bf16 tensor [outer][inner] with a box of box_outer rows x 64 columns, 128B swizzle.
+bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint32_t box_outer) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {inner * 2};
+    cuuint32_t box[2] = {64, box_outer};
+    cuuint32_t es[2] = {1, 1};
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_NUM };
+
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+        else prev = -1;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+}  // namespace
+
+struct trimmoe {
+    trimmoe_config cfg;
+    trimmoe_weights w;
+    int dev = 0, num_sms = 0, n13 = 1;
+    std::string err;
+    cudaStream_t last_stream = nullptr;
+    std::vector<void*> allocs;
+
+    // decision tables
+    uint8_t* cand_m = nullptr;
+    uint8_t* cand_k = nullptr;
+    float* cand_Q = nullptr;
+    int* ncand = nullptr;
+    float *trans = nullptr, *comp = nullptr, *P = nullptr, *theta = nullptr, *lambda = nullptr, *eps = nullptr;
+
+    // workspaces
+    int32_t* topk_idx = nullptr;
+    float* topk_g = nullptr;
+    float* I = nullptr;
+    float* xi = nullptr;
+    uint8_t* action = nullptr;
+    uint8_t* exp_sel = nullptr;
+    uint8_t* srv_sel = nullptr;
+    int32_t *perm = nullptr, *pos_pair = nullptr, *pos_sh = nullptr, *goff = nullptr;
+    int32_t *blk_counts = nullptr, *blk_base = nullptr;
+    __nv_bfloat16 *Xp = nullptr, *act = nullptr, *act_sh = nullptr, *Y = nullptr, *Ysh = nullptr;
+    DevCounters* ctr = nullptr;
+    int* dev_err = nullptr;
+    int rows_xp = 0;
+
+    CUtensorMap tmXp, tmAct, tmActSh;
+    std::vector<CUtensorMap> tmW13, tmW2, tmW13sh, tmW2sh;
+
+    // host-buffer forward
+    trimmoe_tokens dtok = {};
+
+    // counters kept on the host
+    uint64_t launches = 0, layer_calls = 0;
+
+    // profiling
+    std::vector<cudaEvent_t> ev_free;
+    std::vector<std::pair<std::pair<cudaEvent_t, cudaEvent_t>, int>> ev_pending;
+    double ms[K_NUM] = {0};
+    uint64_t n_gemm_up = 0, n_gemm_down = 0;
+
+    trimmoe_status fail(trimmoe_status s, const std::string& m) {
+        err = m;
+        return s;
+    }
+
+    template <class T>
+    bool dalloc(T** p, size_t n) {
+        void* q = nullptr;
+        if (n == 0) n = 1;
+        if (cudaMalloc(&q, n * sizeof(T)) != cudaSuccess) {
+            cudaGetLastError();
+            return false;
+        }
+        allocs.push_back(q);
+        *p = static_cast<T*>(q);
+        return true;
+    }
+
+    cudaEvent_t get_event() {
+        if (!ev_free.empty()) {
+            cudaEvent_t e = ev_free.back();
+            ev_free.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        cudaEventCreate(&e);
+        return e;
+    }
+
+    // Launch helper: records profile events around fn() when enabled.
+    template <class Fn>
+    cudaError_t timed(int kind, cudaStream_t st, Fn fn) {
+        cudaEvent_t a = nullptr, b = nullptr;
+        if (cfg.profile) {
+            a = get_event();
+            b = get_event();
+            cudaEventRecord(a, st);
+        }
+        cudaError_t e = fn();
+        if (cfg.profile) {
+            cudaEventRecord(b, st);
+            ev_pending.push_back({{a, b}, kind});
+        }
+        return e;
+    }
+
+    void drain_events() {
+        for (auto& pe : ev_pending) {
+            float t = 0.f;
+            if (cudaEventElapsedTime(&t, pe.first.first, pe.first.second) == cudaSuccess) ms[pe.second] += t;
+            ev_free.push_back(pe.first.first);
+            ev_free.push_back(pe.first.second);
+        }
+        ev_pending.clear();
+    }
+};
+
+namespace {
+
+trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
+    if (c->N < 1 || c->d < 1 || c->E < 1 || c->k < 1 || c->F < 1 || c->M < 1 || c->H < 1 || c->C < 1 ||
+        c->T_max < 1 || c->F_sh < 0 || c->n_sub < 0) {
+        why = "config: every dimension must be positive";
+        return TRIMMOE_ERR_ARG;
+    }
+    if (c->act != 0 && c->act != 1) { why = "config: act must be 0 (ReLU) or 1 (SwiGLU)"; return TRIMMOE_ERR_ARG; }
+    if (!(c->d_ref_ms > 0.f) || !std::isfinite(c->d_ref_ms)) { why = "config: d_ref_ms must be > 0"; return TRIMMOE_ERR_ARG; }
+    if (c->d % 256) { why = "config: d must be a multiple of 256"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->act == 1 && c->F % 128) { why = "config: SwiGLU F must be a multiple of 128"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->act == 0 && c->F % 256) { why = "config: ReLU F must be a multiple of 256"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->F_sh % 128) { why = "config: F_sh must be a multiple of 128"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->E > kMaxE) { why = "config: E > 128"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->k > kMaxK || c->k > c->E) { why = "config: k must be <= min(E, 8)"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->M > kMaxM) { why = "config: M > 16"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->C > kMaxC) { why = "config: C > 256"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->M * c->E > kMaxME) { why = "config: M*E > 1024"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->H > kMaxH) { why = "config: H > 6"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->n_sub > 3) { why = "config: n_sub > 3"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if ((long long)c->T_max * (c->k + 1) >= (1ll << 31)) { why = "config: T_max too large"; return TRIMMOE_ERR_UNSUPPORTED; }
+    return TRIMMOE_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmoe_weights* w,
+                                         const trimmoe_tables* tab, trimmoe_handle* out) {
+    auto create_fail = [&](trimmoe_status s, const std::string& m) {
+        std::lock_guard<std::mutex> g(g_err_mu);
+        g_create_error = m;
+        return s;
+    };
+    if (!out) return create_fail(TRIMMOE_ERR_ARG, "create: out is NULL");
+    *out = nullptr;
+    if (!cfg || !w || !tab) return create_fail(TRIMMOE_ERR_ARG, "create: NULL argument");
+    std::string why;
+    trimmoe_status st = validate_config(cfg, why);
+    if (st != TRIMMOE_OK) return create_fail(st, why);
+    const trimmoe_config c = *cfg;
+    const int N = c.N, E = c.E, M = c.M, d = c.d;
+    const int n13 = c.act == 1 ? 2 : 1;
+    if (!w->W_r || !w->b_r || !w->W_x || !w->b_x || !w->W13 || !w->W2)
+        return create_fail(TRIMMOE_ERR_ARG, "create: NULL weight pointer");
+    if ((c.F_sh > 0) != (w->W13_sh != nullptr && w->W2_sh != nullptr))
+        return create_fail(TRIMMOE_ERR_ARG, "create: shared-expert weights must be given iff F_sh > 0");
+    if (!aligned16(w->W_r) || !aligned16(w->W_x) || !aligned16(w->W13) || !aligned16(w->W2) ||
+        (c.F_sh && (!aligned16(w->W13_sh) || !aligned16(w->W2_sh))))
+        return create_fail(TRIMMOE_ERR_ARG, "create: weights must be 16-byte aligned");
+    if (!tab->place || !tab->sim || !tab->sub_thresh || !tab->trans_ms || !tab->comp_ms || !tab->theta ||
+        !tab->lambda || !tab->eps || (N > 1 && !tab->P))
+        return create_fail(TRIMMOE_ERR_ARG, "create: NULL table pointer");
+
+    // Coverage (Eq. 2) and table sanity.
+    const uint32_t mmask = (M >= 16) ? 0xFFFFu : ((1u << M) - 1u);
+    for (int l = 0; l < N; ++l)
+        for (int e = 0; e < E; ++e)
+            if ((tab->place[l * E + e] & mmask) == 0) {
+                char b[96];
+                snprintf(b, sizeof b, "create: expert %d of layer %d has no server (Eq. 2)", e, l);
+                return create_fail(TRIMMOE_ERR_COVERAGE, b);
+            }
+    for (int i = 0; i < M * M; ++i)
+        if (!(tab->trans_ms[i] >= 0.f) || !std::isfinite(tab->trans_ms[i]))
+            return create_fail(TRIMMOE_ERR_ARG, "create: trans_ms must be finite and >= 0");
+    for (int i = 0; i < N * M; ++i)
+        if (!(tab->comp_ms[i] >= 0.f) || !std::isfinite(tab->comp_ms[i]))
+            return create_fail(TRIMMOE_ERR_ARG, "create: comp_ms must be finite and >= 0");
+    for (int l = 0; l + 1 < N; ++l)
+        for (int k = 0; k < E; ++k) {
+            double s = 0;
+            for (int kp = 0; kp < E; ++kp) {
+                const float v = tab->P[((size_t)l * E + k) * E + kp];
+                if (!(v >= 0.f) || !std::isfinite(v)) return create_fail(TRIMMOE_ERR_ARG, "create: P entries must be >= 0");
+                s += v;
+            }
+            if (std::fabs(s - 1.0) > 1e-3) return create_fail(TRIMMOE_ERR_ARG, "create: P rows must sum to 1");
+        }
+
+    trimmoe* h = new (std::nothrow) trimmoe();
+    if (!h) return create_fail(TRIMMOE_ERR_OOM, "create: host allocation failed");
+    h->cfg = c;
+    h->w = *w;
+    h->n13 = n13;
+    auto bail = [&](trimmoe_status s, const std::string& m) {
+        trimmoe_destroy(h);
+        return create_fail(s, m);
+    };
+    if (cudaGetDevice(&h->dev) != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, "create: no CUDA device");
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, h->dev) != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, "create: device query failed");
+    if (prop.major != 10) return bail(TRIMMOE_ERR_UNSUPPORTED, "create: needs a Blackwell (sm_10x) device");
+    h->num_sms = prop.multiProcessorCount;
+
+    // Candidate lists V_{l,r} (Sec. III-A): the exact expert, then the n_sub
+    // most similar experts with Sim >= sub_thresh (ties to the lower index),
+    // by expert index; servers ascending within an expert (Eq. 11).
+    std::vector<uint8_t> cm((size_t)N * E * kMaxCand, 0), ck((size_t)N * E * kMaxCand, 0);
+    std::vector<float> cq((size_t)N * E * kMaxCand, 0.f);
+    std::vector<int> nc((size_t)N * E, 0);
+    for (int l = 0; l < N; ++l)
+        for (int r = 0; r < E; ++r) {
+            const float* srow = tab->sim + ((size_t)l * E + r) * E;
+            std::vector<std::pair<float, int>> el;
+            for (int k = 0; k < E; ++k)
+                if (k != r && srow[k] >= tab->sub_thresh[l]) el.push_back({srow[k], k});
+            std::sort(el.begin(), el.end(), [](const std::pair<float, int>& a, const std::pair<float, int>& b) {
+                return a.first > b.first || (a.first == b.first && a.second < b.second);
+            });
+            std::vector<int> ex;
+            for (size_t i = 0; i < el.size() && (int)i < c.n_sub; ++i) ex.push_back(el[i].second);
+            std::sort(ex.begin(), ex.end());
+            ex.insert(ex.begin(), r);
+            int n = 0;
+            const size_t base = ((size_t)l * E + r) * kMaxCand;
+            for (int k : ex) {
+                const float q = (k == r) ? 0.0f : c.phi_beta * ((1.0f - srow[k]) / 2.0f);
+                for (int m = 0; m < M; ++m)
+                    if ((tab->place[l * E + k] >> m) & 1u) {
+                        cm[base + n] = (uint8_t)m;
+                        ck[base + n] = (uint8_t)k;
+                        cq[base + n] = q;
+                        ++n;
+                    }
+            }
+            nc[(size_t)l * E + r] = n;
+        }
+
+    // Device tables and workspaces.
+    const size_t T = (size_t)c.T_max, TK = T * c.k;
+    const int has_sh = c.F_sh > 0;
+    h->rows_xp = (int)(TK + (has_sh ? T : 0));
+    const int nblk = (int)((T + 255) / 256);
+    bool ok = h->dalloc(&h->cand_m, cm.size()) && h->dalloc(&h->cand_k, ck.size()) &&
+              h->dalloc(&h->cand_Q, cq.size()) && h->dalloc(&h->ncand, nc.size()) &&
+              h->dalloc(&h->trans, (size_t)M * M) && h->dalloc(&h->comp, (size_t)N * M) &&
+              h->dalloc(&h->P, (size_t)std::max(N - 1, 1) * E * E) && h->dalloc(&h->theta, N) &&
+              h->dalloc(&h->lambda, N) && h->dalloc(&h->eps, N) && h->dalloc(&h->topk_idx, TK) &&
+              h->dalloc(&h->topk_g, TK) && h->dalloc(&h->I, T) && h->dalloc(&h->xi, T) &&
+              h->dalloc(&h->action, T) && h->dalloc(&h->exp_sel, TK) && h->dalloc(&h->srv_sel, TK) &&
+              h->dalloc(&h->perm, TK + T) && h->dalloc(&h->pos_pair, TK) && h->dalloc(&h->pos_sh, T) &&
+              h->dalloc(&h->goff, (size_t)E + 2) && h->dalloc(&h->blk_counts, (size_t)nblk * (E + 1)) &&
+              h->dalloc(&h->blk_base, (size_t)nblk * (E + 1)) &&
+              h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
+              h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, 1) && h->dalloc(&h->dev_err, 1);
+    if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
+    if (!ok) return bail(TRIMMOE_ERR_OOM, "create: device allocation failed");
+    cudaError_t ce = cudaSuccess;
+    auto up = [&](void* dst, const void* src, size_t bytes) {
+        if (ce == cudaSuccess) ce = cudaMemcpy(dst, src, bytes, cudaMemcpyHostToDevice);
+    };
+    up(h->cand_m, cm.data(), cm.size());
+    up(h->cand_k, ck.data(), ck.size());
+    up(h->cand_Q, cq.data(), cq.size() * 4);
+    up(h->ncand, nc.data(), nc.size() * 4);
+    up(h->trans, tab->trans_ms, (size_t)M * M * 4);
+    up(h->comp, tab->comp_ms, (size_t)N * M * 4);
+    if (N > 1) up(h->P, tab->P, (size_t)(N - 1) * E * E * 4);
+    up(h->theta, tab->theta, N * 4);
+    up(h->lambda, tab->lambda, N * 4);
+    up(h->eps, tab->eps, N * 4);
+    if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters));
+    if (ce == cudaSuccess) ce = cudaMemset(h->dev_err, 0, sizeof(int));
+    if (ce == cudaSuccess) ce = cudaMemset(h->Xp, 0, (size_t)h->rows_xp * d * 2);
+    if (ce != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, std::string("create: ") + cudaGetErrorString(ce));
+
+    // TMA descriptors: activations (128-row boxes) and per-layer weights (256-row boxes).
+    const size_t F13 = (size_t)n13 * c.F;
+    bool tm = make_tmap(&h->tmXp, h->Xp, d, h->rows_xp, 128) && make_tmap(&h->tmAct, h->act, c.F, TK, 128);
+    if (has_sh) tm = tm && make_tmap(&h->tmActSh, h->act_sh, c.F_sh, T, 128);
+    h->tmW13.resize(N);
+    h->tmW2.resize(N);
+    if (has_sh) { h->tmW13sh.resize(N); h->tmW2sh.resize(N); }
+    const __nv_bfloat16* W13 = static_cast<const __nv_bfloat16*>(w->W13);
+    const __nv_bfloat16* W2 = static_cast<const __nv_bfloat16*>(w->W2);
+    for (int l = 0; l < N && tm; ++l) {
+        tm = make_tmap(&h->tmW13[l], W13 + (size_t)l * E * F13 * d, d, (uint64_t)E * F13, 256) &&
+             make_tmap(&h->tmW2[l], W2 + (size_t)l * E * d * c.F, c.F, (uint64_t)E * d, 256);
+        if (tm && has_sh) {
+            const __nv_bfloat16* W13s = static_cast<const __nv_bfloat16*>(w->W13_sh);
+            const __nv_bfloat16* W2s = static_cast<const __nv_bfloat16*>(w->W2_sh);
+            tm = make_tmap(&h->tmW13sh[l], W13s + (size_t)l * 2 * c.F_sh * d, d, (uint64_t)2 * c.F_sh, 256) &&
+                 make_tmap(&h->tmW2sh[l], W2s + (size_t)l * d * c.F_sh, c.F_sh, (uint64_t)d, 256);
+        }
+    }
+    if (!tm) return bail(TRIMMOE_ERR_CUDA, "create: cuTensorMapEncodeTiled failed");
+    *out = h;
+    return TRIMMOE_OK;
+}
+
+static trimmoe_status check_tokens(trimmoe_handle h, const trimmoe_tokens* tok) {
+    if (!tok || !tok->hidden || !tok->s || !tok->Dhat || !tok->Dbar || !tok->pJ || !tok->alive ||
+        !tok->last_exec || !tok->xi_last || !tok->exit_layer)
+        return h->fail(TRIMMOE_ERR_ARG, "tokens: NULL pointer");
+    if (!aligned16(tok->hidden)) return h->fail(TRIMMOE_ERR_ARG, "tokens: hidden must be 16-byte aligned");
+    return TRIMMOE_OK;
+}
+
+static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmoe_tokens* tok,
+                                      trimmoe_layer_out* out, cudaStream_t st) {
+    const trimmoe_config& c = h->cfg;
+    const int E = c.E, K = c.k, d = c.d;
+    const int has_sh = c.F_sh > 0;
+    const size_t F13 = (size_t)h->n13 * c.F;
+
+    DecideParams dp;
+    dp.layer = layer;
+    dp.T = T;
+    dp.N = c.N;
+    dp.d = d;
+    dp.E = E;
+    dp.k = K;
+    dp.C = c.C;
+    dp.M = c.M;
+    dp.H = c.H;
+    dp.omega_T = c.omega_T;
+    dp.omega_D = c.omega_D;
+    dp.d_ref = c.d_ref_ms;
+    dp.h = static_cast<const __nv_bfloat16*>(tok->hidden);
+    dp.W_r = static_cast<const __nv_bfloat16*>(h->w.W_r) + (size_t)layer * E * d;
+    dp.b_r = h->w.b_r + (size_t)layer * E;
+    dp.W_x = layer > 0 ? static_cast<const __nv_bfloat16*>(h->w.W_x) + (size_t)(layer - 1) * c.C * d : nullptr;
+    dp.b_x = layer > 0 ? h->w.b_x + (size_t)(layer - 1) * c.C : nullptr;
+    dp.s = tok->s;
+    dp.Dhat = tok->Dhat;
+    dp.Dbar = tok->Dbar;
+    dp.pJ = tok->pJ;
+    dp.alive = tok->alive;
+    dp.last_exec = tok->last_exec;
+    dp.xi_last = tok->xi_last;
+    dp.exit_layer = tok->exit_layer;
+    dp.topk_idx = (out && out->topk_idx) ? out->topk_idx : h->topk_idx;
+    dp.topk_g = (out && out->topk_g) ? out->topk_g : h->topk_g;
+    dp.I_out = (out && out->I) ? out->I : h->I;
+    dp.xi_out = (out && out->xi) ? out->xi : h->xi;
+    dp.action = (out && out->action) ? out->action : h->action;
+    dp.exp_sel = (out && out->exp_sel) ? out->exp_sel : h->exp_sel;
+    dp.srv_sel = (out && out->srv_sel) ? out->srv_sel : h->srv_sel;
+    dp.tab.cand_m = h->cand_m;
+    dp.tab.cand_k = h->cand_k;
+    dp.tab.cand_Q = h->cand_Q;
+    dp.tab.ncand = h->ncand;
+    dp.tab.trans = h->trans;
+    dp.tab.comp = h->comp;
+    dp.tab.P = h->P;
+    dp.tab.theta = h->theta;
+    dp.tab.lambda = h->lambda;
+    dp.tab.eps = h->eps;
+    dp.ctr = h->ctr;
+
+    cudaError_t e = h->timed(K_DECIDE, st, [&] { return launch_decide(dp, h->num_sms, st); });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("decide: ") + cudaGetErrorString(e));
+
+    CompactParams cp;
+    cp.T = T;
+    cp.k = K;
+    cp.E = E;
+    cp.has_shared = has_sh;
+    cp.nblk = (T + 255) / 256;
+    cp.action = dp.action;
+    cp.exp_sel = dp.exp_sel;
+    cp.blk_counts = h->blk_counts;
+    cp.blk_base = h->blk_base;
+    cp.goff = h->goff;
+    cp.perm = h->perm;
+    cp.pos_pair = h->pos_pair;
+    cp.pos_sh = h->pos_sh;
+    cp.ctr = h->ctr;
+    e = h->timed(K_COMPACT, st, [&] { return launch_compact(cp, st); });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("compact: ") + cudaGetErrorString(e));
+    const int max_rows = T * K + (has_sh ? T : 0);
+    e = h->timed(K_GATHER, st, [&] {
+        return launch_gather(h->perm, h->goff, E, K, d, dp.h, h->Xp, max_rows, h->num_sms, st);
+    });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gather: ") + cudaGetErrorString(e));
+
+    GemmLaunch g1;
+    g1.tmA = &h->tmXp;
+    g1.tmB = &h->tmW13[layer];
+    g1.goff = h->goff;
+    g1.first_group = 0;
+    g1.ngroups = E;
+    g1.a_rebase = 0;
+    g1.out_rebase = 0;
+    g1.K = d;
+    g1.n_tiles_n = (int)(F13 / 256);
+    g1.b_rows_per_group = (int)F13;
+    g1.epi_mode = c.act == 1 ? EPI_SWIGLU : EPI_RELU;
+    g1.out = h->act;
+    g1.ldo = c.F;
+    g1.err = h->dev_err;
+    e = h->timed(K_GEMM_UP, st, [&] { return launch_grouped_gemm(g1, h->num_sms, st); });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm up: ") + cudaGetErrorString(e));
+    GemmLaunch g2 = g1;
+    g2.tmA = &h->tmAct;
+    g2.tmB = &h->tmW2[layer];
+    g2.K = c.F;
+    g2.n_tiles_n = d / 256;
+    g2.b_rows_per_group = d;
+    g2.epi_mode = EPI_STORE;
+    g2.out = h->Y;
+    g2.ldo = d;
+    e = h->timed(K_GEMM_DOWN, st, [&] { return launch_grouped_gemm(g2, h->num_sms, st); });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm down: ") + cudaGetErrorString(e));
+    h->n_gemm_up++;
+    h->n_gemm_down++;
+    h->launches += 7;
+    if (has_sh) {
+        GemmLaunch s1 = g1;
+        s1.tmB = &h->tmW13sh[layer];
+        s1.first_group = E;
+        s1.ngroups = 1;
+        s1.out_rebase = 1;
+        s1.n_tiles_n = 2 * c.F_sh / 256;
+        s1.b_rows_per_group = 2 * c.F_sh;
+        s1.epi_mode = EPI_SWIGLU;
+        s1.out = h->act_sh;
+        s1.ldo = c.F_sh;
+        e = h->timed(K_GEMM_UP, st, [&] { return launch_grouped_gemm(s1, h->num_sms, st); });
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("shared gemm up: ") + cudaGetErrorString(e));
+        GemmLaunch s2 = s1;
+        s2.tmA = &h->tmActSh;
+        s2.tmB = &h->tmW2sh[layer];
+        s2.a_rebase = 1;
+        s2.K = c.F_sh;
+        s2.n_tiles_n = d / 256;
+        s2.b_rows_per_group = d;
+        s2.epi_mode = EPI_STORE;
+        s2.out = h->Ysh;
+        s2.ldo = d;
+        e = h->timed(K_GEMM_DOWN, st, [&] { return launch_grouped_gemm(s2, h->num_sms, st); });
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("shared gemm down: ") + cudaGetErrorString(e));
+        h->n_gemm_up++;
+        h->n_gemm_down++;
+        h->launches += 2;
+    }
+
+    CombineParams bp;
+    bp.T = T;
+    bp.d = d;
+    bp.k = K;
+    bp.renorm = c.renorm_topk;
+    bp.has_shared = has_sh;
+    bp.h = static_cast<__nv_bfloat16*>(tok->hidden);
+    bp.action = dp.action;
+    bp.topk_g = dp.topk_g;
+    bp.pos_pair = h->pos_pair;
+    bp.pos_sh = h->pos_sh;
+    bp.Y = h->Y;
+    bp.Ysh = h->Ysh;
+    e = h->timed(K_COMBINE, st, [&] { return launch_combine(bp, h->num_sms, st); });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("combine: ") + cudaGetErrorString(e));
+    h->launches += 1;
+
+    if (out && out->perm) {
+        e = cudaMemcpyAsync(out->perm, h->perm, ((size_t)T * K + T) * 4, cudaMemcpyDeviceToDevice, st);
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "copy perm failed");
+    }
+    if (out && out->group_off) {
+        e = cudaMemcpyAsync(out->group_off, h->goff, (size_t)(E + 2) * 4, cudaMemcpyDeviceToDevice, st);
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "copy group_off failed");
+    }
+    h->layer_calls++;
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T, trimmoe_tokens* tok,
+                                             trimmoe_layer_out* out, void* stream) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    if (layer < 0 || layer >= h->cfg.N) return h->fail(TRIMMOE_ERR_ARG, "layer_step: layer out of range");
+    if (T < 0 || T > h->cfg.T_max) return h->fail(TRIMMOE_ERR_ARG, "layer_step: T outside [0, T_max]");
+    trimmoe_status s = check_tokens(h, tok);
+    if (s != TRIMMOE_OK) return s;
+    DeviceGuard g(h->dev);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    h->last_stream = st;
+    if (T == 0) return TRIMMOE_OK;
+    return layer_step_impl(h, layer, T, tok, out, st);
+}
+
+extern "C" trimmoe_status trimmoe_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    if (T < 0 || T > h->cfg.T_max) return h->fail(TRIMMOE_ERR_ARG, "forward: T outside [0, T_max]");
+    trimmoe_status s = check_tokens(h, tok);
+    if (s != TRIMMOE_OK) return s;
+    DeviceGuard g(h->dev);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    h->last_stream = st;
+    if (T == 0) return TRIMMOE_OK;
+    for (int l = 0; l < h->cfg.N; ++l) {
+        s = layer_step_impl(h, l, T, tok, nullptr, st);
+        if (s != TRIMMOE_OK) return s;
+    }
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_forward_host(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    if (T < 0 || T > h->cfg.T_max) return h->fail(TRIMMOE_ERR_ARG, "forward_host: T outside [0, T_max]");
+    if (!tok || !tok->hidden || !tok->s || !tok->Dhat || !tok->Dbar || !tok->pJ || !tok->alive ||
+        !tok->last_exec || !tok->xi_last || !tok->exit_layer)
+        return h->fail(TRIMMOE_ERR_ARG, "forward_host: NULL pointer");
+    DeviceGuard g(h->dev);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    h->last_stream = st;
+    const size_t Tm = h->cfg.T_max;
+    trimmoe_tokens& dt = h->dtok;
+    if (!dt.hidden) {
+        __nv_bfloat16* hid = nullptr;
+        bool ok = h->dalloc(&hid, Tm * h->cfg.d) && h->dalloc(&dt.s, Tm) && h->dalloc(&dt.Dhat, Tm) &&
+                  h->dalloc(&dt.Dbar, Tm) && h->dalloc(&dt.pJ, Tm) && h->dalloc(&dt.alive, Tm) &&
+                  h->dalloc(&dt.last_exec, Tm) && h->dalloc(&dt.xi_last, Tm) && h->dalloc(&dt.exit_layer, Tm);
+        dt.hidden = hid;
+        if (!ok) {
+            dt.hidden = nullptr;
+            return h->fail(TRIMMOE_ERR_OOM, "forward_host: device allocation failed");
+        }
+    }
+    const size_t n = (size_t)T;
+    struct Cp { void* dst; const void* src; size_t bytes; };
+    const Cp in[] = {{dt.hidden, tok->hidden, n * h->cfg.d * 2}, {dt.s, tok->s, n}, {dt.Dhat, tok->Dhat, n * 4},
+                     {dt.Dbar, tok->Dbar, n * 4}, {dt.pJ, tok->pJ, n * 4}, {dt.alive, tok->alive, n},
+                     {dt.last_exec, tok->last_exec, n}, {dt.xi_last, tok->xi_last, n * 4},
+                     {dt.exit_layer, tok->exit_layer, n * 2}};
+    for (const Cp& c : in)
+        if (cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
+            return h->fail(TRIMMOE_ERR_CUDA, "forward_host: host-to-device copy failed");
+    for (int l = 0; l < h->cfg.N && T > 0; ++l) {
+        trimmoe_status s = layer_step_impl(h, l, T, &dt, nullptr, st);
+        if (s != TRIMMOE_OK) return s;
+    }
+    for (const Cp& c : in)
+        if (cudaMemcpyAsync(const_cast<void*>(c.src), c.dst, c.bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+            return h->fail(TRIMMOE_ERR_CUDA, "forward_host: device-to-host copy failed");
+    if (cudaStreamSynchronize(st) != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "forward_host: sync failed");
+    int derr = 0;
+    cudaMemcpy(&derr, h->dev_err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "forward_host: a kernel timed out waiting");
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) {
+    if (!h || !out) return TRIMMOE_ERR_ARG;
+    DeviceGuard g(h->dev);
+    if (cudaStreamSynchronize(h->last_stream) != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, std::string("stats: ") + cudaGetErrorString(cudaGetLastError()));
+    DevCounters dc;
+    int derr = 0;
+    if (cudaMemcpy(&dc, h->ctr, sizeof dc, cudaMemcpyDeviceToHost) != cudaSuccess ||
+        cudaMemcpy(&derr, h->dev_err, sizeof derr, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, "stats: copy failed");
+    h->drain_events();
+    const trimmoe_config& c = h->cfg;
+    std::memset(out, 0, sizeof *out);
+    out->layer_tokens = dc.layer_tokens;
+    out->exec_tokens = dc.exec_tokens;
+    out->skipped = dc.skipped;
+    out->exited = dc.exited;
+    out->pairs_local_exact = dc.pairs_local_exact;
+    out->pairs_local_sub = dc.pairs_local_sub;
+    out->pairs_remote_exact = dc.pairs_remote_exact;
+    out->pairs_remote_sub = dc.pairs_remote_sub;
+    out->shared_rows = dc.shared_rows;
+    out->delay_ms = dc.delay_ms;
+    out->remote_hops = (double)dc.remote_hops;
+    float r;
+    std::memcpy(&r, &dc.max_budget_ratio_bits, 4);
+    out->max_budget_ratio = r;
+    out->device_error = derr;
+    out->launches = h->launches;
+    out->layer_calls = h->layer_calls;
+    const double n13F = (double)h->n13 * c.F;
+    out->flops_gemm_up = 2.0 * dc.pairs_total * n13F * c.d + 2.0 * dc.shared_rows * 2.0 * c.F_sh * c.d;
+    out->flops_gemm_down = 2.0 * dc.pairs_total * (double)c.d * c.F + 2.0 * dc.shared_rows * (double)c.d * c.F_sh;
+    out->gemm_flops = out->flops_gemm_up + out->flops_gemm_down;
+    out->ms_decide = h->ms[K_DECIDE];
+    out->ms_compact = h->ms[K_COMPACT];
+    out->ms_gather = h->ms[K_GATHER];
+    out->ms_gemm_up = h->ms[K_GEMM_UP];
+    out->ms_gemm_down = h->ms[K_GEMM_DOWN];
+    out->ms_combine = h->ms[K_COMBINE];
+    out->n_gemm_up = h->n_gemm_up;
+    out->n_gemm_down = h->n_gemm_down;
+    if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "stats: a kernel timed out waiting");
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    DeviceGuard g(h->dev);
+    if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "reset: sync failed");
+    h->drain_events();
+    if (cudaMemset(h->ctr, 0, sizeof(DevCounters)) != cudaSuccess ||
+        cudaMemset(h->dev_err, 0, sizeof(int)) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, "reset: memset failed");
+    for (double& m : h->ms) m = 0.0;
+    h->launches = h->layer_calls = h->n_gemm_up = h->n_gemm_down = 0;
+    return TRIMMOE_OK;
+}
+
+extern "C" const char* trimmoe_last_error(trimmoe_handle h) {
+    if (!h) {
+        std::lock_guard<std::mutex> g(g_err_mu);
+        return g_create_error.c_str();
+    }
+    return h->err.c_str();
+}
+
+extern "C" void trimmoe_destroy(trimmoe_handle h) {
+    if (!h) return;
+    DeviceGuard g(h->dev);
+    cudaDeviceSynchronize();
+    h->drain_events();
+    for (cudaEvent_t e : h->ev_free) cudaEventDestroy(e);
+    for (void* p : h->allocs) cudaFree(p);
+    delete h;
+}

@@ -1,0 +1,210 @@
+"""GPU parity: the CUDA library (through the C ABI) against the CPU oracle.
+
+Small configurations run every layer teacher-forced with every row checked;
+the model-sized configurations check every decision and a seeded sample of
+hidden rows at the sizes and launch configuration the benchmark uses.
+"""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2608_00573_gb300 import binding as B
+from paper_2608_00573_gb300 import workload as W
+from tests.gpu_helpers import compare_layer, make_engine
+from tests.oracle_helpers import small_cfg
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="session", autouse=True)
+def built_library():
+    from paper_2608_00573_gb300 import build
+    build.build()
+    B.lib()
+
+
+def _run_all_layers(cfg, T=None, mutate_tokens=None, layers=None, row_sample=None):
+    import torch
+    eng, om, tables, small, experts = make_engine(cfg, T_max=T or cfg.T)
+    tok = W.make_tokens(cfg, T=T)
+    if mutate_tokens:
+        mutate_tokens(tok)
+    dev = eng.tokens_to_device(tok)
+    reports = []
+    for l in (layers if layers is not None else range(cfg.N)):
+        reports.append(compare_layer(cfg, om, eng, l, dev, experts, row_sample=row_sample))
+    eng.close()
+    torch.cuda.synchronize()
+    return reports
+
+
+SMALL = {
+    "switch_tiny": W.CONFIGS["switch_tiny"],
+    "swiglu_shared_k4": small_cfg(name="s1", N=3, d=512, E=16, k=4, F=384, F_sh=256, T=1000, M=10,
+                                  H=3, zipf_s=0.8, seed=21),
+    "swiglu_k2_renorm_h2": small_cfg(name="s2", N=4, d=256, E=8, k=2, F=256, T=333, M=10, H=2,
+                                     renorm_topk=1, seed=22),
+    "relu_k1_c64": small_cfg(name="s3", N=3, d=768, E=8, k=1, F=512, C=64, act=W.ACT_RELU, T=200,
+                             M=10, seed=23),
+    "e60_k4_h3": small_cfg(name="s4", N=4, d=256, E=60, k=4, F=128, F_sh=128, T=300, M=10, H=3,
+                           zipf_s=1.0, seed=24),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_layer_parity_small(name):
+    cfg = SMALL[name]
+    reports = _run_all_layers(cfg)
+    tot = {k: sum(r[k] for r in reports) for k in ("exec", "skip", "exit", "near_mismatch")}
+    print(name, tot, [round(r["max_rel_err"], 5) for r in reports])
+    assert tot["exec"] > 0
+
+
+def test_tiny_free_running_forward_matches_oracle():
+    """switch_tiny end to end without teacher forcing."""
+    import torch
+    cfg = W.CONFIGS["switch_tiny"]
+    eng, om, tables, small, experts = make_engine(cfg)
+    tok = W.make_tokens(cfg)
+    dev = eng.tokens_to_device(tok)
+    eng.forward(dev)
+    torch.cuda.synchronize()
+    got = B.Engine.tokens_to_host(dev)
+    h0 = tok.pop("h")
+    h_or, tok_or = O.forward(om, h0, tok)
+    for k in ("s", "alive", "exit_layer", "last_exec"):
+        assert np.array_equal(got[k], tok_or[k]), k
+    assert np.array_equal(got["Dhat"], tok_or["Dhat"]) or np.abs(got["Dhat"] - tok_or["Dhat"]).max() < 1e-6
+    hg = W.bf16_bits_to_f32(got["h"]).astype(np.float64)
+    ho = W.bf16_bits_to_f32(h_or).astype(np.float64)
+    err = np.abs(hg - ho).max(axis=1) / np.abs(ho).max(axis=1)
+    assert err.max() <= 2e-2
+    eng.close()
+
+
+def test_edge_cases_empty_single_and_dead():
+    import torch
+    cfg = SMALL["swiglu_shared_k4"]
+    eng, om, tables, small, experts = make_engine(cfg, T_max=1000)
+    # T = 0: a no-op
+    tok = W.make_tokens(cfg, T=1000)
+    dev = eng.tokens_to_device(tok)
+    h_before = dev["hidden"].clone()
+    eng.layer_step(0, dev, T=0)
+    torch.cuda.synchronize()
+    assert torch.equal(h_before, dev["hidden"])
+    # T = 1
+    tok1 = W.make_tokens(cfg, T=1)
+    r = compare_layer(cfg, om, eng, 0, eng.tokens_to_device(tok1), experts)
+    assert r["live"] == 1
+    # all tokens dead: nothing changes
+    tokd = W.make_tokens(cfg, T=257)
+    tokd["alive"][:] = 0
+    devd = eng.tokens_to_device(tokd)
+    r = compare_layer(cfg, om, eng, 1, devd, experts)
+    assert r["dead"] == 257
+    # exited mid-way: every other token dead, layer > 0 with last_exec set
+    tokh = W.make_tokens(cfg, T=999)
+    tokh["alive"][::2] = 0
+    tokh["last_exec"][:] = 1
+    r = compare_layer(cfg, om, eng, 2, eng.tokens_to_device(tokh), experts)
+    assert r["dead"] == 500
+    eng.close()
+
+
+@pytest.mark.parametrize("shared", [0, 256])
+def test_all_tokens_skip(shared):
+    """Every token sits on a server without any candidate, importance always
+    under theta and a near-free skip: the whole layer is skipped."""
+    cfg = small_cfg(name="skipall", N=2, d=256, E=8, k=2, F=256, F_sh=shared, T=300, M=4, H=1,
+                    n_sub=0, seed=31)
+    import torch
+    small = W.make_small_weights(cfg)
+    tables = W.make_tables(cfg, small["W_r"])
+    tables["place"][:] = np.uint16(0b1110)          # nothing on server 0
+    tables["theta"][:] = 1.0
+    tables["lam"][:] = 1e-6
+    experts = W.make_expert_weights_host(cfg)
+    eng = B.Engine(cfg, tables, small, experts, T_max=cfg.T)
+    om = O.OracleModel(cfg, tables, small, experts)
+    tok = W.make_tokens(cfg)
+    tok["s"][:] = 0
+    r = compare_layer(cfg, om, eng, 0, eng.tokens_to_device(tok), experts)
+    assert r["skip"] == cfg.T
+    eng.close()
+    torch.cuda.synchronize()
+
+
+def test_empty_experts_and_concentrated_routing():
+    """Strong router bias: most experts receive no pair (empty groups in the GEMM)."""
+    cfg = small_cfg(name="skew", N=2, d=256, E=16, k=2, F=256, T=500, M=10, zipf_s=6.0, seed=41)
+    reports = _run_all_layers(cfg)
+    assert all(r["exec"] > 0 for r in reports)
+
+
+def test_forward_host_equals_device_forward():
+    import torch
+    cfg = SMALL["swiglu_shared_k4"]
+    eng, om, tables, small, experts = make_engine(cfg, T_max=1000)
+    tok = W.make_tokens(cfg, T=1000)
+    dev = eng.tokens_to_device(tok)
+    eng.forward(dev)
+    torch.cuda.synchronize()
+    want = B.Engine.tokens_to_host(dev)
+    host = {k: v.cpu().pin_memory() for k, v in eng.tokens_to_device(tok).items()}
+    eng.forward_host(host)
+    got = B.Engine.tokens_to_host(host)
+    for k in want:
+        assert np.array_equal(want[k], got[k]), k
+    st = eng.stats()
+    assert st["status"] == 0 and st["device_error"] == 0
+    assert st["exec_tokens"] + st["skipped"] + st["exited"] == st["layer_tokens"]
+    eng.close()
+
+
+def test_stats_counters_consistent():
+    import torch
+    cfg = SMALL["swiglu_k2_renorm_h2"]
+    eng, om, tables, small, experts = make_engine(cfg, profile=True)
+    tok = W.make_tokens(cfg)
+    dev = eng.tokens_to_device(tok)
+    eng.reset_stats()
+    eng.forward(dev)
+    st = eng.stats()
+    assert st["status"] == 0
+    pairs = st["pairs_local_exact"] + st["pairs_local_sub"] + st["pairs_remote_exact"] + st["pairs_remote_sub"]
+    assert pairs == st["exec_tokens"] * cfg.k
+    assert st["exec_tokens"] + st["skipped"] + st["exited"] == st["layer_tokens"]
+    assert st["max_budget_ratio"] <= 1.0
+    assert st["layer_calls"] == cfg.N and st["ms_gemm_up"] > 0
+    host = B.Engine.tokens_to_host(dev)
+    assert int((host["alive"] == 0).sum()) == st["exited"]
+    eng.close()
+
+
+def test_create_rejects_bad_input():
+    cfg = SMALL["swiglu_k2_renorm_h2"]
+    small = W.make_small_weights(cfg)
+    tables = W.make_tables(cfg, small["W_r"])
+    experts = W.make_expert_weights_host(cfg)
+    bad = dict(tables)
+    bad["place"] = tables["place"].copy()
+    bad["place"][1, 3] = 0
+    with pytest.raises(B.TrimmoeError) as ei:
+        B.Engine(cfg, bad, small, experts, T_max=16)
+    assert ei.value.status == -5
+    with pytest.raises(B.TrimmoeError) as ei:
+        B.Engine(cfg.replace(d=200), tables, small, experts, T_max=16)
+    assert ei.value.status == -2
+    bad = dict(tables)
+    bad["P"] = tables["P"] * 2
+    with pytest.raises(B.TrimmoeError) as ei:
+        B.Engine(cfg, bad, small, experts, T_max=16)
+    assert ei.value.status == -1
+    eng = B.Engine(cfg, tables, small, experts, T_max=16)
+    tok = eng.tokens_to_device(W.make_tokens(cfg, T=16))
+    with pytest.raises(B.TrimmoeError):
+        eng.layer_step(cfg.N, tok)
+    with pytest.raises(B.TrimmoeError):
+        eng.layer_step(0, tok, T=17)
+    eng.close()
