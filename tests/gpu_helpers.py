@@ -25,13 +25,17 @@ HIDDEN_TOL = 2e-2
 NEAR_SHARE = 1e-3
 
 
-def make_engine(cfg, T_max=None, device_experts=False, profile=False):
-    small = W.make_small_weights(cfg)
-    tables = W.make_tables(cfg, small["W_r"])
-    if device_experts:
-        experts = W.make_expert_weights_device(cfg)
+def make_engine(cfg, T_max=None, device_experts=False, profile=False, theta=None, exit_bias=None,
+                experts=None):
+    """Engine + oracle on the seeded workload; theta / exit_bias override the
+    calibrated skip thresholds and exit-head biases (every layer)."""
+    small = W.make_small_weights(cfg, calib="auto" if exit_bias is None else {"exit_bias": [exit_bias] * cfg.N})
+    tables = W.make_tables(cfg, small["W_r"], calib="auto" if theta is None else {"theta": [theta] * cfg.N})
+    if experts is None:
+        experts = W.make_expert_weights_device(cfg) if device_experts else W.make_expert_weights_host(cfg)
+        device_experts = device_experts
     else:
-        experts = W.make_expert_weights_host(cfg)
+        device_experts = True
     eng = B.Engine(cfg, tables, small, experts, T_max=T_max or cfg.T, profile=profile)
     om = O.OracleModel(cfg, tables, small, None if device_experts else experts)
     return eng, om, tables, small, experts

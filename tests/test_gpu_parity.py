@@ -23,9 +23,10 @@ def built_library():
     B.lib()
 
 
-def _run_all_layers(cfg, T=None, mutate_tokens=None, layers=None, row_sample=None):
+def _run_all_layers(cfg, T=None, mutate_tokens=None, layers=None, row_sample=None, theta=None,
+                    exit_bias=None):
     import torch
-    eng, om, tables, small, experts = make_engine(cfg, T_max=T or cfg.T)
+    eng, om, tables, small, experts = make_engine(cfg, T_max=T or cfg.T, theta=theta, exit_bias=exit_bias)
     tok = W.make_tokens(cfg, T=T)
     if mutate_tokens:
         mutate_tokens(tok)
@@ -38,6 +39,7 @@ def _run_all_layers(cfg, T=None, mutate_tokens=None, layers=None, row_sample=Non
     return reports
 
 
+# (config, theta, exit-head bias): thresholds chosen so every action occurs.
 SMALL = {
     "switch_tiny": W.CONFIGS["switch_tiny"],
     "swiglu_shared_k4": small_cfg(name="s1", N=3, d=512, E=16, k=4, F=384, F_sh=256, T=1000, M=10,
@@ -51,13 +53,20 @@ SMALL = {
 }
 
 
+KNOBS = {"switch_tiny": (None, None), "swiglu_shared_k4": (0.9, 1.0), "swiglu_k2_renorm_h2": (0.9, 1.0),
+         "relu_k1_c64": (0.9, 5.0), "e60_k4_h3": (0.6, 1.0)}
+
+
 @pytest.mark.parametrize("name", list(SMALL))
 def test_layer_parity_small(name):
     cfg = SMALL[name]
-    reports = _run_all_layers(cfg)
+    theta, bias = KNOBS[name]
+    reports = _run_all_layers(cfg, theta=theta, exit_bias=bias)
     tot = {k: sum(r[k] for r in reports) for k in ("exec", "skip", "exit", "near_mismatch")}
     print(name, tot, [round(r["max_rel_err"], 5) for r in reports])
     assert tot["exec"] > 0
+    if name != "switch_tiny":
+        assert tot["skip"] > 0 and tot["exit"] > 0, tot
 
 
 def test_tiny_free_running_forward_matches_oracle():
