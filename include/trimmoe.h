@@ -61,7 +61,8 @@ enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
  *  omega_T, omega_D: weights of Eq. (21)/(31); d_ref_ms: d^ref of Eq. (31);
  *  phi_beta: Q = phi_beta * (1 - Sim)/2 (Eq. 3 with a linear phi);
  *  profile: 1 = record CUDA events around each kernel launch (trimmoe_stats
- *  then reports per-kernel device time).
+ *  then reports per-kernel device time);
+ *  norm_eps: epsilon of the pre-FFN RMSNorm (used when W_norm != NULL).
  * Supported: d % 256 == 0; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
  * F_sh % 128 == 0; E <= 128; k <= min(E, 8); C <= 256; M*E <= 1024; H <= 6;
  * n_sub <= 3. */
@@ -73,6 +74,7 @@ typedef struct {
     int T_max;
     float omega_T, omega_D, d_ref_ms, phi_beta;
     int profile;
+    float norm_eps;
 } trimmoe_config;
 
 /* Weights (device, bf16 except the biases, borrowed; 16-byte aligned).
@@ -82,7 +84,11 @@ typedef struct {
  *       interleaved in blocks of 128: rows [256b, 256b+128) are gate rows
  *       128b..128b+127 and rows [256b+128, 256b+256) the matching up rows.
  *  W2   [N][E][d][F]
- *  W13_sh [N][2*F_sh][d] (same interleave), W2_sh [N][d][F_sh]; NULL if F_sh == 0. */
+ *  W13_sh [N][2*F_sh][d] (same interleave), W2_sh [N][d][F_sh]; NULL if F_sh == 0.
+ *  W_norm [N][d] weights gamma_l of the MoE sublayer's pre-FFN RMSNorm, or NULL
+ *       for none.  With it, layer l computes r = 1/sqrt(mean(h^2) + norm_eps);
+ *       the router reads h*r*gamma_l (fp32), the experts its bf16 rounding, the
+ *       exit head h*r, and the combine adds to h itself (pre-norm residual). */
 typedef struct {
     const void* W_r;
     const float* b_r;
@@ -92,6 +98,7 @@ typedef struct {
     const void* W2;
     const void* W13_sh;
     const void* W2_sh;
+    const void* W_norm;
 } trimmoe_weights;
 
 /* The paper's input tables (host, copied at create).

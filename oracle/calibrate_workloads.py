@@ -84,7 +84,8 @@ def _head_logits(om, Wx, h_row):
     wx = np.ascontiguousarray(Wx, dtype=np.uint16)
     bx = np.zeros(cfg.C, np.float32)
     hr = np.ascontiguousarray(h_row, dtype=np.uint16)
-    O.lib().or_exit_conf(C.byref(om.m), wx.ctypes.data, bx.ctypes.data, hr.ctypes.data, out.ctypes.data)
+    O.lib().or_exit_conf(C.byref(om.m), wx.ctypes.data, bx.ctypes.data, hr.ctypes.data,
+                         int(cfg.norm), out.ctypes.data)
     return out.astype(np.float64)
 
 

@@ -38,7 +38,7 @@ def build(force: bool = False) -> str:
 class OrModel(C.Structure):
     _fields_ = [(n, C.c_int) for n in
                 ("N", "d", "E", "k", "F", "F_sh", "C", "M", "H", "act", "renorm_topk", "n_sub")] + \
-               [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref", "phi_beta")] + [
+               [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref", "phi_beta", "norm_eps")] + [
         ("place", C.c_void_p), ("sim", C.c_void_p), ("sub_thresh", C.c_void_p),
         ("trans", C.c_void_p), ("comp", C.c_void_p), ("P", C.c_void_p), ("theta", C.c_void_p),
         ("lambda_", C.c_void_p), ("eps", C.c_void_p)]
@@ -46,7 +46,7 @@ class OrModel(C.Structure):
 
 class OrLayerWeights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in
-                ("W_r", "b_r", "W_x_prev", "b_x_prev", "W13", "W2", "W13_sh", "W2_sh")]
+                ("W_r", "b_r", "W_x_prev", "b_x_prev", "W13", "W2", "W13_sh", "W2_sh", "W_norm")]
 
 
 class OrTokens(C.Structure):
@@ -74,8 +74,10 @@ def lib():
         if _lib is None:
             L = C.CDLL(build())
             vp, i, f = C.c_void_p, C.c_int, C.c_float
-            L.or_router.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp]
-            L.or_exit_conf.argtypes = [vp, vp, vp, vp, vp]
+            L.or_router.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+            L.or_exit_conf.argtypes = [vp, vp, vp, vp, i, vp]
+            L.or_rms_factor.argtypes = [vp, i, f]
+            L.or_rms_factor.restype = C.c_double
             L.or_exit_conf.restype = f
             L.or_sub_loss.argtypes = [vp, i, i, i]
             L.or_sub_loss.restype = f
@@ -117,13 +119,14 @@ class OracleModel:
             N=cfg.N, d=cfg.d, E=cfg.E, k=cfg.k, F=cfg.F, F_sh=cfg.F_sh, C=cfg.C, M=cfg.M, H=cfg.H,
             act=cfg.act, renorm_topk=cfg.renorm_topk, n_sub=cfg.n_sub,
             omega_T=cfg.omega_T, omega_D=cfg.omega_D, d_ref=t["d_ref"], phi_beta=cfg.phi_beta,
+            norm_eps=cfg.norm_eps,
             place=_p(keep("place", t["place"], np.uint16)), sim=_p(keep("sim", t["sim"], np.float32)),
             sub_thresh=_p(keep("sub_thresh", t["sub_thresh"], np.float32)),
             trans=_p(keep("trans", t["trans"], np.float32)), comp=_p(keep("comp", t["comp"], np.float32)),
             P=_p(keep("P", t["P"] if t["P"].size else np.zeros((1, cfg.E, cfg.E)), np.float32)),
             theta=_p(keep("theta", t["theta"], np.float32)), lambda_=_p(keep("lam", t["lam"], np.float32)),
             eps=_p(keep("eps", t["eps"], np.float32)))
-        self.small = {k: np.ascontiguousarray(v) for k, v in small.items()}
+        self.small = {k: (None if v is None else np.ascontiguousarray(v)) for k, v in small.items()}
         self.experts = experts   # dict of numpy arrays (bf16 bits) per layer or full, or None
 
     def layer_weights(self, l, experts_l=None):
@@ -137,10 +140,11 @@ class OracleModel:
         wr = np.ascontiguousarray(s["W_r"][l], dtype=np.uint16)
         wx = np.ascontiguousarray(s["W_x"][l - 1], dtype=np.uint16) if l > 0 else None
         bx = np.ascontiguousarray(s["b_x"][l - 1], dtype=np.float32) if l > 0 else None
+        wn = np.ascontiguousarray(s["W_norm"][l], dtype=np.uint16) if s.get("W_norm") is not None else None
         lw = OrLayerWeights(W_r=_p(wr), b_r=_p(br), W_x_prev=_p(wx), b_x_prev=_p(bx),
                             W13=_p(ex.get("W13")), W2=_p(ex.get("W2")),
-                            W13_sh=_p(ex.get("W13_sh")), W2_sh=_p(ex.get("W2_sh")))
-        lw._keep = (wr, br, wx, bx, ex)
+                            W13_sh=_p(ex.get("W13_sh")), W2_sh=_p(ex.get("W2_sh")), W_norm=_p(wn))
+        lw._keep = (wr, br, wx, bx, ex, wn)
         return lw
 
 
@@ -208,16 +212,25 @@ def router(om: OracleModel, l, h_row):
     topk = np.zeros(16, np.int32); g = np.zeros(16, np.float32); I = np.zeros(1, np.float32)
     wr = np.ascontiguousarray(om.small["W_r"][l], dtype=np.uint16)
     br = np.ascontiguousarray(om.small["b_r"][l], dtype=np.float32)
+    wn = om.small.get("W_norm")
+    wn = None if wn is None else np.ascontiguousarray(wn[l], dtype=np.uint16)
     hr = np.ascontiguousarray(h_row, dtype=np.uint16)
-    lib().or_router(C.byref(om.m), _p(wr), _p(br), _p(hr), _p(z), _p(p), _p(topk), _p(g), _p(I))
+    lib().or_router(C.byref(om.m), _p(wr), _p(br), _p(wn), _p(hr), _p(z), _p(p), _p(topk), _p(g), _p(I))
     return z, p, topk[:cfg.k].copy(), g[:cfg.k].copy(), float(I[0])
 
 
-def exit_conf(om: OracleModel, W_x_l, b_x_l, h_row):
+def exit_conf(om: OracleModel, W_x_l, b_x_l, h_row, normalise=None):
     wx = np.ascontiguousarray(W_x_l, dtype=np.uint16)
     bx = np.ascontiguousarray(b_x_l, dtype=np.float32)
     hr = np.ascontiguousarray(h_row, dtype=np.uint16)
-    return float(lib().or_exit_conf(C.byref(om.m), _p(wx), _p(bx), _p(hr), None))
+    if normalise is None:
+        normalise = om.small.get("W_norm") is not None
+    return float(lib().or_exit_conf(C.byref(om.m), _p(wx), _p(bx), _p(hr), int(normalise), None))
+
+
+def rms_factor(om: OracleModel, h_row):
+    hr = np.ascontiguousarray(h_row, dtype=np.uint16)
+    return float(lib().or_rms_factor(_p(hr), om.cfg.d, C.c_float(om.cfg.norm_eps)))
 
 
 def candidates(om: OracleModel, l, r):

@@ -12,7 +12,12 @@
 //
 // Readings of the paper where it is silent or garbled (each one is listed with
 // its reason in the design notes):
+//  * the MoE sublayer is pre-norm (as in the three evaluated models): with norm
+//    weights gamma_l the router and the experts read x = h * r * gamma_l,
+//    r = 1/sqrt(mean(h^2) + eps); the exit head reads h * r; the residual is h.
+//    The router uses x unrounded, the experts its bf16 rounding;
 //  * importance I = sum of the full-softmax probabilities of the top-k set (Eq. 4);
+//  * a NaN logit ranks as -infinity;
 //  * top-k is ordered by logit, descending, ties to the lower expert index;
 //  * exit head: C == 1 -> sigmoid (Sec. IV-A); C > 1 -> max softmax probability;
 //  * exit is an action at layer l, admissible iff l > 0, layer l-1 was executed
@@ -77,7 +82,7 @@ extern "C" {
 // Model hyper-parameters and the paper's input tables (all host memory).
 typedef struct {
     int N, d, E, k, F, F_sh, C, M, H, act, renorm_topk, n_sub;
-    float omega_T, omega_D, d_ref, phi_beta;
+    float omega_T, omega_D, d_ref, phi_beta, norm_eps;
     const uint16_t* place;     // [N][E] server bit mask, x_{m,l,k} (Eq. 1-2)
     const float* sim;          // [N][E][E] Sim_l(r, k) (Eq. 3)
     const float* sub_thresh;   // [N] substitute admission threshold on Sim
@@ -99,6 +104,7 @@ typedef struct {
     const uint16_t* W2;        // [E][d][F]
     const uint16_t* W13_sh;    // [2*F_sh][d] or NULL
     const uint16_t* W2_sh;     // [d][F_sh] or NULL
+    const uint16_t* W_norm;    // [d] RMSNorm weights of this layer, NULL = no normalisation
 } OrLayerWeights;
 
 // Per-token state (host arrays of length T), updated in place.
@@ -145,11 +151,32 @@ typedef struct {
 
 // ---------------------------------------------------------------- routing
 
-// Router logits, softmax and top-k; importance by Eq. (4).
-void or_router(const OrModel* md, const uint16_t* W_r, const float* b_r, const uint16_t* h,
-               float* z, float* p, int* topk, float* g, float* I) {
+// RMS factor r = 1 / sqrt(mean(h^2) + eps) of the pre-FFN RMSNorm.
+double or_rms_factor(const uint16_t* h, int d, float eps) {
+    double ss = 0.0;
+    for (int i = 0; i < d; ++i) ss += (double)bf2f(h[i]) * (double)bf2f(h[i]);
+    return 1.0 / std::sqrt(ss / d + (double)eps);
+}
+
+// Router logits on the normalised hidden state, softmax and top-k; importance
+// by Eq. (4).  W_norm == NULL: the router reads h itself.
+void or_router(const OrModel* md, const uint16_t* W_r, const float* b_r, const uint16_t* W_norm,
+               const uint16_t* h, float* z, float* p, int* topk, float* g, float* I) {
     const int E = md->E, d = md->d;
-    for (int e = 0; e < E; ++e) z[e] = (float)dot_bf16(h, W_r + (size_t)e * d, d) + b_r[e];
+    if (W_norm) {
+        const double r = or_rms_factor(h, d, md->norm_eps);
+        for (int e = 0; e < E; ++e) {
+            const uint16_t* w = W_r + (size_t)e * d;
+            double acc = 0.0;
+            for (int i = 0; i < d; ++i)
+                acc += (double)bf2f(h[i]) * (double)bf2f(W_norm[i]) * (double)bf2f(w[i]);
+            z[e] = (float)(acc * r) + b_r[e];
+        }
+    } else {
+        for (int e = 0; e < E; ++e) z[e] = (float)dot_bf16(h, W_r + (size_t)e * d, d) + b_r[e];
+    }
+    for (int e = 0; e < E; ++e)
+        if (z[e] != z[e]) z[e] = -kInf;
     float zmax = -kInf;
     for (int e = 0; e < E; ++e) zmax = std::max(zmax, z[e]);
     float S = 0.0f;
@@ -159,7 +186,7 @@ void or_router(const OrModel* md, const uint16_t* W_r, const float* b_r, const u
     for (int j = 0; j < md->k; ++j) {
         int best = -1;
         for (int e = 0; e < E; ++e)
-            if (!used[e] && (best < 0 || z[e] > z[best])) best = e;
+            if (!used[e] && (best < 0 || z[e] > z[best])) best = e;   // ties: lower index
         used[best] = 1;
         topk[j] = best;
     }
@@ -169,12 +196,14 @@ void or_router(const OrModel* md, const uint16_t* W_r, const float* b_r, const u
 }
 
 // Exit-head confidence xi = h_l(h) in [0, 1] (Eq. 7).  C == 1: sigmoid head of
-// Sec. IV-A; C > 1: the largest softmax probability over C classes.
+// Sec. IV-A; C > 1: the largest softmax probability over C classes.  With
+// normalise != 0 the head reads the RMS-normalised state h * r.
 float or_exit_conf(const OrModel* md, const uint16_t* W_x, const float* b_x, const uint16_t* h,
-                   float* logits_out) {
+                   int normalise, float* logits_out) {
     const int C = md->C, d = md->d;
+    const double r = normalise ? or_rms_factor(h, d, md->norm_eps) : 1.0;
     std::vector<float> x(C);
-    for (int c = 0; c < C; ++c) x[c] = (float)dot_bf16(h, W_x + (size_t)c * d, d) + b_x[c];
+    for (int c = 0; c < C; ++c) x[c] = (float)(dot_bf16(h, W_x + (size_t)c * d, d) * r) + b_x[c];
     if (logits_out) for (int c = 0; c < C; ++c) logits_out[c] = x[c];
     if (C == 1) return 1.0f / (1.0f + expf(-x[0]));
     float xm = -kInf;
@@ -413,9 +442,10 @@ void or_decide_token(const OrModel* md, const OrLayerWeights* lw, int l, const u
     std::vector<float> z(md->E), p(md->E);
     int topk[16];
     float g[16], I;
-    or_router(md, lw->W_r, lw->b_r, h, z.data(), p.data(), topk, g, &I);
+    or_router(md, lw->W_r, lw->b_r, lw->W_norm, h, z.data(), p.data(), topk, g, &I);
     float xi = -1.0f;
-    if (l > 0 && last_exec && lw->W_x_prev) xi = or_exit_conf(md, lw->W_x_prev, lw->b_x_prev, h, nullptr);
+    if (l > 0 && last_exec && lw->W_x_prev)
+        xi = or_exit_conf(md, lw->W_x_prev, lw->b_x_prev, h, lw->W_norm != nullptr, nullptr);
     or_decide_given(md, l, topk, g, I, xi, s, Dhat, Dbar, pJ, last_exec, out);
     // Near-threshold flags for the comparison protocol.
     const float band = 1e-5f;
@@ -515,9 +545,16 @@ int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uin
         const OrDecision& D = dec[t];
         if (D.action != A_EXEC && D.action != A_SKIP) continue;
         if (row_mask && !row_mask[t]) continue;
-        const uint16_t* x = hin.data() + (size_t)t * d;
+        const uint16_t* hrow = hin.data() + (size_t)t * d;
         std::vector<float> acc(d);
-        for (int o = 0; o < d; ++o) acc[o] = bf2f(x[o]);
+        for (int o = 0; o < d; ++o) acc[o] = bf2f(hrow[o]);
+        // Expert input: bf16 rounding of the normalised state (or h itself).
+        std::vector<uint16_t> xn(hrow, hrow + d);
+        if (lw->W_norm) {
+            const double r = or_rms_factor(hrow, d, md->norm_eps);
+            for (int i = 0; i < d; ++i) xn[i] = d2bf((double)bf2f(hrow[i]) * r * (double)bf2f(lw->W_norm[i]));
+        }
+        const uint16_t* x = xn.data();
         std::vector<uint16_t> y(d);
         if (D.action == A_EXEC) {
             float gs = 0.0f;

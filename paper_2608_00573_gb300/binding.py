@@ -34,11 +34,12 @@ class trimmoe_config(C.Structure):
     _fields_ = [(n, C.c_int) for n in ("N", "d", "E", "k", "F", "F_sh", "C", "M", "H", "act",
                                        "renorm_topk", "n_sub", "T_max")] + \
                [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref_ms", "phi_beta")] + \
-               [("profile", C.c_int)]
+               [("profile", C.c_int), ("norm_eps", C.c_float)]
 
 
 class trimmoe_weights(C.Structure):
-    _fields_ = [(n, C.c_void_p) for n in ("W_r", "b_r", "W_x", "b_x", "W13", "W2", "W13_sh", "W2_sh")]
+    _fields_ = [(n, C.c_void_p) for n in ("W_r", "b_r", "W_x", "b_x", "W13", "W2", "W13_sh", "W2_sh",
+                                          "W_norm")]
 
 
 class trimmoe_tables(C.Structure):
@@ -196,13 +197,14 @@ class Engine:
             "W13": dt(experts["W13"], torch.bfloat16), "W2": dt(experts["W2"], torch.bfloat16),
             "W13_sh": dt(experts["W13_sh"], torch.bfloat16) if cfg.F_sh else None,
             "W2_sh": dt(experts["W2_sh"], torch.bfloat16) if cfg.F_sh else None,
+            "W_norm": dt(small["W_norm"], torch.bfloat16) if small.get("W_norm") is not None else None,
         }
         self.tables = {k: np.ascontiguousarray(v) for k, v in tables.items() if k != "d_ref"}
         self.c_cfg = trimmoe_config(
             N=cfg.N, d=cfg.d, E=cfg.E, k=cfg.k, F=cfg.F, F_sh=cfg.F_sh, C=cfg.C, M=cfg.M, H=cfg.H,
             act=cfg.act, renorm_topk=cfg.renorm_topk, n_sub=cfg.n_sub, T_max=T_max,
             omega_T=cfg.omega_T, omega_D=cfg.omega_D, d_ref_ms=float(tables["d_ref"]),
-            phi_beta=cfg.phi_beta, profile=1 if profile else 0)
+            phi_beta=cfg.phi_beta, profile=1 if profile else 0, norm_eps=cfg.norm_eps)
         self.c_w = trimmoe_weights(**{k: _ptr(v) for k, v in self.w.items()})
         t = self.tables
         P = t["P"].astype(np.float32) if t["P"].size else None

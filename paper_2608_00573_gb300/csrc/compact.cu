@@ -117,10 +117,13 @@ __global__ void __launch_bounds__(32) scatter_kernel(const CompactParams p) {
     }
 }
 
-// Xp[row] = h[token of row] for every compacted row; one warp per row.
+// Xp[row] = expert input of the row's token: bf16(h * r * gamma) with the
+// pre-FFN RMSNorm, or h itself without it; one warp per row.
 __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ goff, int E, int k,
                                                      int d, const __nv_bfloat16* __restrict__ h,
+                                                     const float* __restrict__ rnorm,
+                                                     const __nv_bfloat16* __restrict__ gamma,
                                                      __nv_bfloat16* __restrict__ Xp) {
     const int nrows = goff[E + 1];
     const int routed = goff[E];
@@ -132,7 +135,22 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
         const int t = r < routed ? code / k : code;
         const uint4* src = reinterpret_cast<const uint4*>(h + (size_t)t * d);
         uint4* dst = reinterpret_cast<uint4*>(Xp + (size_t)r * d);
-        for (int c = lane; c < nchunk; c += 32) dst[c] = src[c];
+        if (!gamma) {
+            for (int c = lane; c < nchunk; c += 32) dst[c] = src[c];
+            continue;
+        }
+        const float rn = rnorm[t];
+        const uint4* gv4 = reinterpret_cast<const uint4*>(gamma);
+        for (int c = lane; c < nchunk; c += 32) {
+            const uint4 hv = src[c];
+            const uint4 gv = __ldg(gv4 + c);
+            uint4 o;
+            o.x = pack_bf16x2(bf16_lo(hv.x) * rn * bf16_lo(gv.x), bf16_hi(hv.x) * rn * bf16_hi(gv.x));
+            o.y = pack_bf16x2(bf16_lo(hv.y) * rn * bf16_lo(gv.y), bf16_hi(hv.y) * rn * bf16_hi(gv.y));
+            o.z = pack_bf16x2(bf16_lo(hv.z) * rn * bf16_lo(gv.z), bf16_hi(hv.z) * rn * bf16_hi(gv.z));
+            o.w = pack_bf16x2(bf16_lo(hv.w) * rn * bf16_lo(gv.w), bf16_hi(hv.w) * rn * bf16_hi(gv.w));
+            dst[c] = o;
+        }
     }
 }
 
@@ -147,12 +165,12 @@ cudaError_t launch_compact(const CompactParams& p, cudaStream_t st) {
 }
 
 cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
-                          const __nv_bfloat16* h, __nv_bfloat16* Xp, int max_rows, int num_sms,
-                          cudaStream_t st) {
+                          const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,
+                          __nv_bfloat16* Xp, int max_rows, int num_sms, cudaStream_t st) {
     if (max_rows <= 0) return cudaSuccess;
     int blocks = (max_rows + 7) / 8;
     blocks = blocks < num_sms * 8 ? blocks : num_sms * 8;
-    gather_kernel<<<blocks, 256, 0, st>>>(perm, goff, E, k, d, h, Xp);
+    gather_kernel<<<blocks, 256, 0, st>>>(perm, goff, E, k, d, h, rnorm, gamma, Xp);
     return cudaGetLastError();
 }
 

@@ -69,9 +69,11 @@ __device__ __forceinline__ float dot8(const float (&h)[8], uint4 w) {
     return a;
 }
 
-// out[r] = dot(h_row, W[r]) + b[r] for r < R; lanes split d in 16-byte chunks.
-__device__ void warp_gemv(const uint4* __restrict__ hrow, const __nv_bfloat16* __restrict__ W,
-                          const float* __restrict__ b, int R, int d, int lane, float* out) {
+// out[r] = dot(h_row * gamma, W[r]) * scale + b[r] for r < R (gamma may be NULL);
+// lanes split d in 16-byte chunks.
+__device__ void warp_gemv(const uint4* __restrict__ hrow, const __nv_bfloat16* __restrict__ gamma,
+                          const __nv_bfloat16* __restrict__ W, const float* __restrict__ b, int R,
+                          int d, int lane, float scale, float* out) {
     const int nchunk = d >> 3;
     for (int r0 = 0; r0 < R; r0 += 8) {
         const int nr = min(8, R - r0);
@@ -80,8 +82,13 @@ __device__ void warp_gemv(const uint4* __restrict__ hrow, const __nv_bfloat16* _
         for (int i = 0; i < 8; ++i) acc[i] = 0.f;
         for (int c = lane; c < nchunk; c += 32) {
             const uint4 hv = hrow[c];
-            const float hf[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
-                                 bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
+            float hf[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
+                           bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
+            if (gamma) {
+                const uint4 gv = __ldg(reinterpret_cast<const uint4*>(gamma) + c);
+                hf[0] *= bf16_lo(gv.x); hf[1] *= bf16_hi(gv.x); hf[2] *= bf16_lo(gv.y); hf[3] *= bf16_hi(gv.y);
+                hf[4] *= bf16_lo(gv.z); hf[5] *= bf16_hi(gv.z); hf[6] *= bf16_lo(gv.w); hf[7] *= bf16_hi(gv.w);
+            }
 #pragma unroll
             for (int i = 0; i < 8; ++i)
                 if (i < nr) {
@@ -92,7 +99,7 @@ __device__ void warp_gemv(const uint4* __restrict__ hrow, const __nv_bfloat16* _
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc[i] = warp_sum(acc[i]);
         if (lane == 0)
-            for (int i = 0; i < nr; ++i) out[r0 + i] = __fadd_rn(acc[i], b[r0 + i]);
+            for (int i = 0; i < nr; ++i) out[r0 + i] = __fadd_rn(__fmul_rn(acc[i], scale), b[r0 + i]);
     }
     __syncwarp();
 }
@@ -159,8 +166,27 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         const int last_exec = p.last_exec[t];
         const uint4* hrow = reinterpret_cast<const uint4*>(p.h + (size_t)t * p.d);
 
-        // Router logits, softmax (Eq. 4) and top-k by logit.
-        warp_gemv(hrow, p.W_r, p.b_r, E, p.d, lane, zs);
+        // Pre-FFN RMSNorm factor r = 1/sqrt(mean(h^2) + eps).
+        float rn = 1.f;
+        if (p.W_norm) {
+            float ss = 0.f;
+            for (int c = lane; c < (p.d >> 3); c += 32) {
+                const uint4 hv = hrow[c];
+                const float v[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
+                                    bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
+            }
+            ss = warp_sum(ss);
+            rn = rsqrtf(ss / (float)p.d + p.norm_eps);
+            if (lane == 0) p.rnorm[t] = rn;
+        }
+        // Router logits on the normalised state, softmax (Eq. 4), top-k by logit
+        // (a NaN logit ranks as -infinity).
+        warp_gemv(hrow, p.W_norm, p.W_r, p.b_r, E, p.d, lane, rn, zs);
+        for (int e = lane; e < E; e += 32)
+            if (zs[e] != zs[e]) zs[e] = -kInf;
+        __syncwarp();
         float zmax = -FLT_MAX;
         for (int e = lane; e < E; e += 32) zmax = fmaxf(zmax, zs[e]);
         zmax = warp_max(zmax);
@@ -178,7 +204,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         float g[kMaxK];
         unsigned used = 0u;   // bit i: expert lane + 32 i taken
         for (int j = 0; j < K; ++j) {
-            float bz = -FLT_MAX;
+            float bz = -kInf;
             int be = 0x7fffffff;
             for (int i = 0, e = lane; e < E; ++i, e += 32)
                 if (!((used >> i) & 1u) && (zs[e] > bz || (zs[e] == bz && e < be))) { bz = zs[e]; be = e; }
@@ -193,7 +219,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         float xi = -1.f;
         const bool have_xi = (l > 0) && last_exec && (p.W_x != nullptr);
         if (have_xi) {
-            warp_gemv(hrow, p.W_x, p.b_x, C, p.d, lane, xs);
+            warp_gemv(hrow, nullptr, p.W_x, p.b_x, C, p.d, lane, rn, xs);
             if (C == 1) {
                 xi = __fdiv_rn(1.f, __fadd_rn(1.f, expf(-xs[0])));
             } else {

@@ -55,6 +55,9 @@ struct DecideParams {
     const float* b_r;
     const __nv_bfloat16* W_x;   // [C][d] head of layer-1, NULL at layer 0
     const float* b_x;
+    const __nv_bfloat16* W_norm;   // [d] RMSNorm weights of this layer, NULL = none
+    float norm_eps;
+    float* rnorm;               // [T] RMS factor r per token (written when W_norm)
     uint8_t* s;
     float* Dhat;
     const float* Dbar;
@@ -115,8 +118,8 @@ struct CombineParams {
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);
 cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
-                          const __nv_bfloat16* h, __nv_bfloat16* Xp, int max_rows, int num_sms,
-                          cudaStream_t st);
+                          const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,
+                          __nv_bfloat16* Xp, int max_rows, int num_sms, cudaStream_t st);
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st);
 size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);

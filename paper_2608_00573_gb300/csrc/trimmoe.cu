@@ -92,6 +92,7 @@ struct trimmoe {
     uint8_t* exp_sel = nullptr;
     uint8_t* srv_sel = nullptr;
     int32_t *perm = nullptr, *pos_pair = nullptr, *pos_sh = nullptr, *goff = nullptr;
+    float* rnorm = nullptr;
     int32_t *blk_counts = nullptr, *blk_base = nullptr;
     __nv_bfloat16 *Xp = nullptr, *act = nullptr, *act_sh = nullptr, *Y = nullptr, *Ysh = nullptr;
     DevCounters* ctr = nullptr;
@@ -180,6 +181,7 @@ trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
     }
     if (c->act != 0 && c->act != 1) { why = "config: act must be 0 (ReLU) or 1 (SwiGLU)"; return TRIMMOE_ERR_ARG; }
     if (!(c->d_ref_ms > 0.f) || !std::isfinite(c->d_ref_ms)) { why = "config: d_ref_ms must be > 0"; return TRIMMOE_ERR_ARG; }
+    if (!(c->norm_eps >= 0.f) || !std::isfinite(c->norm_eps)) { why = "config: norm_eps must be >= 0"; return TRIMMOE_ERR_ARG; }
     if (c->d % 256) { why = "config: d must be a multiple of 256"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->act == 1 && c->F % 128) { why = "config: SwiGLU F must be a multiple of 128"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->act == 0 && c->F % 256) { why = "config: ReLU F must be a multiple of 256"; return TRIMMOE_ERR_UNSUPPORTED; }
@@ -220,7 +222,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     if ((c.F_sh > 0) != (w->W13_sh != nullptr && w->W2_sh != nullptr))
         return create_fail(TRIMMOE_ERR_ARG, "create: shared-expert weights must be given iff F_sh > 0");
     if (!aligned16(w->W_r) || !aligned16(w->W_x) || !aligned16(w->W13) || !aligned16(w->W2) ||
-        (c.F_sh && (!aligned16(w->W13_sh) || !aligned16(w->W2_sh))))
+        (c.F_sh && (!aligned16(w->W13_sh) || !aligned16(w->W2_sh))) || (w->W_norm && !aligned16(w->W_norm)))
         return create_fail(TRIMMOE_ERR_ARG, "create: weights must be 16-byte aligned");
     if (!tab->place || !tab->sim || !tab->sub_thresh || !tab->trans_ms || !tab->comp_ms || !tab->theta ||
         !tab->lambda || !tab->eps || (N > 1 && !tab->P))
@@ -314,6 +316,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->topk_g, TK) && h->dalloc(&h->I, T) && h->dalloc(&h->xi, T) &&
               h->dalloc(&h->action, T) && h->dalloc(&h->exp_sel, TK) && h->dalloc(&h->srv_sel, TK) &&
               h->dalloc(&h->perm, TK + T) && h->dalloc(&h->pos_pair, TK) && h->dalloc(&h->pos_sh, T) &&
+              h->dalloc(&h->rnorm, T) &&
               h->dalloc(&h->goff, (size_t)E + 2) && h->dalloc(&h->blk_counts, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->blk_base, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
@@ -396,6 +399,11 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.b_r = h->w.b_r + (size_t)layer * E;
     dp.W_x = layer > 0 ? static_cast<const __nv_bfloat16*>(h->w.W_x) + (size_t)(layer - 1) * c.C * d : nullptr;
     dp.b_x = layer > 0 ? h->w.b_x + (size_t)(layer - 1) * c.C : nullptr;
+    const __nv_bfloat16* gamma =
+        h->w.W_norm ? static_cast<const __nv_bfloat16*>(h->w.W_norm) + (size_t)layer * d : nullptr;
+    dp.W_norm = gamma;
+    dp.norm_eps = c.norm_eps;
+    dp.rnorm = h->rnorm;
     dp.s = tok->s;
     dp.Dhat = tok->Dhat;
     dp.Dbar = tok->Dbar;
@@ -445,7 +453,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("compact: ") + cudaGetErrorString(e));
     const int max_rows = T * K + (has_sh ? T : 0);
     e = h->timed(K_GATHER, st, [&] {
-        return launch_gather(h->perm, h->goff, E, K, d, dp.h, h->Xp, max_rows, h->num_sms, st);
+        return launch_gather(h->perm, h->goff, E, K, d, dp.h, h->rnorm, gamma, h->Xp, max_rows, h->num_sms, st);
     });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gather: ") + cudaGetErrorString(e));
 

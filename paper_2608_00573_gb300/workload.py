@@ -10,6 +10,9 @@ Switch-Base-8E, Qwen-MoE-A2.7B, Mixtral-8x7B); the paper's weights, datasets
 and testbed are not available, so every value here is synthetic:
 
 * weights ~ N(0, 1/fan_in) stored as bf16; hidden states ~ N(0, 1) in bf16;
+  RMSNorm weights of the MoE sublayer ~ N(1, 0.1^2) in bf16 (all three models
+  are pre-norm; without the norm a random-weight SwiGLU stack overflows bf16
+  within about ten layers);
 * router bias b_e = -s * ln(e + 1), which makes expert popularity Zipf(s);
 * users are blocks of 128 tokens; each user's access server a(i) (Eq. 12) is
   drawn Zipf(1.0) over the M servers, with p_J = 0.9 and a per-token budget
@@ -77,6 +80,8 @@ class WorkloadConfig:
     exit_target: float = 0.0         # target fraction of tokens exited
     exit_peak: Optional[float] = None
     exit_width: float = 2.0
+    norm: bool = True                # pre-FFN RMSNorm of the MoE sublayer
+    norm_eps: float = 1e-6
     seed: int = 0
 
     @property
@@ -213,10 +218,14 @@ def make_tables(cfg: WorkloadConfig, W_r_bits: Optional[np.ndarray] = None,
 
 
 def make_small_weights(cfg: WorkloadConfig, calib: Optional[dict] = "auto") -> dict:
-    """Router, exit-head weights (always host) -- small for every configuration."""
+    """Router, exit-head and norm weights (always host) -- small for every configuration."""
     rng = np.random.default_rng([cfg.seed, 202])
     N, E, d, C = cfg.N, cfg.E, cfg.d, cfg.C
     W_r = _normal_bf16(rng, (N, E, d), 1.0 / math.sqrt(d))
+    W_norm = None
+    if cfg.norm:
+        W_norm = f32_to_bf16_bits((1.0 + 0.1 * np.random.default_rng([cfg.seed, 505]).standard_normal(
+            (N, d))).astype(np.float32))
     b_r = np.tile((-cfg.zipf_s * np.log(np.arange(E) + 1.0)).astype(np.float32), (N, 1))
     W_x = _normal_bf16(rng, (N, C, d), 1.0 / math.sqrt(d))
     b_x = np.zeros((N, C), dtype=np.float32)
@@ -226,7 +235,7 @@ def make_small_weights(cfg: WorkloadConfig, calib: Optional[dict] = "auto") -> d
         b_x[:, 0] = np.asarray(calib["exit_bias"], dtype=np.float32)
     else:
         b_x[:, 0] = -30.0                                     # no exits
-    return dict(W_r=W_r, b_r=b_r, W_x=W_x, b_x=b_x)
+    return dict(W_r=W_r, b_r=b_r, W_x=W_x, b_x=b_x, W_norm=W_norm)
 
 
 def make_expert_weights_host(cfg: WorkloadConfig) -> dict:

@@ -86,9 +86,12 @@ def test_router_matches_sort_and_softmax():
     h = W.f32_to_bf16_bits(rng.standard_normal((40, cfg.d)).astype(np.float32))
     for l in range(cfg.N):
         Wr = W.bf16_bits_to_f32(om.small["W_r"][l]).astype(np.float64)
+        gam = W.bf16_bits_to_f32(om.small["W_norm"][l]).astype(np.float64)
         for t in range(h.shape[0]):
             z, p, topk, g, I = O.router(om, l, h[t])
-            zr = (W.bf16_bits_to_f32(h[t]).astype(np.float64) @ Wr.T).astype(np.float32) + om.small["b_r"][l]
+            hf = W.bf16_bits_to_f32(h[t]).astype(np.float64)
+            x = hf / np.sqrt(np.mean(hf * hf) + cfg.norm_eps) * gam       # RMSNorm
+            zr = (x @ Wr.T).astype(np.float32) + om.small["b_r"][l]
             np.testing.assert_allclose(z, zr, rtol=0, atol=1e-5)
             order = np.lexsort((np.arange(cfg.E), -z.astype(np.float64)))
             assert list(topk) == list(order[: cfg.k])
@@ -111,7 +114,7 @@ def test_importance_is_one_when_k_equals_E():
 
 
 def test_router_tie_goes_to_lower_index():
-    cfg = small_cfg(E=6, k=2)
+    cfg = small_cfg(E=6, k=2, norm=False)
     om, *_ = build_small(cfg, with_experts=False)
     om.small["W_r"][0][:] = 0          # all logits = bias
     om.small["b_r"][0][:] = np.array([0, 1, 1, 0.5, 1, 0], np.float32)
@@ -148,8 +151,12 @@ def test_exit_head_closed_forms():
     h[3] = 2.0
     cfg = small_cfg(C=1, d=d)
     om, *_ = build_small(cfg, with_experts=False)
-    xi = O.exit_conf(om, W.f32_to_bf16_bits(Wx), np.zeros(1, np.float32), W.f32_to_bf16_bits(h))
+    xi = O.exit_conf(om, W.f32_to_bf16_bits(Wx), np.zeros(1, np.float32), W.f32_to_bf16_bits(h), normalise=False)
     assert xi == pytest.approx(1.0 / (1.0 + math.exp(-1.0)), rel=1e-6)
+    # RMS-normalised input: mean(h^2) = 4/64, so w.h is scaled by 1/sqrt(1/16 + eps)
+    xi = O.exit_conf(om, W.f32_to_bf16_bits(Wx), np.zeros(1, np.float32), W.f32_to_bf16_bits(h), normalise=True)
+    x = 1.0 / math.sqrt(1.0 / 16 + cfg.norm_eps)
+    assert xi == pytest.approx(1.0 / (1.0 + math.exp(-x)), rel=1e-6)
 
 
 # -------------------------------------------------------------- candidates
@@ -469,7 +476,10 @@ def _numpy_dense_moe(cfg, small, ex, h_bits):
     T, d, F, G = h.shape[0], cfg.d, cfg.F, W.GATE_UP_GROUP
     for l in range(cfg.N):
         Wr = W.bf16_bits_to_f32(small["W_r"][l]).astype(np.float64)
-        z = (h @ Wr.T).astype(np.float32) + small["b_r"][l]
+        gam = W.bf16_bits_to_f32(small["W_norm"][l]).astype(np.float64)
+        xn = h / np.sqrt(np.mean(h * h, axis=1, keepdims=True) + cfg.norm_eps) * gam   # RMSNorm
+        z = (xn @ Wr.T).astype(np.float32) + small["b_r"][l]
+        xb = bf16_round(xn.astype(np.float32)).astype(np.float64)                   # expert input
         out = h.copy()
         for t in range(T):
             order = np.lexsort((np.arange(cfg.E), -z[t].astype(np.float64)))[: cfg.k]
@@ -478,7 +488,7 @@ def _numpy_dense_moe(cfg, small, ex, h_bits):
             g = p[order]
             if cfg.renorm_topk:
                 g = g / g.sum()
-            x = h[t]
+            x = xb[t]
             for j, e in enumerate(order):
                 w13 = W.bf16_bits_to_f32(ex["W13"][l, e]).astype(np.float64).reshape(F // G, 2, G, d)
                 gate, up = w13[:, 0].reshape(F, d), w13[:, 1].reshape(F, d)
