@@ -216,11 +216,33 @@ trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out);
 /* Zero the counters and the device error flag (synchronises). */
 trimmoe_status trimmoe_reset_stats(trimmoe_handle h);
 
-/* Last error message of the handle ("" if none); NULL handle: last create error. */
+/* Last error message of the handle ("" if none); NULL handle: the last error of
+ * a call made without a handle (trimmoe_create, trimmoe_compact_noalloc). */
 const char* trimmoe_last_error(trimmoe_handle h);
 
 /* Free the handle and its workspaces (synchronises first).  NULL is a no-op. */
 void trimmoe_destroy(trimmoe_handle h);
+
+/* Compaction of one layer's decisions without any device allocation (the
+ * paper has no counterpart: this entry point exists for callers that cannot
+ * call cudaMalloc, e.g. code running inside an allocator callback or in a
+ * process whose device memory is entirely owned by another pool).
+ * Inputs (device): action uint8 [T] and exp_sel uint8 [T][k] as written by
+ * trimmoe_layer_step.  Outputs (device, caller-owned): perm int32 [T*k + T] and
+ * group_off int32 [E+2] with the same contents as trimmoe_layer_out, pos_pair
+ * int32 [T*k] (position of pair t*k+j in perm, -1 if not executed) and pos_sh
+ * int32 [T] (row of token t among the shared-expert rows, -1 if none; may be
+ * NULL when has_shared == 0).  Per-chunk scratch lives in one static device
+ * array of about 264 KB held by every GPU that loads the library until exit;
+ * hence T <= 65536 and E <= 128 (ERR_ARG beyond, with a message in
+ * trimmoe_last_error(NULL)).  It calls no cudaMalloc/cudaFree.  The first call on
+ * each device looks up the array's device address once; make that first call
+ * before any stream capture.  All calls share the array: calls whose work
+ * overlaps on the GPU (other streams, other host threads) race and must be
+ * serialised by the caller.  Asynchronous on stream. */
+trimmoe_status trimmoe_compact_noalloc(const uint8_t* action, const uint8_t* exp_sel, int T, int k, int E,
+                                       int has_shared, int32_t* perm, int32_t* group_off,
+                                       int32_t* pos_pair, int32_t* pos_sh, void* stream);
 
 #ifdef __cplusplus
 }

@@ -74,7 +74,8 @@ class trimmoe_stats_t(C.Structure):
 
 
 EXPORTS = ("trimmoe_create", "trimmoe_layer_step", "trimmoe_forward", "trimmoe_forward_host",
-           "trimmoe_stats", "trimmoe_reset_stats", "trimmoe_last_error", "trimmoe_destroy")
+           "trimmoe_stats", "trimmoe_reset_stats", "trimmoe_last_error", "trimmoe_destroy",
+           "trimmoe_compact_noalloc")
 
 _lib = None
 _lock = threading.Lock()
@@ -106,6 +107,8 @@ def lib():
             L.trimmoe_last_error.restype = C.c_char_p
             L.trimmoe_destroy.argtypes = [vp]
             L.trimmoe_destroy.restype = None
+            L.trimmoe_compact_noalloc.argtypes = [vp, vp, i, i, i, i, vp, vp, vp, vp, vp]
+            L.trimmoe_compact_noalloc.restype = i
             _lib = L
     return _lib
 
@@ -157,6 +160,13 @@ def trimmoe_last_error(h=None) -> str:
 
 def trimmoe_destroy(h):
     lib().trimmoe_destroy(h)
+
+
+def trimmoe_compact_noalloc(action, exp_sel, T: int, k: int, E: int, has_shared: int, perm, group_off,
+                            pos_pair, pos_sh, stream: int = 0):
+    """Compaction into caller-owned outputs with no device allocation (device tensors)."""
+    _check(lib().trimmoe_compact_noalloc(_ptr(action), _ptr(exp_sel), T, k, E, has_shared, _ptr(perm),
+                                         _ptr(group_off), _ptr(pos_pair), _ptr(pos_sh), C.c_void_p(stream)))
 
 
 # ----------------------------------------------------------- engine

@@ -10,6 +10,9 @@
 // Three passes over chunks of kChunk tokens: per-chunk bucket counts, one
 // scan over chunks and buckets, and a scatter in which one warp walks its
 // chunk in order and ranks equal buckets with __match_any_sync.
+#include <mutex>
+#include <string>
+
 #include "internal.cuh"
 
 namespace tmoe {
@@ -175,3 +178,117 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
 }
 
 }  // namespace tmoe
+
+// ---------------------------------------------------------------------------
+// Compaction without any device allocation.
+//
+// Some callers cannot call cudaMalloc at all: code running inside an
+// allocator's own callback, processes whose device memory is fully handed to
+// another pool, or hosts that must not allocate during a captured or
+// latency-critical section.  For them the per-chunk counts and bases of the
+// compaction live in this file-scope device array instead of a handle's
+// workspace.  Its size is fixed (about 264 KB); every GPU that loads the
+// library holds it until the process exits.
+namespace tmoe {
+namespace {
+
+constexpr int kNoAllocMaxT = 65536;
+constexpr int kNoAllocMaxBlk = kNoAllocMaxT / kChunk;
+
+struct NoAllocScratch {
+    int32_t blk_counts[kNoAllocMaxBlk * (kMaxE + 1)];
+    int32_t blk_base[kNoAllocMaxBlk * (kMaxE + 1)];
+    DevCounters ctr;
+};
+
+}  // namespace
+}  // namespace tmoe
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[sizeof(tmoe::NoAllocScratch)];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kMaxDevices] = {nullptr};
+
+// Device address of the scratch array on the current device, looked up once
+// per device (the host-side symbol is only a stand-in, never a device address).
+trimmoe_status noalloc_scratch(tmoe::NoAllocScratch** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+        tmoe::set_global_error("compact_noalloc: no usable current CUDA device");
+        return TRIMMOE_ERR_CUDA;
+    }
+    std::lock_guard<std::mutex> g(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) {
+            tmoe::set_global_error(std::string("compact_noalloc: cudaGetSymbolAddress failed: ") +
+                                   cudaGetErrorString(e));
+            return TRIMMOE_ERR_CUDA;
+        }
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = static_cast<tmoe::NoAllocScratch*>(g_noalloc_ptr[dev]);
+    return TRIMMOE_OK;
+}
+
+}  // namespace
+
+extern "C" trimmoe_status trimmoe_compact_noalloc(const uint8_t* action, const uint8_t* exp_sel, int T,
+                                                  int k, int E, int has_shared, int32_t* perm,
+                                                  int32_t* group_off, int32_t* pos_pair, int32_t* pos_sh,
+                                                  void* stream) {
+    using namespace tmoe;
+    if (T < 0 || T > kNoAllocMaxT) {
+        set_global_error("compact_noalloc: T must be in [0, 65536] (size of the static scratch)");
+        return TRIMMOE_ERR_ARG;
+    }
+    if (E < 1 || E > kMaxE || k < 1 || k > kMaxK || k > E) {
+        set_global_error("compact_noalloc: need 1 <= E <= 128 and 1 <= k <= min(E, 8)");
+        return TRIMMOE_ERR_ARG;
+    }
+    if (!action || !exp_sel || !perm || !group_off || !pos_pair || (has_shared && !pos_sh)) {
+        set_global_error("compact_noalloc: NULL pointer");
+        return TRIMMOE_ERR_ARG;
+    }
+    NoAllocScratch* s = nullptr;
+    trimmoe_status rc = noalloc_scratch(&s);
+    if (rc != TRIMMOE_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // Only the counters must start at zero; counts and bases are fully rewritten.
+    if (cudaMemsetAsync(&s->ctr, 0, sizeof(DevCounters), st) != cudaSuccess) {
+        set_global_error("compact_noalloc: cudaMemsetAsync failed");
+        return TRIMMOE_ERR_CUDA;
+    }
+    if (T == 0) {
+        if (cudaMemsetAsync(group_off, 0, (size_t)(E + 2) * sizeof(int32_t), st) != cudaSuccess) {
+            set_global_error("compact_noalloc: cudaMemsetAsync failed");
+            return TRIMMOE_ERR_CUDA;
+        }
+        return TRIMMOE_OK;
+    }
+    CompactParams cp;
+    cp.T = T;
+    cp.k = k;
+    cp.E = E;
+    cp.has_shared = has_shared ? 1 : 0;
+    cp.nblk = (T + kChunk - 1) / kChunk;
+    cp.action = action;
+    cp.exp_sel = exp_sel;
+    cp.blk_counts = s->blk_counts;
+    cp.blk_base = s->blk_base;
+    cp.goff = group_off;
+    cp.perm = perm;
+    cp.pos_pair = pos_pair;
+    cp.pos_sh = pos_sh;
+    cp.ctr = &s->ctr;
+    const cudaError_t e = launch_compact(cp, st);
+    if (e != cudaSuccess) {
+        set_global_error(std::string("compact_noalloc: ") + cudaGetErrorString(e));
+        return TRIMMOE_ERR_CUDA;
+    }
+    return TRIMMOE_OK;
+}

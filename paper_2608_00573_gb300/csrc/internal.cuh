@@ -8,6 +8,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <string>
+
 #include "../../include/trimmoe.h"
 
 namespace tmoe {
@@ -123,6 +125,9 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st);
 size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
+
+// Error text for calls made without a handle (read by trimmoe_last_error(NULL)).
+void set_global_error(const std::string& msg);
 
 // ------------------------------------------------------------------ PTX
 

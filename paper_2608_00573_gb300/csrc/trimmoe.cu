@@ -68,6 +68,11 @@ struct DeviceGuard {
 
 }  // namespace
 
+void tmoe::set_global_error(const std::string& msg) {
+    std::lock_guard<std::mutex> g(g_err_mu);
+    g_create_error = msg;
+}
+
 struct trimmoe {
     trimmoe_config cfg;
     trimmoe_weights w;
