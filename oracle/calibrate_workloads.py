@@ -1,11 +1,13 @@
 """Write paper_2608_00573_gb300/workload_calib.json (skip thresholds, exit biases).
 
 Stand-in for the offline threshold calibration of Sec. IV-B (Eq. 24-25) on the
-synthetic workloads: theta_l is the importance quantile at which about the
-target share of layer-tokens is admitted to skip, and the exit head's class-0
-bias is set per layer so that the share of tokens whose confidence reaches p_J
-follows the target exit profile.  Only the oracle computes router outputs and
-exit-head logits here; the sample is the first tokens of the seeded input.
+synthetic workloads.  The exit head's class-0 bias is set per layer so that the
+share of tokens whose confidence reaches p_J follows the target exit profile;
+then theta_l is the importance quantile q (the same q for every layer) found
+by bisection so that an oracle decisions-only pilot over all layers skips the
+target share of live layer-tokens.  Only the oracle computes router outputs,
+exit-head logits and decisions here; the sample is the first tokens of the
+seeded input.
 
     python oracle/calibrate_workloads.py            # all workloads
 """
@@ -24,10 +26,7 @@ from oracle import oracle as O  # noqa: E402
 from paper_2608_00573_gb300 import workload as W  # noqa: E402
 
 SAMPLE = 1024
-# Share of layer-tokens whose execute candidates are all remote on these
-# placements (2-4 replicas of 10 servers, plus substitutes); skip admission by
-# importance is scaled by its inverse.
-REMOTE_SHARE = 0.5
+PILOT = 512
 
 
 def calibrate(name: str) -> dict:
@@ -37,11 +36,8 @@ def calibrate(name: str) -> dict:
     om = O.OracleModel(cfg, tables, small)
     tok = W.make_tokens(cfg, T=max(cfg.T, SAMPLE))
     h = tok["h"][:SAMPLE]
-    q = min(1.0, cfg.skip_target / REMOTE_SHARE)
-    theta = []
-    for l in range(cfg.N):
-        I = np.array([O.router(om, l, h[t])[4] for t in range(len(h))], dtype=np.float64)
-        theta.append(float(np.quantile(I, q)) if q > 0 else -1.0)
+    Is = [np.array([O.router(om, l, h[t])[4] for t in range(len(h))], dtype=np.float64)
+          for l in range(cfg.N)]
     # Exit: target share of the still-alive tokens at layer l with xi >= p_J.
     prof = W.exit_profile(cfg)
     alive = 1.0
@@ -74,7 +70,45 @@ def calibrate(name: str) -> dict:
             else:
                 hi = mid
         bias[l - 1] = float(hi)
-    return {"theta": theta, "exit_bias": bias, "sample_tokens": SAMPLE, "skip_quantile": q}
+    small_b = dict(small)
+    small_b["b_x"] = small["b_x"].copy()
+    small_b["b_x"][:, 0] = np.asarray(bias, dtype=np.float32)
+    pilot = {k: v[:PILOT] for k, v in tok.items()}
+
+    def skip_share(q):
+        tab = dict(tables)
+        tab["theta"] = np.array([np.quantile(I, q) for I in Is], dtype=np.float32)
+        kappa = max(cfg.skip_target * cfg.N, 1.0)
+        tab["eps"] = np.full(cfg.N, cfg.budget / kappa, dtype=np.float32)
+        tab["lam"] = (tab["eps"] / np.maximum(tab["theta"], 1e-6)).astype(np.float32)
+        pm = O.OracleModel(cfg, tab, small_b, None)
+        hh = pilot["h"]
+        st = {k: v for k, v in pilot.items() if k != "h"}
+        skipped = live = 0
+        for l in range(cfg.N):
+            hh, st, out = O.layer_step(pm, l, hh, st, row_mask=np.zeros(len(hh), np.uint8))
+            a = out["action"]
+            skipped += int((a == O.A_SKIP).sum())
+            live += int((a != O.A_DEAD).sum())
+        return skipped / max(live, 1), tab["theta"]
+
+    q = 0.0
+    theta = [-1.0] * cfg.N
+    achieved = 0.0
+    if cfg.skip_target > 0:
+        lo, hi = 0.0, 1.0
+        for _ in range(9):
+            mid = 0.5 * (lo + hi)
+            sh, th = skip_share(mid)
+            if sh < cfg.skip_target:
+                lo = mid
+            else:
+                hi = mid
+        q = hi
+        achieved, th = skip_share(q)
+        theta = [float(x) for x in th]
+    return {"theta": theta, "exit_bias": bias, "sample_tokens": SAMPLE, "pilot_tokens": PILOT,
+            "skip_quantile": q, "pilot_skip_share": achieved}
 
 
 def _head_logits(om, Wx, h_row):

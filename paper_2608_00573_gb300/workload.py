@@ -96,24 +96,33 @@ class WorkloadConfig:
         return dataclasses.replace(self, **kw)
 
 
+# Slope of phi in Q = phi((1 - Sim)/2) (Eq. 3).  The paper takes phi from its
+# reference [37], which is not available; 0.001 makes a substitution cost about
+# 2.5% of the 2% per-token budget, which reproduces the execution mix the paper
+# reports for Mixtral (Fig. 5(b): most executions local, about one in ten
+# layer-tokens skipped).
+PHI_BETA = 0.001
+
 # The five workloads: four model-shaped forwards and the decode stress case.
 CONFIGS = {
     "switch_tiny": WorkloadConfig(
         name="switch_tiny", N=4, d=768, E=8, k=1, F=3072, C=64, act=ACT_RELU, T=64,
-        placement="subset3", trans="uniform", skip_target=0.2, exit_target=0.15, seed=0),
+        placement="subset3", trans="uniform", skip_target=0.2, exit_target=0.15,
+        phi_beta=PHI_BETA, seed=0),
     "switch": WorkloadConfig(
         name="switch", N=12, d=768, E=8, k=1, F=3072, C=64, act=ACT_RELU, T=4096,
-        zipf_s=1.2, skip_target=0.20, exit_target=0.15, seed=1),
+        zipf_s=1.2, skip_target=0.20, exit_target=0.15, phi_beta=PHI_BETA, seed=1),
     "qwen": WorkloadConfig(
         name="qwen", N=24, d=2048, E=60, k=4, F=1408, F_sh=5632, C=1, act=ACT_SWIGLU,
-        T=8192, zipf_s=1.0, skip_target=0.11, exit_target=0.12, seed=2),
+        T=8192, zipf_s=1.0, skip_target=0.11, exit_target=0.12, phi_beta=PHI_BETA, seed=2),
     "mixtral": WorkloadConfig(
         name="mixtral", N=32, d=4096, E=8, k=2, F=14336, C=1, act=ACT_SWIGLU, renorm_topk=1,
-        T=16384, zipf_s=1.0, skip_target=0.11, exit_target=0.12, exit_peak=21.0, seed=3),
+        T=16384, zipf_s=1.0, skip_target=0.11, exit_target=0.12, exit_peak=21.0,
+        phi_beta=PHI_BETA, seed=3),
     "mixtral_decode": WorkloadConfig(
         name="mixtral_decode", N=32, d=4096, E=8, k=2, F=14336, C=1, act=ACT_SWIGLU,
         renorm_topk=1, T=256, zipf_s=1.5, skip_target=0.11, exit_target=0.40,
-        exit_peak=18.0, exit_width=4.0, seed=4),
+        exit_peak=18.0, exit_width=4.0, phi_beta=PHI_BETA, seed=4),
 }
 
 
