@@ -137,10 +137,29 @@ class ClockSampler:
                 "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": len(rows)}
 
 
+def workload_config(args):
+    """The named workload; --layers / --tokens shrink it for profiling runs."""
+    from paper_2608_00573_gb300 import workload as W
+    cfg = W.CONFIGS[args.config]
+    if args.layers or args.tokens:
+        over = {}
+        if args.layers:
+            over["N"] = args.layers
+        if args.tokens:
+            over["T"] = args.tokens
+        calib = W.load_calibration(cfg.name)
+        cfg = cfg.replace(**over)
+        cfg._calib = None if calib is None else {k: (v[: cfg.N] if isinstance(v, list) else v)
+                                                 for k, v in calib.items()}
+        cfg.name = f"{cfg.name}[N={cfg.N},T={cfg.T}]"
+    return cfg
+
+
 def make_workload(cfg, device):
     from paper_2608_00573_gb300 import workload as W
-    small = W.make_small_weights(cfg)
-    tables = W.make_tables(cfg, small["W_r"])
+    calib = getattr(cfg, "_calib", "auto")
+    small = W.make_small_weights(cfg, calib=calib)
+    tables = W.make_tables(cfg, small["W_r"], calib=calib)
     experts = W.make_expert_weights_device(cfg, device=device)
     tok = W.make_tokens(cfg)
     return small, tables, experts, tok
@@ -186,8 +205,7 @@ def run_reference(args):
     if rank != 0:
         return
     import torch
-    from paper_2608_00573_gb300 import workload as W
-    cfg = W.CONFIGS[args.config]
+    cfg = workload_config(args)
     device = "cuda" if torch.cuda.is_available() else "cpu"
     small, tables, experts, tok = make_workload(cfg, device)
     n_tok, n_layers = CPU_SAMPLE.get(cfg.name, (64, 2))
@@ -216,7 +234,7 @@ def run_ours(args):
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
     B.lib()
-    cfg = W.CONFIGS[args.config]
+    cfg = workload_config(args)
     T = cfg.T
     small, tables, experts, tok = make_workload(cfg, device)
     eng = B.Engine(cfg, tables, small, experts, T_max=T, device=device, profile=True)
@@ -342,6 +360,8 @@ def main():
     ap.add_argument("--config", default="mixtral")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0, help="profiling only: first N layers of the workload")
+    ap.add_argument("--tokens", type=int, default=0, help="profiling only: T tokens instead of the workload's")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
