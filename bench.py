@@ -313,7 +313,7 @@ def run_ours(args):
     per_fwd_flops = st["gemm_flops"] / args.steps
     fwd_roof_ms = per_fwd_flops / (peaks["bf16_sus"] * 1e12) * 1e3
     kernel_ms = {k: st[f"ms_{k}"] / args.steps for k in
-                 ("decide", "compact", "gather", "gemm_up", "gemm_down", "combine")}
+                 ("router", "decide", "compact", "gather", "gemm_up", "gemm_down", "combine")}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",

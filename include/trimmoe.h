@@ -185,6 +185,7 @@ typedef struct {
     double ms_decide, ms_compact, ms_gather, ms_gemm_up, ms_gemm_down, ms_combine;
     uint64_t n_gemm_up, n_gemm_down;
     double flops_gemm_up, flops_gemm_down;
+    double ms_router;             /* router / exit-head logits kernel (profile != 0) */
 } trimmoe_stats_t;
 
 /* Validate, copy the tables, derive the candidate lists V_{l,r} and losses Q,

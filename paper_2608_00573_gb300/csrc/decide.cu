@@ -1,15 +1,23 @@
-// Kernel (a): fused router + exit head + skip test + substitute-or-fetch with
-// server argmin and look-ahead + state update, one warp per live token.
+// Kernel (a): exit gate + skip test + substitute-or-fetch with server argmin and
+// look-ahead + state update, one warp per live token.
 //
 // Paper: Sec. V, Algorithm 2 lines 7-23.  Router and importance: Eq. (4);
 // exit confidence: Eq. (7)-(9); skip admission: Eq. (5), (34), (35); per-step
 // cost: Eq. (30)-(32); look-ahead cost-to-go: Eq. (38)-(39); choice: Eq. (40);
 // updates: Eq. (41)-(42).
 //
-// Every decision quantity after the dot products is fp32 with one fixed
-// operation order written with explicit round-to-nearest intrinsics (no fused
-// multiply-add), so that the integer outcomes are reproducible bit for bit.
-// Dot products accumulate in fp32 across lanes.
+// The router and exit-head logits come from kernel a0 (router.cu).  Every
+// decision quantity after them is fp32 with one fixed operation order written
+// with explicit round-to-nearest intrinsics (no fused multiply-add), so that the
+// integer outcomes are reproducible bit for bit.  The delay part of the execute
+// cost, omega_T * (d / d_ref), is read from a per-layer table computed at create
+// with the same operations.
+//
+// Look-ahead per future layer l': (1) one pass over the layer's candidates
+// stages, in shared memory, the feasibility (Q <= R), the quality term
+// omega_D * Q / Dbar and the deeper cost-to-go Phi(m_c, k_c) of each
+// candidate; (2) each (m, k') value is a minimum over its candidates of
+// table + staged terms; (3) Phi_{l'-1}(m, k) = sum_k' P(k -> k') V(m, k').
 #include <float.h>
 
 #include "internal.cuh"
@@ -56,60 +64,10 @@ __device__ __forceinline__ void warp_argmax(float& v, int& i) {
     }
 }
 
-__device__ __forceinline__ float dot8(const float (&h)[8], uint4 w) {
-    float a = 0.f;
-    a = fmaf(h[0], bf16_lo(w.x), a);
-    a = fmaf(h[1], bf16_hi(w.x), a);
-    a = fmaf(h[2], bf16_lo(w.y), a);
-    a = fmaf(h[3], bf16_hi(w.y), a);
-    a = fmaf(h[4], bf16_lo(w.z), a);
-    a = fmaf(h[5], bf16_hi(w.z), a);
-    a = fmaf(h[6], bf16_lo(w.w), a);
-    a = fmaf(h[7], bf16_hi(w.w), a);
-    return a;
-}
-
-// out[r] = dot(h_row * gamma, W[r]) * scale + b[r] for r < R (gamma may be NULL);
-// lanes split d in 16-byte chunks.
-__device__ void warp_gemv(const uint4* __restrict__ hrow, const __nv_bfloat16* __restrict__ gamma,
-                          const __nv_bfloat16* __restrict__ W, const float* __restrict__ b, int R,
-                          int d, int lane, float scale, float* out) {
-    const int nchunk = d >> 3;
-    for (int r0 = 0; r0 < R; r0 += 8) {
-        const int nr = min(8, R - r0);
-        float acc[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-        for (int c = lane; c < nchunk; c += 32) {
-            const uint4 hv = hrow[c];
-            float hf[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
-                           bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
-            if (gamma) {
-                const uint4 gv = __ldg(reinterpret_cast<const uint4*>(gamma) + c);
-                hf[0] *= bf16_lo(gv.x); hf[1] *= bf16_hi(gv.x); hf[2] *= bf16_lo(gv.y); hf[3] *= bf16_hi(gv.y);
-                hf[4] *= bf16_lo(gv.z); hf[5] *= bf16_hi(gv.z); hf[6] *= bf16_lo(gv.w); hf[7] *= bf16_hi(gv.w);
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if (i < nr) {
-                    const uint4 wv = __ldg(reinterpret_cast<const uint4*>(W + (size_t)(r0 + i) * d) + c);
-                    acc[i] += dot8(hf, wv);
-                }
-        }
-#pragma unroll
-        for (int i = 0; i < 8; ++i) acc[i] = warp_sum(acc[i]);
-        if (lane == 0)
-            for (int i = 0; i < nr; ++i) out[r0 + i] = __fadd_rn(__fmul_rn(acc[i], scale), b[r0 + i]);
-    }
-    __syncwarp();
-}
-
-// Per-step delay (Eq. 30) and execute cost (Eq. 31) from server s to m.
-__device__ __forceinline__ float exec_cost(const DecideParams& p, int l, int s, int m, float Q,
+// Execute cost f(m, k) of Eq. (31) from the delay table and the quality term.
+__device__ __forceinline__ float exec_cost(const DecideParams& p, const float* ct_row, int m, float Q,
                                            float Dbar) {
-    const float tr = (m != s) ? p.tab.trans[s * p.M + m] : 0.f;
-    const float dly = __fadd_rn(tr, p.tab.comp[l * p.M + m]);
-    float c = __fmul_rn(p.omega_T, __fdiv_rn(dly, p.d_ref));
+    float c = ct_row[m];
     if (Q > 0.f) c = __fadd_rn(c, __fmul_rn(p.omega_D, __fdiv_rn(Q, Dbar)));
     return c;
 }
@@ -127,13 +85,19 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
     const int warp = threadIdx.x >> 5;
     const int E = p.E, M = p.M, C = p.C, K = p.k, l = p.layer;
     const int ME = M * E;
+    const int MC = p.tab.max_layer_cand;
     // Per-warp scratch: logits z[E], probabilities pr[E], head logits x[C],
-    // look-ahead tables V[M*E] and Phi[M*E].
-    float* zs = smem + (size_t)warp * (2 * E + C + 2 * ME);
+    // look-ahead tables V[M*E] and Phi[M*E], staged candidate terms.
+    const size_t per_warp = (size_t)(2 * E + C + 2 * ME + 2 * MC) + (size_t)((MC + 3) / 4) * 2;
+    float* zs = smem + (size_t)warp * per_warp;
     float* ps = zs + E;
     float* xs = ps + E;
     float* bufV = xs + C;
     float* bufPhi = bufV + ME;
+    float* cqt = bufPhi + ME;                  // omega_D * Q / Dbar, or -1: no quality term
+    float* cph = cqt + MC;                     // deeper cost-to-go of the candidate
+    uint8_t* cok = reinterpret_cast<uint8_t*>(cph + MC);   // Q <= R
+    uint8_t* cmv = cok + ((MC + 3) & ~3);                  // server of the candidate
 
     __shared__ unsigned long long blk_cnt[9];
     __shared__ double blk_delay;
@@ -141,6 +105,9 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
     if (threadIdx.x < 9) blk_cnt[threadIdx.x] = 0ull;
     if (threadIdx.x == 0) { blk_delay = 0.0; blk_ratio = 0u; }
     __syncthreads();
+
+    const int* coff_l = p.tab.cand_off + l * (E + 1);
+    const float* ct_l = p.tab.ctab + (size_t)l * M * M;
 
     WarpCounters wc = {};
     const int nwarps = gridDim.x * kWarps;
@@ -164,28 +131,14 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         const float Dbar = p.Dbar[t];
         const float pJ = p.pJ[t];
         const int last_exec = p.last_exec[t];
-        const uint4* hrow = reinterpret_cast<const uint4*>(p.h + (size_t)t * p.d);
 
-        // Pre-FFN RMSNorm factor r = 1/sqrt(mean(h^2) + eps).
-        float rn = 1.f;
-        if (p.W_norm) {
-            float ss = 0.f;
-            for (int c = lane; c < (p.d >> 3); c += 32) {
-                const uint4 hv = hrow[c];
-                const float v[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
-                                    bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
-#pragma unroll
-                for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
-            }
-            ss = warp_sum(ss);
-            rn = rsqrtf(ss / (float)p.d + p.norm_eps);
-            if (lane == 0) p.rnorm[t] = rn;
+        // Router logits (kernel a0), softmax (Eq. 4), top-k by logit (a NaN
+        // logit ranks as -infinity).
+        const float* zrow = p.z + (size_t)t * p.zs;
+        for (int e = lane; e < E; e += 32) {
+            const float v = zrow[e];
+            zs[e] = (v != v) ? -kInf : v;
         }
-        // Router logits on the normalised state, softmax (Eq. 4), top-k by logit
-        // (a NaN logit ranks as -infinity).
-        warp_gemv(hrow, p.W_norm, p.W_r, p.b_r, E, p.d, lane, rn, zs);
-        for (int e = lane; e < E; e += 32)
-            if (zs[e] != zs[e]) zs[e] = -kInf;
         __syncwarp();
         float zmax = -FLT_MAX;
         for (int e = lane; e < E; e += 32) zmax = fmaxf(zmax, zs[e]);
@@ -217,9 +170,10 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
 
         // Exit confidence of the previous layer's head (Eq. 7), exit gate (Eq. 8-9).
         float xi = -1.f;
-        const bool have_xi = (l > 0) && last_exec && (p.W_x != nullptr);
+        const bool have_xi = (l > 0) && last_exec && p.has_head;
         if (have_xi) {
-            warp_gemv(hrow, nullptr, p.W_x, p.b_x, C, p.d, lane, rn, xs);
+            for (int c = lane; c < C; c += 32) xs[c] = zrow[E + c];
+            __syncwarp();
             if (C == 1) {
                 xi = __fdiv_rn(1.f, __fadd_rn(1.f, expf(-xs[0])));
             } else {
@@ -237,13 +191,12 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         // Transmission necessity (Eq. 35) over the budget-feasible candidates (Eq. 34).
         float Gamma = 0.f;
         for (int j = 0; j < K; ++j) {
-            const int base = (l * E + topk[j]) * kMaxCand;
-            const int n = p.tab.ncand[l * E + topk[j]];
+            const int c0 = coff_l[topk[j]], c1 = coff_l[topk[j] + 1];
             float gmin = kInf;
-            for (int c = lane; c < n; c += 32) {
-                const float Q = p.tab.cand_Q[base + c];
+            for (int c = c0 + lane; c < c1; c += 32) {
+                const float Q = p.tab.cand_Q[c];
                 if (__fadd_rn(Dhat, Q) <= Dbar) {
-                    const int m = p.tab.cand_m[base + c];
+                    const int m = p.tab.cand_m[c];
                     gmin = fminf(gmin, (m != s) ? p.tab.trans[s * M + m] : 0.f);
                 }
             }
@@ -259,29 +212,48 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         for (int jj = top; jj >= 1; --jj) {
             const int lp = l + jj;
             const float eps = p.tab.eps[lp];
+            const int* coff = p.tab.cand_off + lp * (E + 1);
+            const int cb = coff[0];
+            const int nc = coff[E] - cb;
+            // (1) per-candidate terms
+            for (int c = lane; c < nc; c += 32) {
+                const float Q = p.tab.cand_Q[cb + c];
+                const int mm = p.tab.cand_m[cb + c];
+                cok[c] = (Q <= R) ? 1 : 0;
+                cqt[c] = (Q > 0.f) ? __fmul_rn(p.omega_D, __fdiv_rn(Q, Dbar)) : -1.f;
+                cph[c] = have_phi ? bufPhi[mm * E + p.tab.cand_k[cb + c]] : 0.f;
+                cmv[c] = (uint8_t)mm;
+            }
+            __syncwarp();
+            // (2) V(m, k') = best next action from m for target k'
+            const float* ct = p.tab.ctab + (size_t)lp * M * M;
+            const float skip_cost = __fmul_rn(p.omega_D, __fdiv_rn(eps, Dbar));
+            const bool skip_budget = eps <= R;
             for (int idx = lane; idx < ME; idx += 32) {
                 const int m = idx / E, kp = idx - (idx / E) * E;
-                const int base = (lp * E + kp) * kMaxCand;
-                const int n = p.tab.ncand[lp * E + kp];
+                const int s0 = coff[kp] - cb, s1 = coff[kp + 1] - cb;
+                const float* ctm = ct + m * M;
                 float best = kInf;
                 bool local = false;
-                for (int c = 0; c < n; ++c) {
-                    const float Q = p.tab.cand_Q[base + c];
-                    if (!(Q <= R)) continue;
-                    const int mm = p.tab.cand_m[base + c];
-                    float v = exec_cost(p, lp, m, mm, Q, Dbar);
-                    if (have_phi) v = __fadd_rn(v, bufPhi[mm * E + p.tab.cand_k[base + c]]);
+                for (int c = s0; c < s1; ++c) {
+                    if (!cok[c]) continue;
+                    const int mm = cmv[c];
+                    float v = ctm[mm];
+                    const float q = cqt[c];
+                    if (q >= 0.f) v = __fadd_rn(v, q);
+                    if (have_phi) v = __fadd_rn(v, cph[c]);
                     best = fminf(best, v);
                     local |= (mm == m);
                 }
-                if (!local && eps <= R) {
-                    float v = __fmul_rn(p.omega_D, __fdiv_rn(eps, Dbar));
+                if (!local && skip_budget) {
+                    float v = skip_cost;
                     if (have_phi) v = __fadd_rn(v, bufPhi[m * E + kp]);
                     best = fminf(best, v);
                 }
                 bufV[idx] = best;
             }
             __syncwarp();
+            // (3) Phi_{l'-1}(m, k)
             const float* Pl = p.tab.P + (size_t)(lp - 1) * E * E;
             for (int idx = lane; idx < ME; idx += 32) {
                 const int m = idx / E, k = idx - (idx / E) * E;
@@ -296,28 +268,27 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         }
 
         // Execute plan: slot 0 by f + Phi, later slots by f (Eq. 40), budget by Eq. (34).
+        const float* ct_s = ct_l + s * M;
         int esel[kMaxK], msel[kMaxK];
         float Drun = Dhat, tot = 0.f;
         for (int j = 0; j < K; ++j) {
-            const int base = (l * E + topk[j]) * kMaxCand;
-            const int n = p.tab.ncand[l * E + topk[j]];
-            float bv = kInf, bf = 0.f;
+            const int c0 = coff_l[topk[j]], c1 = coff_l[topk[j] + 1];
+            float bv = kInf;
             int bi = 0x7fffffff;
-            for (int c = lane; c < n; c += 32) {
-                const float Q = p.tab.cand_Q[base + c];
+            for (int c = c0 + lane; c < c1; c += 32) {
+                const float Q = p.tab.cand_Q[c];
                 if (!(__fadd_rn(Dhat, Q) <= Dbar)) continue;
                 if (!(__fadd_rn(Drun, Q) <= Dbar)) continue;
-                const int m = p.tab.cand_m[base + c];
-                const float f = exec_cost(p, l, s, m, Q, Dbar);
+                const int m = p.tab.cand_m[c];
+                const float f = exec_cost(p, ct_s, m, Q, Dbar);
                 float v = f;
-                if (j == 0) v = __fadd_rn(f, have_phi ? bufPhi[m * E + p.tab.cand_k[base + c]] : 0.f);
-                if (v < bv) { bv = v; bi = c; bf = f; }
+                if (j == 0) v = __fadd_rn(f, have_phi ? bufPhi[m * E + p.tab.cand_k[c]] : 0.f);
+                if (v < bv) { bv = v; bi = c; }
             }
             warp_argmin(bv, bi);
-            bf = __shfl_sync(0xffffffffu, bf, bi & 31);
-            esel[j] = p.tab.cand_k[base + bi];
-            msel[j] = p.tab.cand_m[base + bi];
-            Drun = __fadd_rn(Drun, p.tab.cand_Q[base + bi]);
+            esel[j] = p.tab.cand_k[bi];
+            msel[j] = p.tab.cand_m[bi];
+            Drun = __fadd_rn(Drun, p.tab.cand_Q[bi]);
             tot = (j == 0) ? bv : __fadd_rn(tot, bv);
         }
         const float tot_exec = tot;
@@ -404,17 +375,23 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
 
 }  // namespace
 
+size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand) {
+    const size_t MC = (size_t)max_layer_cand;
+    const size_t per_warp = (size_t)(2 * E + C + 2 * M * E) + 2 * MC + ((MC + 3) / 4) * 2;
+    return per_warp * sizeof(float) * kWarps;
+}
+
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    const size_t per_warp = (size_t)(2 * p.E + p.C + 2 * p.M * p.E) * sizeof(float);
-    const size_t smem = per_warp * kWarps;
+    const size_t smem = decide_smem_bytes(p.E, p.C, p.M, p.tab.max_layer_cand);
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(decide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             96 * 1024);
+                                             200 * 1024);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
+    if (smem > 200 * 1024) return cudaErrorInvalidValue;
     int blocks = (p.T + kWarps - 1) / kWarps;
     blocks = blocks < num_sms * 16 ? blocks : num_sms * 16;
     decide_kernel<<<blocks, kWarps * 32, smem, st>>>(p);

@@ -37,10 +37,12 @@ struct DevCounters {
 
 // Per-layer decision tables on the device (built at create).
 struct DevTables {
-    const uint8_t* cand_m;   // [N][E][kMaxCand] server of candidate
-    const uint8_t* cand_k;   // [N][E][kMaxCand] expert of candidate
-    const float* cand_Q;     // [N][E][kMaxCand] substitution loss Q_l(r, k)
-    const int* ncand;        // [N][E]
+    const uint8_t* cand_m;   // flat candidate lists, all layers: server of candidate
+    const uint8_t* cand_k;   // expert of candidate
+    const float* cand_Q;     // substitution loss Q_l(r, k) (Eq. 3)
+    const int* cand_off;     // [N][E+1] start of target r's list in the flat arrays
+    const float* ctab;       // [N][M][M] omega_T * (d(m -> m') / d_ref) (Eq. 30-31)
+    int max_layer_cand;      // largest number of candidates of one layer
     const float* trans;      // [M][M]
     const float* comp;       // [N][M]
     const float* P;          // [N-1][E][E]
@@ -49,17 +51,30 @@ struct DevTables {
     const float* eps;        // [N]
 };
 
+// Router and exit-head logits of one layer (kernel a0).
+struct RouterParams {
+    int T, d;
+    int n_out;                  // E + C logits per token
+    int n_lo;                   // leading rows with a lo part (E)
+    int ng;                     // rows per pass (multiple of 8, <= 64)
+    int zs;                     // row stride of z
+    int use_norm;
+    float norm_eps;
+    const __nv_bfloat16* h;
+    const uint8_t* alive;
+    const __nv_bfloat16* Bhi;   // [n_out][d] hi(gamma * W_r) then W_x of the previous layer
+    const __nv_bfloat16* Blo;   // [E][d] lo(gamma * W_r)
+    const float* bias;          // [n_out]
+    float* z;                   // [T][zs]
+    float* rnorm;               // [T]
+};
+
 struct DecideParams {
     int layer, T, N, d, E, k, C, M, H;
     float omega_T, omega_D, d_ref;
-    const __nv_bfloat16* h;
-    const __nv_bfloat16* W_r;   // [E][d] of this layer
-    const float* b_r;
-    const __nv_bfloat16* W_x;   // [C][d] head of layer-1, NULL at layer 0
-    const float* b_x;
-    const __nv_bfloat16* W_norm;   // [d] RMSNorm weights of this layer, NULL = none
-    float norm_eps;
-    float* rnorm;               // [T] RMS factor r per token (written when W_norm)
+    const float* z;             // [T][zs] router logits then exit-head logits
+    int zs;
+    int has_head;               // exit head of the previous layer available (layer > 0)
     uint8_t* s;
     float* Dhat;
     const float* Dbar;
@@ -117,7 +132,11 @@ struct CombineParams {
 };
 
 // Launchers (one translation unit each).
+cudaError_t launch_router(const RouterParams& p, cudaStream_t st);
+size_t router_smem_bytes(int ng);
+int router_pass_rows(int n_out);
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
+size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand);
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);
 cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
                           const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,

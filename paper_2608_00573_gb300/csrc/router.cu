@@ -1,0 +1,205 @@
+// Kernel (a0): router and exit-head logits of a layer on the tensor cores.
+//
+//   z[t][e]     = r_t * sum_i h[t][i] * gamma_i * W_r[e][i] + b_r[e]     e < E   (Eq. 4 input)
+//   z[t][E + c] = r_t * sum_i h[t][i] * W_x[c][i]            + b_x[c]     c < C   (Eq. 7 input)
+// with r_t = 1/sqrt(mean_i h[t][i]^2 + eps) (1 without the pre-FFN RMSNorm).
+//
+// The router's gamma * W_r products are exact in fp32 and split exactly into
+// two bf16 matrices (hi + lo), so two bf16 MMAs give the logits without
+// rounding the normalised input.  Each 16-wide k step starts its MMA from zero
+// and its partial is added to IEEE fp32 registers (__fadd_rn): the tensor
+// core's own accumulation then only touches sums of 16-32 exact products, which
+// keeps the logits at fp32 accuracy (the decisions compare them to 1e-5).
+// mma.sync m16n8k16 (bf16 in, fp32 accumulate): the contraction is tiny (E + C
+// outputs per token) and the kernel is bound by streaming h from HBM, so the
+// tensor cores only remove the per-element unpack/FMA instruction cost.
+// One block = 64 tokens (4 warps x 16), d streamed in 64-column slabs through
+// a 4-stage cp.async ring in padded shared memory, ldmatrix fragments.
+// Dead tokens are zero-filled without reading HBM.
+#include "internal.cuh"
+
+namespace tmoe {
+
+namespace {
+
+constexpr int kTok = 64;
+constexpr int kKS = 64;
+constexpr int kPad = 72;          // padded smem row (bf16): conflict-free ldmatrix
+constexpr int kStages = 4;
+constexpr int kNG = 64;           // outputs per pass (8 n-tiles of 8)
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldmatrix_x2(uint32_t (&r)[2], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];"
+                 : "=r"(r[0]), "=r"(r[1])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+__global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
+    extern __shared__ __align__(16) uint8_t sm[];
+    const int NG = p.ng;                       // padded rows per pass (<= kNG, multiple of 8)
+    __nv_bfloat16* sA = reinterpret_cast<__nv_bfloat16*>(sm);
+    __nv_bfloat16* sBh = sA + kStages * kTok * kPad;
+    __nv_bfloat16* sBl = sBh + kStages * NG * kPad;
+    __shared__ float ssq[kTok];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int t0 = blockIdx.x * kTok;
+    const int nslab = p.d / kKS;
+    const int g = lane >> 2, tig = lane & 3;
+
+    for (int ng0 = 0; ng0 < p.n_out; ng0 += NG) {
+        const int nrows = min(NG, p.n_out - ng0);
+        const int ntile = (nrows + 7) >> 3;
+        const bool any_lo = ng0 < p.n_lo;
+        float sq = 0.f;
+        float acc[kNG / 8][4];
+#pragma unroll
+        for (int j = 0; j < kNG / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+
+        auto load_slab = [&](int s) {
+            const int buf = s % kStages;
+            for (int i = tid; i < kTok * (kKS / 8); i += 128) {
+                const int r = i >> 3, c = i & 7;
+                const int t = t0 + r;
+                const bool ok = t < p.T && p.alive[t];
+                const __nv_bfloat16* src = p.h + (size_t)(ok ? t : 0) * p.d + s * kKS + c * 8;
+                cp_async16(smem_u32(sA + (buf * kTok + r) * kPad + c * 8), src, ok ? 16 : 0);
+            }
+            for (int i = tid; i < NG * (kKS / 8); i += 128) {
+                const int r = i >> 3, c = i & 7;
+                const bool ok = r < nrows;
+                const size_t off = (size_t)(ng0 + (ok ? r : 0)) * p.d + s * kKS + c * 8;
+                cp_async16(smem_u32(sBh + (buf * NG + r) * kPad + c * 8), p.Bhi + off, ok ? 16 : 0);
+                if (any_lo) {
+                    const bool okl = ok && (ng0 + r) < p.n_lo;
+                    cp_async16(smem_u32(sBl + (buf * NG + r) * kPad + c * 8), p.Blo + off, okl ? 16 : 0);
+                }
+            }
+        };
+
+        for (int s = 0; s < kStages - 1; ++s) {
+            if (s < nslab) load_slab(s);
+            cp_async_commit();
+        }
+        for (int s = 0; s < nslab; ++s) {
+            cp_async_wait<kStages - 2>();
+            __syncthreads();
+            if (s + kStages - 1 < nslab) load_slab(s + kStages - 1);
+            cp_async_commit();
+            const int buf = s % kStages;
+            const __nv_bfloat16* A = sA + buf * kTok * kPad;
+            if (ng0 == 0) {                     // sum of squares for the RMS factor
+                const __nv_bfloat16* row = A + (tid >> 1) * kPad + (tid & 1) * 32;
+#pragma unroll
+                for (int q = 0; q < 32; q += 8) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(row + q);
+                    const float f[8] = {bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y),
+                                        bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w)};
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) sq = fmaf(f[u], f[u], sq);
+                }
+            }
+#pragma unroll
+            for (int kk = 0; kk < kKS / 16; ++kk) {
+                uint32_t a[4];
+                const int ar = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int ac = kk * 16 + (lane >> 4) * 8;
+                ldmatrix_x4(a, smem_u32(A + ar * kPad + ac));
+                const int br = (lane & 7);
+                const int bc = kk * 16 + ((lane >> 3) & 1) * 8;
+#pragma unroll
+                for (int j = 0; j < kNG / 8; ++j) {
+                    if (j < ntile) {
+                        uint32_t b[2];
+                        float part[4] = {0.f, 0.f, 0.f, 0.f};
+                        ldmatrix_x2(b, smem_u32(sBh + (buf * NG + j * 8 + br) * kPad + bc));
+                        mma_bf16_16816(part, a, b);
+                        if (ng0 + j * 8 < p.n_lo) {
+                            ldmatrix_x2(b, smem_u32(sBl + (buf * NG + j * 8 + br) * kPad + bc));
+                            mma_bf16_16816(part, a, b);
+                        }
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) acc[j][q] = __fadd_rn(acc[j][q], part[q]);
+                    }
+                }
+            }
+        }
+        cp_async_wait<0>();
+        if (ng0 == 0) {
+            sq += __shfl_xor_sync(0xffffffffu, sq, 1);
+            if ((tid & 1) == 0) ssq[tid >> 1] = sq;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int r = warp * 16 + g + half * 8;
+            const int t = t0 + r;
+            if (t >= p.T || !p.alive[t]) continue;
+            const float rn = p.use_norm ? rsqrtf(ssq[r] / (float)p.d + p.norm_eps) : 1.f;
+            if (ng0 == 0 && tig == 0 && p.use_norm) p.rnorm[t] = rn;
+            float* zrow = p.z + (size_t)t * p.zs;
+#pragma unroll
+            for (int j = 0; j < kNG / 8; ++j) {
+                if (j < ntile) {
+#pragma unroll
+                    for (int q = 0; q < 2; ++q) {
+                        const int col = ng0 + j * 8 + tig * 2 + q;
+                        if (col < p.n_out)
+                            zrow[col] = __fadd_rn(__fmul_rn(acc[j][half * 2 + q], rn), p.bias[col]);
+                    }
+                }
+            }
+        }
+        __syncthreads();
+    }
+}
+
+}  // namespace
+
+size_t router_smem_bytes(int ng) {
+    return (size_t)kStages * (kTok + 2 * ng) * kPad * sizeof(__nv_bfloat16);
+}
+
+int router_pass_rows(int n_out) {
+    const int r = ((n_out + 7) / 8) * 8;
+    return r < kNG ? r : kNG;
+}
+
+cudaError_t launch_router(const RouterParams& p, cudaStream_t st) {
+    if (p.T <= 0) return cudaSuccess;
+    if (p.d % kKS) return cudaErrorInvalidValue;
+    const size_t smem = router_smem_bytes(p.ng);
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(router_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)router_smem_bytes(kNG));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int blocks = (p.T + kTok - 1) / kTok;
+    router_kernel<<<blocks, 128, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace tmoe

@@ -53,7 +53,21 @@ bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_NUM };
+enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_NUM };
+
+inline float bf16_to_float(uint16_t b) {
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    std::memcpy(&f, &u, 4);
+    return f;
+}
+
+inline uint16_t float_to_bf16(float f) {   // round to nearest even (finite inputs)
+    uint32_t u;
+    std::memcpy(&u, &f, 4);
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
 
 struct DeviceGuard {
     int prev = -1;
@@ -85,7 +99,13 @@ struct trimmoe {
     uint8_t* cand_m = nullptr;
     uint8_t* cand_k = nullptr;
     float* cand_Q = nullptr;
-    int* ncand = nullptr;
+    int* cand_off = nullptr;
+    __nv_bfloat16* rt_hi = nullptr;   // [N][E+C][d] router (gamma folded, hi part) then exit head of layer-1
+    __nv_bfloat16* rt_lo = nullptr;   // [N][E][d] lo part of gamma * W_r
+    float* rt_bias = nullptr;         // [N][E+C]
+    float* zbuf = nullptr;            // [T_max][E+C] logits
+    float* ctab = nullptr;
+    int max_layer_cand = 1;
     float *trans = nullptr, *comp = nullptr, *P = nullptr, *theta = nullptr, *lambda = nullptr, *eps = nullptr;
 
     // workspaces
@@ -276,12 +296,16 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
 
     // Candidate lists V_{l,r} (Sec. III-A): the exact expert, then the n_sub
     // most similar experts with Sim >= sub_thresh (ties to the lower index),
-    // by expert index; servers ascending within an expert (Eq. 11).
-    std::vector<uint8_t> cm((size_t)N * E * kMaxCand, 0), ck((size_t)N * E * kMaxCand, 0);
-    std::vector<float> cq((size_t)N * E * kMaxCand, 0.f);
-    std::vector<int> nc((size_t)N * E, 0);
-    for (int l = 0; l < N; ++l)
+    // by expert index; servers ascending within an expert (Eq. 11).  Stored
+    // flat, layer after layer, with per-(layer, target) offsets.
+    std::vector<uint8_t> cm, ck;
+    std::vector<float> cq;
+    std::vector<int> coff((size_t)N * (E + 1), 0);
+    int max_layer_cand = 1;
+    for (int l = 0; l < N; ++l) {
+        const int layer_start = (int)cm.size();
         for (int r = 0; r < E; ++r) {
+            coff[(size_t)l * (E + 1) + r] = (int)cm.size();
             const float* srow = tab->sim + ((size_t)l * E + r) * E;
             std::vector<std::pair<float, int>> el;
             for (int k = 0; k < E; ++k)
@@ -293,20 +317,73 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
             for (size_t i = 0; i < el.size() && (int)i < c.n_sub; ++i) ex.push_back(el[i].second);
             std::sort(ex.begin(), ex.end());
             ex.insert(ex.begin(), r);
-            int n = 0;
-            const size_t base = ((size_t)l * E + r) * kMaxCand;
             for (int k : ex) {
                 const float q = (k == r) ? 0.0f : c.phi_beta * ((1.0f - srow[k]) / 2.0f);
                 for (int m = 0; m < M; ++m)
                     if ((tab->place[l * E + k] >> m) & 1u) {
-                        cm[base + n] = (uint8_t)m;
-                        ck[base + n] = (uint8_t)k;
-                        cq[base + n] = q;
-                        ++n;
+                        cm.push_back((uint8_t)m);
+                        ck.push_back((uint8_t)k);
+                        cq.push_back(q);
                     }
             }
-            nc[(size_t)l * E + r] = n;
         }
+        coff[(size_t)l * (E + 1) + E] = (int)cm.size();
+        max_layer_cand = std::max(max_layer_cand, (int)cm.size() - layer_start);
+    }
+    // Delay part of the execute cost, omega_T * (d(m -> m') / d_ref) with
+    // d(m -> m') = trans[m][m'] (m != m') + comp[l][m'] (Eq. 30-31), in fp32.
+    std::vector<float> ctab((size_t)N * M * M);
+    for (int l = 0; l < N; ++l)
+        for (int m = 0; m < M; ++m)
+            for (int mp = 0; mp < M; ++mp) {
+                const float tr = (mp != m) ? tab->trans_ms[m * M + mp] : 0.0f;
+                const float dly = tr + tab->comp_ms[l * M + mp];
+                ctab[((size_t)l * M + m) * M + mp] = c.omega_T * (dly / c.d_ref_ms);
+            }
+    if (decide_smem_bytes(E, c.C, M, max_layer_cand) > 200 * 1024) {
+        trimmoe_destroy(h);
+        return create_fail(TRIMMOE_ERR_UNSUPPORTED, "create: candidate lists too long for the decision kernel");
+    }
+    h->max_layer_cand = max_layer_cand;
+
+    // Router tables of kernel a0 (built from the borrowed device weights): per
+    // layer, rows [0, E) hold gamma_l * W_r[l] split exactly into bf16 hi + lo
+    // (a bf16 x bf16 product has at most 16 significant bits), rows [E, E+C) the
+    // exit head of layer l-1 (zero at layer 0); biases likewise.
+    const int n_out = E + c.C;
+    std::vector<uint16_t> hWr((size_t)N * E * d), hWx((size_t)N * c.C * d), hG;
+    std::vector<float> hbr((size_t)N * E), hbx((size_t)N * c.C);
+    {
+        cudaError_t e1 = cudaMemcpy(hWr.data(), w->W_r, hWr.size() * 2, cudaMemcpyDeviceToHost);
+        if (e1 == cudaSuccess) e1 = cudaMemcpy(hWx.data(), w->W_x, hWx.size() * 2, cudaMemcpyDeviceToHost);
+        if (e1 == cudaSuccess) e1 = cudaMemcpy(hbr.data(), w->b_r, hbr.size() * 4, cudaMemcpyDeviceToHost);
+        if (e1 == cudaSuccess) e1 = cudaMemcpy(hbx.data(), w->b_x, hbx.size() * 4, cudaMemcpyDeviceToHost);
+        if (e1 == cudaSuccess && w->W_norm) {
+            hG.resize((size_t)N * d);
+            e1 = cudaMemcpy(hG.data(), w->W_norm, hG.size() * 2, cudaMemcpyDeviceToHost);
+        }
+        if (e1 != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, std::string("create: reading router weights: ") + cudaGetErrorString(e1));
+    }
+    std::vector<uint16_t> rhi((size_t)N * n_out * d, 0), rlo((size_t)N * E * d, 0);
+    std::vector<float> rb((size_t)N * n_out, 0.f);
+    for (int l = 0; l < N; ++l) {
+        for (int e = 0; e < E; ++e) {
+            for (int i = 0; i < d; ++i) {
+                const float wv = bf16_to_float(hWr[((size_t)l * E + e) * d + i]);
+                const float prod = hG.empty() ? wv : wv * bf16_to_float(hG[(size_t)l * d + i]);
+                const uint16_t hi = float_to_bf16(prod);
+                const uint16_t lo = float_to_bf16(prod - bf16_to_float(hi));
+                rhi[((size_t)l * n_out + e) * d + i] = hi;
+                rlo[((size_t)l * E + e) * d + i] = lo;
+            }
+            rb[(size_t)l * n_out + e] = hbr[(size_t)l * E + e];
+        }
+        if (l > 0)
+            for (int cc = 0; cc < c.C; ++cc) {
+                std::memcpy(&rhi[((size_t)l * n_out + E + cc) * d], &hWx[((size_t)(l - 1) * c.C + cc) * d], (size_t)d * 2);
+                rb[(size_t)l * n_out + E + cc] = hbx[(size_t)(l - 1) * c.C + cc];
+            }
+    }
 
     // Device tables and workspaces.
     const size_t T = (size_t)c.T_max, TK = T * c.k;
@@ -314,7 +391,10 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     h->rows_xp = (int)(TK + (has_sh ? T : 0));
     const int nblk = (int)((T + 255) / 256);
     bool ok = h->dalloc(&h->cand_m, cm.size()) && h->dalloc(&h->cand_k, ck.size()) &&
-              h->dalloc(&h->cand_Q, cq.size()) && h->dalloc(&h->ncand, nc.size()) &&
+              h->dalloc(&h->cand_Q, cq.size()) && h->dalloc(&h->cand_off, coff.size()) &&
+              h->dalloc(&h->ctab, ctab.size()) && h->dalloc(&h->rt_hi, rhi.size()) &&
+              h->dalloc(&h->rt_lo, rlo.size()) && h->dalloc(&h->rt_bias, rb.size()) &&
+              h->dalloc(&h->zbuf, T * (size_t)n_out) &&
               h->dalloc(&h->trans, (size_t)M * M) && h->dalloc(&h->comp, (size_t)N * M) &&
               h->dalloc(&h->P, (size_t)std::max(N - 1, 1) * E * E) && h->dalloc(&h->theta, N) &&
               h->dalloc(&h->lambda, N) && h->dalloc(&h->eps, N) && h->dalloc(&h->topk_idx, TK) &&
@@ -335,7 +415,11 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     up(h->cand_m, cm.data(), cm.size());
     up(h->cand_k, ck.data(), ck.size());
     up(h->cand_Q, cq.data(), cq.size() * 4);
-    up(h->ncand, nc.data(), nc.size() * 4);
+    up(h->cand_off, coff.data(), coff.size() * 4);
+    up(h->ctab, ctab.data(), ctab.size() * 4);
+    up(h->rt_hi, rhi.data(), rhi.size() * 2);
+    up(h->rt_lo, rlo.data(), rlo.size() * 2);
+    up(h->rt_bias, rb.data(), rb.size() * 4);
     up(h->trans, tab->trans_ms, (size_t)M * M * 4);
     up(h->comp, tab->comp_ms, (size_t)N * M * 4);
     if (N > 1) up(h->P, tab->P, (size_t)(N - 1) * E * E * 4);
@@ -399,16 +483,31 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.omega_T = c.omega_T;
     dp.omega_D = c.omega_D;
     dp.d_ref = c.d_ref_ms;
-    dp.h = static_cast<const __nv_bfloat16*>(tok->hidden);
-    dp.W_r = static_cast<const __nv_bfloat16*>(h->w.W_r) + (size_t)layer * E * d;
-    dp.b_r = h->w.b_r + (size_t)layer * E;
-    dp.W_x = layer > 0 ? static_cast<const __nv_bfloat16*>(h->w.W_x) + (size_t)(layer - 1) * c.C * d : nullptr;
-    dp.b_x = layer > 0 ? h->w.b_x + (size_t)(layer - 1) * c.C : nullptr;
+    const __nv_bfloat16* hid = static_cast<const __nv_bfloat16*>(tok->hidden);
     const __nv_bfloat16* gamma =
         h->w.W_norm ? static_cast<const __nv_bfloat16*>(h->w.W_norm) + (size_t)layer * d : nullptr;
-    dp.W_norm = gamma;
-    dp.norm_eps = c.norm_eps;
-    dp.rnorm = h->rnorm;
+    const int n_out = E + c.C;
+    RouterParams rp;
+    rp.T = T;
+    rp.d = d;
+    rp.n_out = n_out;
+    rp.n_lo = E;
+    rp.ng = router_pass_rows(n_out);
+    rp.zs = n_out;
+    rp.use_norm = gamma != nullptr;
+    rp.norm_eps = c.norm_eps;
+    rp.h = hid;
+    rp.alive = tok->alive;
+    rp.Bhi = h->rt_hi + (size_t)layer * n_out * d;
+    rp.Blo = h->rt_lo + (size_t)layer * E * d;
+    rp.bias = h->rt_bias + (size_t)layer * n_out;
+    rp.z = h->zbuf;
+    rp.rnorm = h->rnorm;
+    cudaError_t e = h->timed(K_ROUTER, st, [&] { return launch_router(rp, st); });
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("router: ") + cudaGetErrorString(e));
+    dp.z = h->zbuf;
+    dp.zs = n_out;
+    dp.has_head = layer > 0;
     dp.s = tok->s;
     dp.Dhat = tok->Dhat;
     dp.Dbar = tok->Dbar;
@@ -427,7 +526,9 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.tab.cand_m = h->cand_m;
     dp.tab.cand_k = h->cand_k;
     dp.tab.cand_Q = h->cand_Q;
-    dp.tab.ncand = h->ncand;
+    dp.tab.cand_off = h->cand_off;
+    dp.tab.ctab = h->ctab;
+    dp.tab.max_layer_cand = h->max_layer_cand;
     dp.tab.trans = h->trans;
     dp.tab.comp = h->comp;
     dp.tab.P = h->P;
@@ -436,7 +537,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.tab.eps = h->eps;
     dp.ctr = h->ctr;
 
-    cudaError_t e = h->timed(K_DECIDE, st, [&] { return launch_decide(dp, h->num_sms, st); });
+    e = h->timed(K_DECIDE, st, [&] { return launch_decide(dp, h->num_sms, st); });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("decide: ") + cudaGetErrorString(e));
 
     CompactParams cp;
@@ -458,7 +559,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("compact: ") + cudaGetErrorString(e));
     const int max_rows = T * K + (has_sh ? T : 0);
     e = h->timed(K_GATHER, st, [&] {
-        return launch_gather(h->perm, h->goff, E, K, d, dp.h, h->rnorm, gamma, h->Xp, max_rows, h->num_sms, st);
+        return launch_gather(h->perm, h->goff, E, K, d, hid, h->rnorm, gamma, h->Xp, max_rows, h->num_sms, st);
     });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gather: ") + cudaGetErrorString(e));
 
@@ -492,7 +593,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm down: ") + cudaGetErrorString(e));
     h->n_gemm_up++;
     h->n_gemm_down++;
-    h->launches += 7;
+    h->launches += 8;
     if (has_sh) {
         GemmLaunch s1 = g1;
         s1.tmB = &h->tmW13sh[layer];
@@ -529,7 +630,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     bp.k = K;
     bp.renorm = c.renorm_topk;
     bp.has_shared = has_sh;
-    bp.h = static_cast<__nv_bfloat16*>(tok->hidden);
+    bp.h = static_cast<__nv_bfloat16*>(tok->hidden);  // combine writes h in place
     bp.action = dp.action;
     bp.topk_g = dp.topk_g;
     bp.pos_pair = h->pos_pair;
@@ -667,6 +768,7 @@ extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) 
     out->ms_gemm_up = h->ms[K_GEMM_UP];
     out->ms_gemm_down = h->ms[K_GEMM_DOWN];
     out->ms_combine = h->ms[K_COMBINE];
+    out->ms_router = h->ms[K_ROUTER];
     out->n_gemm_up = h->n_gemm_up;
     out->n_gemm_down = h->n_gemm_down;
     if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "stats: a kernel timed out waiting");
