@@ -132,11 +132,22 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         const float pJ = p.pJ[t];
         const int last_exec = p.last_exec[t];
 
-        // Router logits (kernel a0), softmax (Eq. 4), top-k by logit (a NaN
-        // logit ranks as -infinity).
-        const float* zrow = p.z + (size_t)t * p.zs;
+        // Router logits: partial dot products of kernel a0 summed over the column
+        // ranges in order, times the RMS factor, plus the bias; softmax (Eq. 4),
+        // top-k by logit (a NaN logit ranks as -infinity).
+        float rn = 1.f;
+        if (p.use_norm) {
+            float sq = 0.f;
+            for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart[(size_t)ks * p.T + t]);
+            rn = rsqrtf(sq / (float)p.d + p.norm_eps);
+            if (lane == 0) p.rnorm[t] = rn;
+        }
+        const size_t kstride = (size_t)p.T * p.zs;
+        const float* zrow = p.zpart + (size_t)t * p.zs;
         for (int e = lane; e < E; e += 32) {
-            const float v = zrow[e];
+            float acc = 0.f;
+            for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + e]);
+            const float v = __fadd_rn(__fmul_rn(acc, rn), p.bias[e]);
             zs[e] = (v != v) ? -kInf : v;
         }
         __syncwarp();
@@ -172,7 +183,11 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         float xi = -1.f;
         const bool have_xi = (l > 0) && last_exec && p.has_head;
         if (have_xi) {
-            for (int c = lane; c < C; c += 32) xs[c] = zrow[E + c];
+            for (int c = lane; c < C; c += 32) {
+                float acc = 0.f;
+                for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + c]);
+                xs[c] = __fadd_rn(__fmul_rn(acc, rn), p.bias[E + c]);
+            }
             __syncwarp();
             if (C == 1) {
                 xi = __fdiv_rn(1.f, __fadd_rn(1.f, expf(-xs[0])));

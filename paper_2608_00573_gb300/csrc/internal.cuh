@@ -51,29 +51,33 @@ struct DevTables {
     const float* eps;        // [N]
 };
 
-// Router and exit-head logits of one layer (kernel a0).
+// Router and exit-head partial logits of one layer (kernel a0), split over d:
+// block (x, y) covers tokens [64x, 64x+64) and columns [y*d/ksplit, (y+1)*d/ksplit).
 struct RouterParams {
     int T, d;
     int n_out;                  // E + C logits per token
     int n_lo;                   // leading rows with a lo part (E)
     int ng;                     // rows per pass (multiple of 8, <= 64)
-    int zs;                     // row stride of z
-    int use_norm;
-    float norm_eps;
+    int zs;                     // row stride of zpart
+    int ksplit;                 // number of column ranges
     const __nv_bfloat16* h;
     const uint8_t* alive;
     const __nv_bfloat16* Bhi;   // [n_out][d] hi(gamma * W_r) then W_x of the previous layer
     const __nv_bfloat16* Blo;   // [E][d] lo(gamma * W_r)
-    const float* bias;          // [n_out]
-    float* z;                   // [T][zs]
-    float* rnorm;               // [T]
+    float* zpart;               // [ksplit][T][zs] partial dot products
+    float* sqpart;              // [ksplit][T] partial sums of h^2
 };
 
 struct DecideParams {
     int layer, T, N, d, E, k, C, M, H;
     float omega_T, omega_D, d_ref;
-    const float* z;             // [T][zs] router logits then exit-head logits
-    int zs;
+    const float* zpart;         // [ksplit][T][zs] partial router then exit-head dot products
+    const float* sqpart;        // [ksplit][T] partial sums of h^2
+    const float* bias;          // [E + C] router then exit-head biases of this layer
+    int zs, ksplit;
+    int use_norm;
+    float norm_eps;
+    float* rnorm;               // [T] RMS factor r (written when use_norm)
     int has_head;               // exit head of the previous layer available (layer > 0)
     uint8_t* s;
     float* Dhat;
@@ -135,6 +139,7 @@ struct CombineParams {
 cudaError_t launch_router(const RouterParams& p, cudaStream_t st);
 size_t router_smem_bytes(int ng);
 int router_pass_rows(int n_out);
+int router_ksplit(int T, int d, int num_sms);
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand);
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);

@@ -1,8 +1,12 @@
-// Kernel (a0): router and exit-head logits of a layer on the tensor cores.
+// Kernel (a0): router and exit-head dot products of a layer on the tensor cores.
 //
 //   z[t][e]     = r_t * sum_i h[t][i] * gamma_i * W_r[e][i] + b_r[e]     e < E   (Eq. 4 input)
 //   z[t][E + c] = r_t * sum_i h[t][i] * W_x[c][i]            + b_x[c]     c < C   (Eq. 7 input)
 // with r_t = 1/sqrt(mean_i h[t][i]^2 + eps) (1 without the pre-FFN RMSNorm).
+// The columns i are split into ksplit ranges, one per blockIdx.y, so that the
+// grid covers every SM several times even for small token counts; each block
+// writes its partial sums (and partial sums of h^2), and the decision kernel
+// adds the ranges in a fixed order before applying r and the bias.
 //
 // The router's gamma * W_r products are exact in fp32 and split exactly into
 // two bf16 matrices (hi + lo), so two bf16 MMAs give the logits without
@@ -65,7 +69,11 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
     __shared__ float ssq[kTok];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int t0 = blockIdx.x * kTok;
-    const int nslab = p.d / kKS;
+    const int nslab_all = p.d / kKS;
+    const int nslab = nslab_all / p.ksplit;
+    const int slab0 = blockIdx.y * nslab;
+    float* zpart = p.zpart + (size_t)blockIdx.y * p.T * p.zs;
+    float* sqpart = p.sqpart + (size_t)blockIdx.y * p.T;
     const int g = lane >> 2, tig = lane & 3;
 
     for (int ng0 = 0; ng0 < p.n_out; ng0 += NG) {
@@ -79,17 +87,18 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
 
         auto load_slab = [&](int s) {
             const int buf = s % kStages;
+            const int sg = slab0 + s;                 // global slab index
             for (int i = tid; i < kTok * (kKS / 8); i += 128) {
                 const int r = i >> 3, c = i & 7;
                 const int t = t0 + r;
                 const bool ok = t < p.T && p.alive[t];
-                const __nv_bfloat16* src = p.h + (size_t)(ok ? t : 0) * p.d + s * kKS + c * 8;
+                const __nv_bfloat16* src = p.h + (size_t)(ok ? t : 0) * p.d + sg * kKS + c * 8;
                 cp_async16(smem_u32(sA + (buf * kTok + r) * kPad + c * 8), src, ok ? 16 : 0);
             }
             for (int i = tid; i < NG * (kKS / 8); i += 128) {
                 const int r = i >> 3, c = i & 7;
                 const bool ok = r < nrows;
-                const size_t off = (size_t)(ng0 + (ok ? r : 0)) * p.d + s * kKS + c * 8;
+                const size_t off = (size_t)(ng0 + (ok ? r : 0)) * p.d + sg * kKS + c * 8;
                 cp_async16(smem_u32(sBh + (buf * NG + r) * kPad + c * 8), p.Bhi + off, ok ? 16 : 0);
                 if (any_lo) {
                     const bool okl = ok && (ng0 + r) < p.n_lo;
@@ -156,17 +165,15 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
             const int r = warp * 16 + g + half * 8;
             const int t = t0 + r;
             if (t >= p.T || !p.alive[t]) continue;
-            const float rn = p.use_norm ? rsqrtf(ssq[r] / (float)p.d + p.norm_eps) : 1.f;
-            if (ng0 == 0 && tig == 0 && p.use_norm) p.rnorm[t] = rn;
-            float* zrow = p.z + (size_t)t * p.zs;
+            if (ng0 == 0 && tig == 0) sqpart[t] = ssq[r];
+            float* zrow = zpart + (size_t)t * p.zs;
 #pragma unroll
             for (int j = 0; j < kNG / 8; ++j) {
                 if (j < ntile) {
 #pragma unroll
                     for (int q = 0; q < 2; ++q) {
                         const int col = ng0 + j * 8 + tig * 2 + q;
-                        if (col < p.n_out)
-                            zrow[col] = __fadd_rn(__fmul_rn(acc[j][half * 2 + q], rn), p.bias[col]);
+                        if (col < p.n_out) zrow[col] = acc[j][half * 2 + q];
                     }
                 }
             }
@@ -181,6 +188,16 @@ size_t router_smem_bytes(int ng) {
     return (size_t)kStages * (kTok + 2 * ng) * kPad * sizeof(__nv_bfloat16);
 }
 
+// Column ranges per launch: a power of two dividing d/64, chosen so that the
+// grid has at least about four blocks per SM.
+int router_ksplit(int T, int d, int num_sms) {
+    const int nslab = d / kKS;
+    const int tiles = (T + kTok - 1) / kTok;
+    int ks = 1;
+    while (ks < nslab && (long long)tiles * ks < 4ll * num_sms && nslab % (ks * 2) == 0) ks *= 2;
+    return ks;
+}
+
 int router_pass_rows(int n_out) {
     const int r = ((n_out + 7) / 8) * 8;
     return r < kNG ? r : kNG;
@@ -188,7 +205,7 @@ int router_pass_rows(int n_out) {
 
 cudaError_t launch_router(const RouterParams& p, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    if (p.d % kKS) return cudaErrorInvalidValue;
+    if (p.d % kKS || p.ksplit < 1 || (p.d / kKS) % p.ksplit) return cudaErrorInvalidValue;
     const size_t smem = router_smem_bytes(p.ng);
     static bool attr_set = false;
     if (!attr_set) {
@@ -197,8 +214,8 @@ cudaError_t launch_router(const RouterParams& p, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    const int blocks = (p.T + kTok - 1) / kTok;
-    router_kernel<<<blocks, 128, smem, st>>>(p);
+    const dim3 grid((p.T + kTok - 1) / kTok, p.ksplit);
+    router_kernel<<<grid, 128, smem, st>>>(p);
     return cudaGetLastError();
 }
 

@@ -103,7 +103,9 @@ struct trimmoe {
     __nv_bfloat16* rt_hi = nullptr;   // [N][E+C][d] router (gamma folded, hi part) then exit head of layer-1
     __nv_bfloat16* rt_lo = nullptr;   // [N][E][d] lo part of gamma * W_r
     float* rt_bias = nullptr;         // [N][E+C]
-    float* zbuf = nullptr;            // [T_max][E+C] logits
+    float* zbuf = nullptr;            // [rows_part][E+C] partial logits
+    float* sqbuf = nullptr;           // [rows_part] partial sums of squares
+    size_t rows_part = 0;             // max over T <= T_max of ksplit(T) * T
     float* ctab = nullptr;
     int max_layer_cand = 1;
     float *trans = nullptr, *comp = nullptr, *P = nullptr, *theta = nullptr, *lambda = nullptr, *eps = nullptr;
@@ -385,6 +387,9 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
             }
     }
 
+    for (int tt = 1; tt <= c.T_max; ++tt)
+        h->rows_part = std::max(h->rows_part, (size_t)router_ksplit(tt, d, h->num_sms) * tt);
+
     // Device tables and workspaces.
     const size_t T = (size_t)c.T_max, TK = T * c.k;
     const int has_sh = c.F_sh > 0;
@@ -394,7 +399,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->cand_Q, cq.size()) && h->dalloc(&h->cand_off, coff.size()) &&
               h->dalloc(&h->ctab, ctab.size()) && h->dalloc(&h->rt_hi, rhi.size()) &&
               h->dalloc(&h->rt_lo, rlo.size()) && h->dalloc(&h->rt_bias, rb.size()) &&
-              h->dalloc(&h->zbuf, T * (size_t)n_out) &&
+              h->dalloc(&h->zbuf, h->rows_part * (size_t)n_out) && h->dalloc(&h->sqbuf, h->rows_part) &&
               h->dalloc(&h->trans, (size_t)M * M) && h->dalloc(&h->comp, (size_t)N * M) &&
               h->dalloc(&h->P, (size_t)std::max(N - 1, 1) * E * E) && h->dalloc(&h->theta, N) &&
               h->dalloc(&h->lambda, N) && h->dalloc(&h->eps, N) && h->dalloc(&h->topk_idx, TK) &&
@@ -494,19 +499,23 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     rp.n_lo = E;
     rp.ng = router_pass_rows(n_out);
     rp.zs = n_out;
-    rp.use_norm = gamma != nullptr;
-    rp.norm_eps = c.norm_eps;
+    rp.ksplit = router_ksplit(T, d, h->num_sms);
     rp.h = hid;
     rp.alive = tok->alive;
     rp.Bhi = h->rt_hi + (size_t)layer * n_out * d;
     rp.Blo = h->rt_lo + (size_t)layer * E * d;
-    rp.bias = h->rt_bias + (size_t)layer * n_out;
-    rp.z = h->zbuf;
-    rp.rnorm = h->rnorm;
+    rp.zpart = h->zbuf;
+    rp.sqpart = h->sqbuf;
     cudaError_t e = h->timed(K_ROUTER, st, [&] { return launch_router(rp, st); });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("router: ") + cudaGetErrorString(e));
-    dp.z = h->zbuf;
+    dp.zpart = h->zbuf;
+    dp.sqpart = h->sqbuf;
+    dp.bias = h->rt_bias + (size_t)layer * n_out;
     dp.zs = n_out;
+    dp.ksplit = rp.ksplit;
+    dp.use_norm = gamma != nullptr;
+    dp.norm_eps = c.norm_eps;
+    dp.rnorm = h->rnorm;
     dp.has_head = layer > 0;
     dp.s = tok->s;
     dp.Dhat = tok->Dhat;
