@@ -224,6 +224,38 @@ const char* trimmoe_last_error(trimmoe_handle h);
 /* Free the handle and its workspaces (synchronises first).  NULL is a no-op. */
 void trimmoe_destroy(trimmoe_handle h);
 
+/* Runtime feedback between forwards (Alg. 2 line 27): the exit-threshold
+ * update of Eq. (37) and the dual-weight update of Eq. (43).
+ *  user_size: users are blocks of user_size consecutive tokens (Eq. 33);
+ *  eta, p_min: step and floor of Eq. (37); kappa: step of Eq. (43). */
+typedef struct {
+    int user_size;
+    float eta, p_min, kappa;
+} trimmoe_feedback_cfg;
+
+typedef struct {
+    float omega_T, omega_D;       /* weights after the update (used by later calls) */
+    double T_norm;                /* observed normalised delay of the window */
+    double D_util;                /* observed budget utilisation of the window */
+    int users_updated;            /* users whose p_J moved (had exits in the window) */
+    double window_delay_ms;       /* summed per-step delay d(m,k) of the window's executions */
+    double window_ref_slots;      /* token x layer x slot count of the window's calls */
+} trimmoe_feedback_out;
+
+/* End an observation window.  For each user with exits in the window (tokens
+ * with alive == 0 and exit_layer < N; xi_last is the confidence that admitted
+ * the exit), every token's pJ (device, in place) becomes
+ * clamp(pJ + eta * (mean exit confidence - pJ), p_min, 1)  (Eq. 37).
+ * D_util = mean over users of sum(Dhat)/sum(Dbar); T_norm = window delay /
+ * (window_ref_slots * d_ref), the window's delay over the full-depth exact
+ * reference; omega_D = clamp(omega_D + kappa * (D_util - T_norm), 0, 1),
+ * omega_T = 1 - omega_D (Eq. 43); the handle uses the new weights from the
+ * next call on.  The window is everything since the previous trimmoe_feedback
+ * or trimmoe_reset_stats; call it after a forward and before the token state is
+ * re-initialised.  Synchronises the stream.  ERR_ARG on a bad configuration. */
+trimmoe_status trimmoe_feedback(trimmoe_handle h, const trimmoe_feedback_cfg* fb, int T, trimmoe_tokens* tok,
+                                trimmoe_feedback_out* out, void* stream);
+
 /* Compaction of one layer's decisions without any device allocation (the
  * paper has no counterpart: this entry point exists for callers that cannot
  * call cudaMalloc, e.g. code running inside an allocator callback or in a

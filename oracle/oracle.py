@@ -68,6 +68,15 @@ class OrDecision(C.Structure):
                 ("f_sel", C.c_float * 16), ("Dhat_new", C.c_float), ("s_new", C.c_int), ("near", C.c_int)]
 
 
+class OrFeedbackCfg(C.Structure):
+    _fields_ = [("user_size", C.c_int), ("eta", C.c_float), ("p_min", C.c_float), ("kappa", C.c_float)]
+
+
+class OrFeedbackOut(C.Structure):
+    _fields_ = [("omega_T", C.c_float), ("omega_D", C.c_float), ("T_norm", C.c_double),
+                ("D_util", C.c_double), ("users_updated", C.c_int)]
+
+
 def lib():
     global _lib
     with _lock:
@@ -96,6 +105,8 @@ def lib():
             L.or_forward.argtypes = [vp, vp, i, vp, vp, i]
             L.or_forward.restype = i
             L.or_max_threads.restype = i
+            L.or_feedback.argtypes = [vp, i, i, vp, vp, vp, vp, vp, vp, C.c_double, C.c_double, f, f, vp]
+            L.or_feedback.restype = i
             _lib = L
     return _lib
 
@@ -274,3 +285,20 @@ def ffn_row(d, F, act, W13_e, W2_e, x):
 
 def max_threads():
     return int(lib().or_max_threads())
+
+
+def feedback(tok, N, user_size, eta, p_min, kappa, delay_sum_ms, ref_slots, d_ref, omega_D):
+    """Eq. (37) and (43) on host arrays; returns (new pJ, OrFeedbackOut)."""
+    T = len(tok["pJ"])
+    pJ = np.array(tok["pJ"], dtype=np.float32, copy=True)
+    arr = {k: np.ascontiguousarray(tok[k], dtype=dt) for k, dt in
+           (("alive", np.uint8), ("exit_layer", np.int16), ("xi_last", np.float32), ("Dhat", np.float32),
+            ("Dbar", np.float32))}
+    cfg = OrFeedbackCfg(user_size=user_size, eta=eta, p_min=p_min, kappa=kappa)
+    out = OrFeedbackOut()
+    rc = lib().or_feedback(C.byref(cfg), T, N, _p(pJ), _p(arr["alive"]), _p(arr["exit_layer"]), _p(arr["xi_last"]),
+                           _p(arr["Dhat"]), _p(arr["Dbar"]), C.c_double(delay_sum_ms), C.c_double(ref_slots),
+                           C.c_float(d_ref), C.c_float(omega_D), C.byref(out))
+    if rc:
+        raise RuntimeError("or_feedback failed")
+    return pJ, out

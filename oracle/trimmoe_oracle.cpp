@@ -617,6 +617,68 @@ int or_forward(const OrModel* md, const OrLayerWeights* lws, int T, uint16_t* h,
     return 0;
 }
 
+// ------------------------------------------------------- runtime feedback
+
+typedef struct {
+    int user_size;      // tokens per user (consecutive blocks)
+    float eta;          // step of Eq. (37)
+    float p_min;        // floor of the projection in Eq. (37)
+    float kappa;        // step of Eq. (43)
+} OrFeedbackCfg;
+
+typedef struct {
+    float omega_T, omega_D;
+    double T_norm, D_util;
+    int users_updated;
+} OrFeedbackOut;
+
+// Feedback at the end of an observation window (Alg. 2 line 27).
+// Eq. (37): for every user with exits in the window, p_J <- clamp(p_J +
+// eta * (xi_exit_mean - p_J), p_min, 1), where xi_exit_mean is the mean exit
+// confidence of the user's exited tokens.  Eq. (43): omega_D <- clamp(omega_D
+// + kappa * (D_util - T_norm), 0, 1), omega_T = 1 - omega_D, where D_util is the
+// mean over users of sum(Dhat) / sum(Dbar) and T_norm is the window's summed
+// per-step delay over its full-depth exact reference (ref_slots * d_ref).
+int or_feedback(const OrFeedbackCfg* fb, int T, int N, float* pJ, const uint8_t* alive,
+                const int16_t* exit_layer, const float* xi_last, const float* Dhat, const float* Dbar,
+                double delay_sum_ms, double ref_slots, float d_ref, float omega_D, OrFeedbackOut* out) {
+    if (!fb || fb->user_size < 1 || T < 0) return -1;
+    const int us = fb->user_size;
+    const int users = (T + us - 1) / us;
+    double util_sum = 0.0;
+    int updated = 0;
+    for (int u = 0; u < users; ++u) {
+        const int t0 = u * us, t1 = std::min(T, t0 + us);
+        double xs = 0.0, dh = 0.0, db = 0.0;
+        int n = 0;
+        for (int t = t0; t < t1; ++t) {
+            if (!alive[t] && exit_layer[t] < N) { xs += (double)xi_last[t]; ++n; }
+            dh += (double)Dhat[t];
+            db += (double)Dbar[t];
+        }
+        if (n > 0) {
+            const float xbar = (float)(xs / n);
+            for (int t = t0; t < t1; ++t) {
+                float q = pJ[t] + fb->eta * (xbar - pJ[t]);
+                q = std::min(std::max(q, fb->p_min), 1.0f);
+                pJ[t] = q;
+            }
+            ++updated;
+        }
+        util_sum += (db > 0.0) ? dh / db : 0.0;
+    }
+    const double D_util = users > 0 ? util_sum / users : 0.0;
+    const double T_norm = (ref_slots > 0.0) ? delay_sum_ms / (ref_slots * (double)d_ref) : 0.0;
+    double wD = (double)omega_D + (double)fb->kappa * (D_util - T_norm);
+    wD = std::min(std::max(wD, 0.0), 1.0);
+    out->omega_D = (float)wD;
+    out->omega_T = 1.0f - out->omega_D;
+    out->T_norm = T_norm;
+    out->D_util = D_util;
+    out->users_updated = updated;
+    return 0;
+}
+
 int or_max_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();

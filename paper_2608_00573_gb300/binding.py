@@ -73,9 +73,21 @@ class trimmoe_stats_t(C.Structure):
         return {n: getattr(self, n) for n, _ in self._fields_}
 
 
+class trimmoe_feedback_cfg(C.Structure):
+    _fields_ = [("user_size", C.c_int), ("eta", C.c_float), ("p_min", C.c_float), ("kappa", C.c_float)]
+
+
+class trimmoe_feedback_out(C.Structure):
+    _fields_ = [("omega_T", C.c_float), ("omega_D", C.c_float), ("T_norm", C.c_double), ("D_util", C.c_double),
+                ("users_updated", C.c_int), ("window_delay_ms", C.c_double), ("window_ref_slots", C.c_double)]
+
+    def as_dict(self):
+        return {n: getattr(self, n) for n, _ in self._fields_}
+
+
 EXPORTS = ("trimmoe_create", "trimmoe_layer_step", "trimmoe_forward", "trimmoe_forward_host",
            "trimmoe_stats", "trimmoe_reset_stats", "trimmoe_last_error", "trimmoe_destroy",
-           "trimmoe_compact_noalloc")
+           "trimmoe_compact_noalloc", "trimmoe_feedback")
 
 _lib = None
 _lock = threading.Lock()
@@ -108,6 +120,8 @@ def lib():
             L.trimmoe_destroy.argtypes = [vp]
             L.trimmoe_destroy.restype = None
             L.trimmoe_compact_noalloc.argtypes = [vp, vp, i, i, i, i, vp, vp, vp, vp, vp]
+            L.trimmoe_feedback.argtypes = [vp, vp, i, vp, vp, vp]
+            L.trimmoe_feedback.restype = i
             L.trimmoe_compact_noalloc.restype = i
             _lib = L
     return _lib
@@ -160,6 +174,12 @@ def trimmoe_last_error(h=None) -> str:
 
 def trimmoe_destroy(h):
     lib().trimmoe_destroy(h)
+
+
+def trimmoe_feedback(h, fb: trimmoe_feedback_cfg, T: int, tok: trimmoe_tokens, stream: int = 0) -> dict:
+    out = trimmoe_feedback_out()
+    _check(lib().trimmoe_feedback(h, C.byref(fb), T, C.byref(tok), C.byref(out), C.c_void_p(stream)), h)
+    return out.as_dict()
 
 
 def trimmoe_compact_noalloc(action, exp_sel, T: int, k: int, E: int, has_shared: int, perm, group_off,
@@ -296,6 +316,13 @@ class Engine:
 
     def stats(self) -> dict:
         return trimmoe_stats(self.handle)
+
+    def feedback(self, tok: dict, user_size: int, eta: float, p_min: float, kappa: float,
+                 T: Optional[int] = None, stream=None) -> dict:
+        """Eq. (37) / (43) at the end of an observation window (updates tok['pJ'] in place)."""
+        T = tok["s"].shape[0] if T is None else T
+        fb = trimmoe_feedback_cfg(user_size=user_size, eta=eta, p_min=p_min, kappa=kappa)
+        return trimmoe_feedback(self.handle, fb, T, self.c_tokens(tok), self.stream_ptr(stream))
 
     def reset_stats(self):
         trimmoe_reset_stats(self.handle)

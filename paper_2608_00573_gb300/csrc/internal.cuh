@@ -135,6 +135,20 @@ struct CombineParams {
     const __nv_bfloat16* Ysh;
 };
 
+struct FeedbackParams {
+    int T, N, user_size, users;
+    float eta, p_min;
+    float* pJ;
+    const uint8_t* alive;
+    const int16_t* exit_layer;
+    const float* xi_last;
+    const float* Dhat;
+    const float* Dbar;
+    double* util;       // [users]
+    int* updated;       // [users]
+    double* result;     // [2]: mean utilisation, users updated
+};
+
 // Launchers (one translation unit each).
 cudaError_t launch_router(const RouterParams& p, cudaStream_t st);
 size_t router_smem_bytes(int ng);
@@ -149,6 +163,7 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st);
 size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
+cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
 
 // Error text for calls made without a handle (read by trimmoe_last_error(NULL)).
 void set_global_error(const std::string& msg);

@@ -132,6 +132,13 @@ struct trimmoe {
     // host-buffer forward
     trimmoe_tokens dtok = {};
 
+    // runtime feedback: host copies of the delay tables, window counters, scratch
+    std::vector<float> h_trans, h_comp;
+    double win_delay0 = 0.0, win_ref_slots = 0.0;
+    double* fb_util = nullptr;
+    int* fb_updated = nullptr;
+    double* fb_result = nullptr;
+
     // counters kept on the host
     uint64_t launches = 0, layer_calls = 0;
 
@@ -199,6 +206,22 @@ struct trimmoe {
 };
 
 namespace {
+
+// Delay part of the execute cost, omega_T * (d(m -> m') / d_ref) with
+// d(m -> m') = trans[m][m'] (m != m') + comp[l][m'] (Eq. 30-31), in fp32.
+std::vector<float> delay_cost_table(const trimmoe_config& c, const std::vector<float>& trans,
+                                    const std::vector<float>& comp) {
+    const int N = c.N, M = c.M;
+    std::vector<float> ctab((size_t)N * M * M);
+    for (int l = 0; l < N; ++l)
+        for (int m = 0; m < M; ++m)
+            for (int mp = 0; mp < M; ++mp) {
+                const float tr = (mp != m) ? trans[(size_t)m * M + mp] : 0.0f;
+                const float dly = tr + comp[(size_t)l * M + mp];
+                ctab[((size_t)l * M + m) * M + mp] = c.omega_T * (dly / c.d_ref_ms);
+            }
+    return ctab;
+}
 
 trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
     if (c->N < 1 || c->d < 1 || c->E < 1 || c->k < 1 || c->F < 1 || c->M < 1 || c->H < 1 || c->C < 1 ||
@@ -332,16 +355,9 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         coff[(size_t)l * (E + 1) + E] = (int)cm.size();
         max_layer_cand = std::max(max_layer_cand, (int)cm.size() - layer_start);
     }
-    // Delay part of the execute cost, omega_T * (d(m -> m') / d_ref) with
-    // d(m -> m') = trans[m][m'] (m != m') + comp[l][m'] (Eq. 30-31), in fp32.
-    std::vector<float> ctab((size_t)N * M * M);
-    for (int l = 0; l < N; ++l)
-        for (int m = 0; m < M; ++m)
-            for (int mp = 0; mp < M; ++mp) {
-                const float tr = (mp != m) ? tab->trans_ms[m * M + mp] : 0.0f;
-                const float dly = tr + tab->comp_ms[l * M + mp];
-                ctab[((size_t)l * M + m) * M + mp] = c.omega_T * (dly / c.d_ref_ms);
-            }
+    h->h_trans.assign(tab->trans_ms, tab->trans_ms + (size_t)M * M);
+    h->h_comp.assign(tab->comp_ms, tab->comp_ms + (size_t)N * M);
+    std::vector<float> ctab = delay_cost_table(c, h->h_trans, h->h_comp);
     if (decide_smem_bytes(E, c.C, M, max_layer_cand) > 200 * 1024) {
         trimmoe_destroy(h);
         return create_fail(TRIMMOE_ERR_UNSUPPORTED, "create: candidate lists too long for the decision kernel");
@@ -410,7 +426,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->goff, (size_t)E + 2) && h->dalloc(&h->blk_counts, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->blk_base, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
-              h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, 1) && h->dalloc(&h->dev_err, 1);
+              h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, 1) && h->dalloc(&h->dev_err, 1) &&
+              h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2);
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
     if (!ok) return bail(TRIMMOE_ERR_OOM, "create: device allocation failed");
     cudaError_t ce = cudaSuccess;
@@ -659,6 +676,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "copy group_off failed");
     }
     h->layer_calls++;
+    h->win_ref_slots += (double)T * K;
     return TRIMMOE_OK;
 }
 
@@ -795,6 +813,69 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
         return h->fail(TRIMMOE_ERR_CUDA, "reset: memset failed");
     for (double& m : h->ms) m = 0.0;
     h->launches = h->layer_calls = h->n_gemm_up = h->n_gemm_down = 0;
+    h->win_delay0 = 0.0;
+    h->win_ref_slots = 0.0;
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_feedback(trimmoe_handle h, const trimmoe_feedback_cfg* fb, int T,
+                                           trimmoe_tokens* tok, trimmoe_feedback_out* out, void* stream) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    if (!fb || !out) return h->fail(TRIMMOE_ERR_ARG, "feedback: NULL argument");
+    if (fb->user_size < 1 || !(fb->eta >= 0.f) || !std::isfinite(fb->eta) || !(fb->p_min >= 0.f) ||
+        !(fb->p_min <= 1.f) || !(fb->kappa >= 0.f) || !std::isfinite(fb->kappa))
+        return h->fail(TRIMMOE_ERR_ARG, "feedback: need user_size >= 1, eta >= 0, 0 <= p_min <= 1, kappa >= 0");
+    if (T < 0 || T > h->cfg.T_max) return h->fail(TRIMMOE_ERR_ARG, "feedback: T outside [0, T_max]");
+    trimmoe_status s = check_tokens(h, tok);
+    if (s != TRIMMOE_OK) return s;
+    DeviceGuard g(h->dev);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    h->last_stream = st;
+    FeedbackParams p;
+    p.T = T;
+    p.N = h->cfg.N;
+    p.user_size = fb->user_size;
+    p.users = (T + fb->user_size - 1) / fb->user_size;
+    p.eta = fb->eta;
+    p.p_min = fb->p_min;
+    p.pJ = tok->pJ;
+    p.alive = tok->alive;
+    p.exit_layer = tok->exit_layer;
+    p.xi_last = tok->xi_last;
+    p.Dhat = tok->Dhat;
+    p.Dbar = tok->Dbar;
+    p.util = h->fb_util;
+    p.updated = h->fb_updated;
+    p.result = h->fb_result;
+    cudaError_t e = launch_feedback(p, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    double res[2] = {0.0, 0.0};
+    DevCounters dc;
+    if (e == cudaSuccess) e = cudaMemcpy(res, h->fb_result, sizeof res, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemcpy(&dc, h->ctr, sizeof dc, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("feedback: ") + cudaGetErrorString(e));
+    const double window_delay = dc.delay_ms - h->win_delay0;
+    const double ref = h->win_ref_slots;
+    const double D_util = res[0];
+    const double T_norm = (ref > 0.0) ? window_delay / (ref * (double)h->cfg.d_ref_ms) : 0.0;
+    double wD = (double)h->cfg.omega_D + (double)fb->kappa * (D_util - T_norm);
+    wD = std::min(std::max(wD, 0.0), 1.0);
+    trimmoe_config c2 = h->cfg;
+    c2.omega_D = (float)wD;
+    c2.omega_T = 1.0f - c2.omega_D;
+    const std::vector<float> ctab = delay_cost_table(c2, h->h_trans, h->h_comp);
+    e = cudaMemcpy(h->ctab, ctab.data(), ctab.size() * sizeof(float), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "feedback: table upload failed");
+    h->cfg = c2;
+    h->win_delay0 = dc.delay_ms;
+    h->win_ref_slots = 0.0;
+    out->omega_T = c2.omega_T;
+    out->omega_D = c2.omega_D;
+    out->T_norm = T_norm;
+    out->D_util = D_util;
+    out->users_updated = (int)res[1];
+    out->window_delay_ms = window_delay;
+    out->window_ref_slots = ref;
     return TRIMMOE_OK;
 }
 

@@ -39,8 +39,9 @@ def test_header_struct_sizes_match_binding():
     src = r'''
 #include <stdio.h>
 #include "trimmoe.h"
-int main(){printf("%zu %zu %zu %zu %zu %zu\n", sizeof(trimmoe_config), sizeof(trimmoe_weights),
- sizeof(trimmoe_tables), sizeof(trimmoe_tokens), sizeof(trimmoe_layer_out), sizeof(trimmoe_stats_t));}
+int main(){printf("%zu %zu %zu %zu %zu %zu %zu %zu\n", sizeof(trimmoe_config), sizeof(trimmoe_weights),
+ sizeof(trimmoe_tables), sizeof(trimmoe_tokens), sizeof(trimmoe_layer_out), sizeof(trimmoe_stats_t),
+ sizeof(trimmoe_feedback_cfg), sizeof(trimmoe_feedback_out));}
 '''
     import subprocess
     import tempfile
@@ -52,7 +53,8 @@ int main(){printf("%zu %zu %zu %zu %zu %zu\n", sizeof(trimmoe_config), sizeof(tr
         subprocess.check_call(["gcc", "-I", os.path.join(ROOT, "include"), p, "-o", exe])
         got = [int(x) for x in subprocess.check_output([exe]).split()]
     want = [C.sizeof(x) for x in (B.trimmoe_config, B.trimmoe_weights, B.trimmoe_tables, B.trimmoe_tokens,
-                                  B.trimmoe_layer_out, B.trimmoe_stats_t)]
+                                  B.trimmoe_layer_out, B.trimmoe_stats_t, B.trimmoe_feedback_cfg,
+                                  B.trimmoe_feedback_out)]
     assert got == want
 
 
