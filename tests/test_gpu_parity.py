@@ -220,3 +220,29 @@ def test_create_rejects_bad_input():
     with pytest.raises(B.TrimmoeError):
         eng.layer_step(0, tok, T=17)
     eng.close()
+
+
+@pytest.mark.parametrize("name,kw", [
+    ("E128_k8_C256_H6", dict(N=4, d=256, E=128, k=8, F=128, C=256, M=8, H=6, T=300, zipf_s=0.5)),
+    ("M16_E64_k8_shared", dict(N=3, d=512, E=64, k=8, F=256, F_sh=128, M=16, H=3, T=257)),
+])
+def test_layer_parity_at_maximum_dimensions(name, kw):
+    """The largest E, k, M, C and H the library accepts (E <= 128, k <= 8, M <= 16,
+    C <= 256, H <= 6, M*E <= 1024)."""
+    cfg = small_cfg(name=name, seed=91, **kw)
+    reports = _run_all_layers(cfg, theta=0.95, exit_bias=1.0 if cfg.C == 1 else 8.0)
+    tot = {k: sum(r[k] for r in reports) for k in ("exec", "skip", "exit")}
+    print(name, tot)
+    assert tot["exec"] > 0
+
+
+@pytest.mark.parametrize("budget", [0.0, float("inf")])
+def test_budget_edge_cases(budget):
+    """Dbar = 0: only exact execution fits (Q = 0), no skip; Dbar = inf: every
+    substitute and skip fits and Q / Dbar = 0."""
+    cfg = small_cfg(name="budget", N=3, d=256, E=8, k=2, F=256, T=300, M=10, seed=93)
+    def mut(tok):
+        tok["Dbar"][:] = budget
+    reports = _run_all_layers(cfg, mutate_tokens=mut, theta=0.95, exit_bias=1.0)
+    if budget == 0.0:
+        assert sum(r["skip"] for r in reports) == 0
