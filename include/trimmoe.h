@@ -195,13 +195,13 @@ typedef struct {
 trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmoe_weights* w,
                               const trimmoe_tables* tab, trimmoe_handle* out);
 
-/* One MoE layer over tokens [0, T) (Alg. 2, lines 6-25, plus the gated FFN and
+/* One MoE layer over tokens [0, T) (the per-layer body of Algorithm 2, plus the gated FFN and
  * combine).  Dead tokens are untouched.  0 <= layer < N, 0 <= T <= T_max.
  * out may be NULL.  Asynchronous on stream. */
 trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T, trimmoe_tokens* tok,
                                   trimmoe_layer_out* out, void* stream);
 
-/* Layers 0..N-1 in order (Alg. 2, lines 5-26).  Asynchronous on stream. */
+/* Layers 0..N-1 in order (the layer loop of Algorithm 2).  Asynchronous on stream. */
 trimmoe_status trimmoe_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream);
 
 /* trimmoe_forward on HOST buffers: copies hidden and the token state to device
@@ -224,7 +224,7 @@ const char* trimmoe_last_error(trimmoe_handle h);
 /* Free the handle and its workspaces (synchronises first).  NULL is a no-op. */
 void trimmoe_destroy(trimmoe_handle h);
 
-/* Runtime feedback between forwards (Alg. 2 line 27): the exit-threshold
+/* Runtime feedback between forwards (the periodic update of Algorithm 2): the exit-threshold
  * update of Eq. (37) and the dual-weight update of Eq. (43).
  *  user_size: users are blocks of user_size consecutive tokens (Eq. 33);
  *  eta, p_min: step and floor of Eq. (37); kappa: step of Eq. (43). */

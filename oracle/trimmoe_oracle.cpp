@@ -362,7 +362,7 @@ static float value_naive(const OrModel* md, int lp, int h, int m, int kp, float 
 
 // ------------------------------------------------------------ the decision
 
-// One token, one layer: Alg. 2, lines 7-23, given the routing (topk, g, I) and
+// One token, one layer: the per-token body of Algorithm 2, given the routing (topk, g, I) and
 // the exit confidence xi (negative when not evaluated).
 void or_decide_given(const OrModel* md, int l, const int* topk, const float* g, float I, float xi,
                      int s, float Dhat, float Dbar, float pJ, int last_exec, OrDecision* out) {
@@ -497,7 +497,7 @@ void or_ffn_row(int d, int F, int act, const uint16_t* W13, const uint16_t* W2, 
 
 // ---------------------------------------------------------------- layer step
 
-// One MoE layer over T tokens (Alg. 2 lines 6-25 plus the MoE computation the
+// One MoE layer over T tokens (the per-layer body of Algorithm 2 plus the MoE computation the
 // decisions gate).  h is bf16 [T][d], updated in place.  row_mask (may be NULL)
 // limits the FFN/combine to the selected tokens; decisions, state and
 // compaction are always computed for every token.
@@ -607,7 +607,7 @@ int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uin
     return 0;
 }
 
-// Whole forward: layers 0..N-1 (Alg. 2 lines 5-26).
+// Whole forward: layers 0..N-1 (the layer loop of Algorithm 2).
 int or_forward(const OrModel* md, const OrLayerWeights* lws, int T, uint16_t* h, OrTokens* tk,
                int nthreads) {
     for (int l = 0; l < md->N; ++l) {
@@ -632,7 +632,7 @@ typedef struct {
     int users_updated;
 } OrFeedbackOut;
 
-// Feedback at the end of an observation window (Alg. 2 line 27).
+// Feedback at the end of an observation window (the periodic update of Algorithm 2).
 // Eq. (37): for every user with exits in the window, p_J <- clamp(p_J +
 // eta * (xi_exit_mean - p_J), p_min, 1), where xi_exit_mean is the mean exit
 // confidence of the user's exited tokens.  Eq. (43): omega_D <- clamp(omega_D

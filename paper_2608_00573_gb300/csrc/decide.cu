@@ -1,7 +1,7 @@
 // Kernel (a): exit gate + skip test + substitute-or-fetch with server argmin and
 // look-ahead + state update, one warp per live token.
 //
-// Paper: Sec. V, Algorithm 2 lines 7-23.  Router and importance: Eq. (4);
+// Paper: Sec. V, the per-token body of Algorithm 2.  Router and importance: Eq. (4);
 // exit confidence: Eq. (7)-(9); skip admission: Eq. (5), (34), (35); per-step
 // cost: Eq. (30)-(32); look-ahead cost-to-go: Eq. (38)-(39); choice: Eq. (40);
 // updates: Eq. (41)-(42).

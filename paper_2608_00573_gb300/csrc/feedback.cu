@@ -1,4 +1,4 @@
-// Runtime feedback between forwards (Alg. 2 line 27).
+// Runtime feedback between forwards (the periodic update of Algorithm 2, Sec. V-D/V-F).
 //
 // Eq. (37): for every user (a block of user_size consecutive tokens) with exits
 // in the observation window, p_J <- clamp(p_J + eta * (mean exit confidence -

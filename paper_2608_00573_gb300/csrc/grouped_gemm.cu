@@ -7,7 +7,7 @@
 // with epilogue = store (down projection), SwiGLU over the interleaved
 // gate/up columns (W13 of a SwiGLU expert) or ReLU (W1 of a ReLU expert).
 // This is the only dense contraction of the layer step (the expert FFN of the
-// executed layers, Sec. III-B/C, Alg. 2 line 17).
+// executed layers, Sec. III-B/C and the execute branch of Algorithm 2).
 //
 // Design (one CTA per SM, persistent, 192 threads):
 //   warp 0      TMA producer (one lane); also owns the TMEM allocation

@@ -2,7 +2,7 @@
 // candidate lists V_{l,r} with their losses Q (Eq. 3), workspaces, TMA
 // descriptors, and the per-layer launch sequence
 //   decide -> compact -> gather -> FFN gate/up -> FFN down -> combine
-// (Alg. 2 lines 6-25 plus the MoE computation they gate).
+// (the per-layer body of Algorithm 2 plus the MoE computation it gates).
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
