@@ -141,6 +141,8 @@ def workload_config(args):
     """The named workload; --layers / --tokens shrink it for profiling runs."""
     from paper_2608_00573_gb300 import workload as W
     cfg = W.CONFIGS[args.config]
+    if args.exit_prediction:
+        cfg = cfg.replace(n_centroids=args.exit_prediction)
     if args.layers or args.tokens:
         over = {}
         if args.layers:
@@ -319,7 +321,8 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": cfg.name, "T": T, "N": cfg.N, "d": cfg.d, "E": cfg.E, "k": cfg.k, "F": cfg.F,
-                   "F_sh": cfg.F_sh, "H": cfg.H, "budget": cfg.budget, "parallelism": f"replicas{world}",
+                   "F_sh": cfg.F_sh, "H": cfg.H, "budget": cfg.budget, "exit_prediction_centroids": cfg.n_centroids,
+                   "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (expert weights and hidden states)"},
         "roofline": roof,
         "forward_roofline": {"gemm_flops_per_forward": per_fwd_flops, "roofline_ms": fwd_roof_ms,
@@ -362,6 +365,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=0, help="profiling only: first N layers of the workload")
     ap.add_argument("--tokens", type=int, default=0, help="profiling only: T tokens instead of the workload's")
+    ap.add_argument("--exit-prediction", type=int, default=0,
+                    help="K_c centroids per layer for the token-similarity exit prediction (Eq. 36); 0 = off")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -62,7 +62,9 @@ enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
  *  phi_beta: Q = phi_beta * (1 - Sim)/2 (Eq. 3 with a linear phi);
  *  profile: 1 = record CUDA events around each kernel launch (trimmoe_stats
  *  then reports per-kernel device time);
- *  norm_eps: epsilon of the pre-FFN RMSNorm (used when W_norm != NULL).
+ *  norm_eps: epsilon of the pre-FFN RMSNorm (used when W_norm != NULL);
+ *  n_centroids: K_c centroids per layer for the token-similarity exit-point
+ *  prediction of Eq. (36) (0 = off, at most 256).
  * Supported: d % 256 == 0; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
  * F_sh % 128 == 0; E <= 128; k <= min(E, 8); C <= 256; M*E <= 1024; H <= 6;
  * n_sub <= 3. */
@@ -75,6 +77,7 @@ typedef struct {
     float omega_T, omega_D, d_ref_ms, phi_beta;
     int profile;
     float norm_eps;
+    int n_centroids;
 } trimmoe_config;
 
 /* Weights (device, bf16 except the biases, borrowed; 16-byte aligned).
@@ -88,7 +91,9 @@ typedef struct {
  *  W_norm [N][d] weights gamma_l of the MoE sublayer's pre-FFN RMSNorm, or NULL
  *       for none.  With it, layer l computes r = 1/sqrt(mean(h^2) + norm_eps);
  *       the router reads h*r*gamma_l (fp32), the experts its bf16 rounding, the
- *       exit head h*r, and the combine adds to h itself (pre-norm residual). */
+ *       exit head h*r, and the combine adds to h itself (pre-norm residual).
+ *  centroids [N][K_c][d] (n_centroids > 0): representations entering layer l
+ *       of the token-similarity reference set (Eq. 36); read at create. */
 typedef struct {
     const void* W_r;
     const float* b_r;
@@ -99,6 +104,7 @@ typedef struct {
     const void* W13_sh;
     const void* W2_sh;
     const void* W_norm;
+    const void* centroids;
 } trimmoe_weights;
 
 /* The paper's input tables (host, copied at create).
@@ -122,6 +128,7 @@ typedef struct {
     const float* theta;
     const float* lambda;
     const float* eps;
+    const float* centroid_exit;
 } trimmoe_tables;
 
 /* Per-token state (device, borrowed, length >= T; updated in place).
@@ -150,7 +157,9 @@ typedef struct {
  *  perm int32 [T*k + T]: the executed pairs t*k+j ordered by (expert, t, j),
  *  then the tokens that run the shared expert (executed or skipped) by t;
  *  group_off int32 [E+2]: pairs of expert e are perm[group_off[e] ..
- *  group_off[e+1]), shared rows perm[group_off[E] .. group_off[E+1]). */
+ *  group_off[e+1]), shared rows perm[group_off[E] .. group_off[E+1]);
+ *  lhat int16 [T]: predicted exit layer (Eq. 36; N without prediction, -1 for
+ *  dead tokens). */
 typedef struct {
     int32_t* topk_idx;
     float* topk_g;
@@ -161,6 +170,7 @@ typedef struct {
     uint8_t* srv_sel;
     int32_t* perm;
     int32_t* group_off;
+    int16_t* lhat;
 } trimmoe_layer_out;
 
 /* Counters accumulated since create / the last reset (Fig. 5(b) categories). */

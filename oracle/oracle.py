@@ -41,12 +41,13 @@ class OrModel(C.Structure):
                [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref", "phi_beta", "norm_eps")] + [
         ("place", C.c_void_p), ("sim", C.c_void_p), ("sub_thresh", C.c_void_p),
         ("trans", C.c_void_p), ("comp", C.c_void_p), ("P", C.c_void_p), ("theta", C.c_void_p),
-        ("lambda_", C.c_void_p), ("eps", C.c_void_p)]
+        ("lambda_", C.c_void_p), ("eps", C.c_void_p), ("n_centroids", C.c_int)]
 
 
 class OrLayerWeights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in
-                ("W_r", "b_r", "W_x_prev", "b_x_prev", "W13", "W2", "W13_sh", "W2_sh", "W_norm")]
+                ("W_r", "b_r", "W_x_prev", "b_x_prev", "W13", "W2", "W13_sh", "W2_sh", "W_norm",
+                 "centroids", "centroid_exit")]
 
 
 class OrTokens(C.Structure):
@@ -57,7 +58,7 @@ class OrTokens(C.Structure):
 class OrLayerOut(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in
                 ("topk_idx", "topk_g", "I", "xi", "action", "exp_sel", "srv_sel", "perm",
-                 "group_off", "near", "Gamma", "tot_exec", "tot_skip")]
+                 "group_off", "near", "Gamma", "tot_exec", "tot_skip", "lhat")]
 
 
 class OrDecision(C.Structure):
@@ -65,7 +66,8 @@ class OrDecision(C.Structure):
                [(n, C.c_float) for n in ("I", "xi", "Gamma", "tot_exec", "tot_skip", "Lambda")] + \
                [(n, C.c_int) for n in ("action", "skip_ok", "exit_ok")] + \
                [("exp_sel", C.c_int * 16), ("srv_sel", C.c_int * 16), ("Q_sel", C.c_float * 16),
-                ("f_sel", C.c_float * 16), ("Dhat_new", C.c_float), ("s_new", C.c_int), ("near", C.c_int)]
+                ("f_sel", C.c_float * 16), ("Dhat_new", C.c_float), ("s_new", C.c_int), ("near", C.c_int),
+                ("Lhat", C.c_int)]
 
 
 class OrFeedbackCfg(C.Structure):
@@ -95,6 +97,9 @@ def lib():
             L.or_exec_cost.argtypes = [vp, i, i, i, f, f]
             L.or_exec_cost.restype = f
             L.or_lookahead_table.argtypes = [vp, i, f, f, vp]
+            L.or_lookahead_table_capped.argtypes = [vp, i, f, f, i, vp]
+            L.or_predict_exit.argtypes = [vp, vp, vp, vp, vp, vp]
+            L.or_predict_exit.restype = i
             L.or_phi_naive.argtypes = [vp, i, i, i, i, f, f]
             L.or_phi_naive.restype = f
             L.or_decide_given.argtypes = [vp, i, vp, vp, f, f, i, f, f, f, i, vp]
@@ -136,7 +141,7 @@ class OracleModel:
             trans=_p(keep("trans", t["trans"], np.float32)), comp=_p(keep("comp", t["comp"], np.float32)),
             P=_p(keep("P", t["P"] if t["P"].size else np.zeros((1, cfg.E, cfg.E)), np.float32)),
             theta=_p(keep("theta", t["theta"], np.float32)), lambda_=_p(keep("lam", t["lam"], np.float32)),
-            eps=_p(keep("eps", t["eps"], np.float32)))
+            eps=_p(keep("eps", t["eps"], np.float32)), n_centroids=cfg.n_centroids)
         self.small = {k: (None if v is None else np.ascontiguousarray(v)) for k, v in small.items()}
         self.experts = experts   # dict of numpy arrays (bf16 bits) per layer or full, or None
 
@@ -152,10 +157,15 @@ class OracleModel:
         wx = np.ascontiguousarray(s["W_x"][l - 1], dtype=np.uint16) if l > 0 else None
         bx = np.ascontiguousarray(s["b_x"][l - 1], dtype=np.float32) if l > 0 else None
         wn = np.ascontiguousarray(s["W_norm"][l], dtype=np.uint16) if s.get("W_norm") is not None else None
+        cc = ce = None
+        if self.cfg.n_centroids and s.get("centroids") is not None:
+            cc = np.ascontiguousarray(s["centroids"][l], dtype=np.uint16)
+            ce = np.ascontiguousarray(s["centroid_exit"][l], dtype=np.float32)
         lw = OrLayerWeights(W_r=_p(wr), b_r=_p(br), W_x_prev=_p(wx), b_x_prev=_p(bx),
                             W13=_p(ex.get("W13")), W2=_p(ex.get("W2")),
-                            W13_sh=_p(ex.get("W13_sh")), W2_sh=_p(ex.get("W2_sh")), W_norm=_p(wn))
-        lw._keep = (wr, br, wx, bx, ex, wn)
+                            W13_sh=_p(ex.get("W13_sh")), W2_sh=_p(ex.get("W2_sh")), W_norm=_p(wn),
+                            centroids=_p(cc), centroid_exit=_p(ce))
+        lw._keep = (wr, br, wx, bx, ex, wn, cc, ce)
         return lw
 
 
@@ -182,7 +192,7 @@ def alloc_layer_out(T, cfg):
         exp_sel=np.zeros(T * K, np.uint8), srv_sel=np.zeros(T * K, np.uint8),
         perm=np.full(T * K + T, -1, np.int32), group_off=np.zeros(E + 2, np.int32),
         near=np.zeros(T, np.uint8), Gamma=np.zeros(T, np.float32), tot_exec=np.zeros(T, np.float32),
-        tot_skip=np.zeros(T, np.float32))
+        tot_skip=np.zeros(T, np.float32), lhat=np.zeros(T, np.int16))
     return OrLayerOut(**{k: _p(v) for k, v in o.items()}), o
 
 
@@ -259,6 +269,21 @@ def lookahead_table(om, l, R, Dbar):
     out = np.zeros(om.cfg.M * om.cfg.E, np.float32)
     lib().or_lookahead_table(C.byref(om.m), l, C.c_float(R), C.c_float(Dbar), _p(out))
     return out.reshape(om.cfg.M, om.cfg.E)
+
+
+def lookahead_table_capped(om, l, R, Dbar, cap):
+    out = np.zeros(om.cfg.M * om.cfg.E, np.float32)
+    lib().or_lookahead_table_capped(C.byref(om.m), l, C.c_float(R), C.c_float(Dbar), cap, _p(out))
+    return out.reshape(om.cfg.M, om.cfg.E)
+
+
+def predict_exit(om, centroids_l, centroid_exit_l, h_row):
+    c = np.ascontiguousarray(centroids_l, dtype=np.uint16)
+    e = np.ascontiguousarray(centroid_exit_l, dtype=np.float32)
+    hr = np.ascontiguousarray(h_row, dtype=np.uint16)
+    best = np.zeros(1, np.float32); gap = np.zeros(1, np.float32)
+    L = lib().or_predict_exit(C.byref(om.m), _p(c), _p(e), _p(hr), _p(best), _p(gap))
+    return int(L), float(best[0]), float(gap[0])
 
 
 def phi_naive(om, l, h, m, k, R, Dbar):

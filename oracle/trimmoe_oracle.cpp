@@ -92,6 +92,7 @@ typedef struct {
     const float* theta;        // [N] importance thresholds (Eq. 24)
     const float* lambda_;      // [N] slope of Lambda = lambda * I (Eq. 5)
     const float* eps;          // [N] per-layer skip tolerance (Eq. 25)
+    int n_centroids;           // K_c centroids per layer for Eq. (36); 0 = no exit prediction
 } OrModel;
 
 // Weights of one layer (host, bf16 bits).
@@ -105,6 +106,8 @@ typedef struct {
     const uint16_t* W13_sh;    // [2*F_sh][d] or NULL
     const uint16_t* W2_sh;     // [d][F_sh] or NULL
     const uint16_t* W_norm;    // [d] RMSNorm weights of this layer, NULL = no normalisation
+    const uint16_t* centroids; // [K_c][d] representations entering this layer (Eq. 36)
+    const float* centroid_exit;// [K_c] average exit layer of each centroid's calibration tokens
 } OrLayerWeights;
 
 // Per-token state (host arrays of length T), updated in place.
@@ -134,6 +137,7 @@ typedef struct {
     float* Gamma;        // [T]
     float* tot_exec;     // [T]
     float* tot_skip;     // [T] (+inf when skip not admitted)
+    int16_t* lhat;       // [T] predicted exit layer (Eq. 36), N without prediction, -1 dead
 } OrLayerOut;
 
 // One token's decision at one layer.
@@ -147,6 +151,7 @@ typedef struct {
     float Dhat_new;
     int s_new;
     int near;
+    int Lhat;          // predicted exit layer (Eq. 36), or N without a prediction
 } OrDecision;
 
 // ---------------------------------------------------------------- routing
@@ -310,10 +315,11 @@ static float phi_entry(const OrModel* md, int l, int m, int k, const float* V) {
 }
 
 // Phi^{(H-1)}_l(m, k) for every (m, k), evaluated bottom-up from the deepest
-// future layer (memoised form of Eq. 39).  Zero when H == 1 or l is the last layer.
-void or_lookahead_table(const OrModel* md, int l, float R, float Dbar, float* phi_out) {
+// future layer (memoised form of Eq. 39).  Zero when H == 1 or l is the last
+// layer.  cap limits the future layers to l+1 .. l+cap (a predicted exit).
+void or_lookahead_table_capped(const OrModel* md, int l, float R, float Dbar, int cap, float* phi_out) {
     const int M = md->M, E = md->E;
-    const int top = std::min(md->H - 1, md->N - 1 - l);
+    const int top = std::min(std::min(md->H - 1, md->N - 1 - l), cap);
     std::vector<float> V(M * E), phi_next(M * E), phi_cur(M * E);
     bool have_next = false;
     for (int j = top; j >= 1; --j) {
@@ -325,6 +331,34 @@ void or_lookahead_table(const OrModel* md, int l, float R, float Dbar, float* ph
         have_next = true;
     }
     for (int i = 0; i < M * E; ++i) phi_out[i] = have_next ? phi_next[i] : 0.0f;
+}
+
+void or_lookahead_table(const OrModel* md, int l, float R, float Dbar, float* phi_out) {
+    or_lookahead_table_capped(md, l, R, Dbar, 1 << 30, phi_out);
+}
+
+// Token-similarity exit-point prediction (Eq. 36): the nearest centroid by
+// cosine similarity (ties to the lower index) gives L_hat = round(mean exit
+// layer of its calibration tokens), rounding halves up.  *best_score and *gap
+// receive the best score and its margin over the second best (scores are the
+// cosine similarities times |h|, which does not change the order).
+int or_predict_exit(const OrModel* md, const uint16_t* centroids, const float* centroid_exit,
+                    const uint16_t* h, float* best_score, float* gap) {
+    const int K = md->n_centroids, d = md->d;
+    int best = -1;
+    float bs = 0.0f, second = -kInf;
+    for (int j = 0; j < K; ++j) {
+        const uint16_t* c = centroids + (size_t)j * d;
+        double nn = 0.0;
+        for (int i = 0; i < d; ++i) nn += (double)bf2f(c[i]) * (double)bf2f(c[i]);
+        const float cn = (float)std::sqrt(nn);
+        const float sc = (cn > 0.0f) ? (float)dot_bf16(h, c, d) / cn : -kInf;
+        if (best < 0 || sc > bs) { second = (best < 0) ? -kInf : bs; best = j; bs = sc; }
+        else if (sc > second) second = sc;
+    }
+    if (gap) *gap = bs - second;
+    if (best_score) *best_score = bs;
+    return (int)std::floor((double)centroid_exit[best] + 0.5);
 }
 
 static float value_naive(const OrModel* md, int lp, int h, int m, int kp, float R, float Dbar);
@@ -364,8 +398,8 @@ static float value_naive(const OrModel* md, int lp, int h, int m, int kp, float 
 
 // One token, one layer: the per-token body of Algorithm 2, given the routing (topk, g, I) and
 // the exit confidence xi (negative when not evaluated).
-void or_decide_given(const OrModel* md, int l, const int* topk, const float* g, float I, float xi,
-                     int s, float Dhat, float Dbar, float pJ, int last_exec, OrDecision* out) {
+void or_decide_given_capped(const OrModel* md, int l, const int* topk, const float* g, float I, float xi,
+                            int s, float Dhat, float Dbar, float pJ, int last_exec, int cap, OrDecision* out) {
     const int K = md->k, M = md->M, E = md->E;
     OrDecision D;
     std::memset(&D, 0, sizeof(D));
@@ -399,7 +433,7 @@ void or_decide_given(const OrModel* md, int l, const int* topk, const float* g, 
     // Look-ahead cost-to-go Phi^{(H-1)}_l (Eq. 39).
     const float R = Dbar - Dhat;
     std::vector<float> phi(M * E);
-    or_lookahead_table(md, l, R, Dbar, phi.data());
+    or_lookahead_table_capped(md, l, R, Dbar, cap, phi.data());
 
     // Slot 0: argmin of f + Phi (Eq. 40); later slots: argmin of f.
     float Drun = Dhat;
@@ -433,7 +467,13 @@ void or_decide_given(const OrModel* md, int l, const int* topk, const float* g, 
     if (D.action == A_EXEC) { D.s_new = D.srv_sel[0]; D.Dhat_new = Drun; }     // Eq. (41)
     else if (D.action == A_SKIP) { D.s_new = s; D.Dhat_new = Dhat + Lambda; }   // Eq. (42)
     else { D.s_new = s; D.Dhat_new = Dhat; }
+    D.Lhat = md->N;
     *out = D;
+}
+
+void or_decide_given(const OrModel* md, int l, const int* topk, const float* g, float I, float xi,
+                     int s, float Dhat, float Dbar, float pJ, int last_exec, OrDecision* out) {
+    or_decide_given_capped(md, l, topk, g, I, xi, s, Dhat, Dbar, pJ, last_exec, 1 << 30, out);
 }
 
 // Full per-token decision: router + exit head + or_decide_given.
@@ -446,10 +486,20 @@ void or_decide_token(const OrModel* md, const OrLayerWeights* lw, int l, const u
     float xi = -1.0f;
     if (l > 0 && last_exec && lw->W_x_prev)
         xi = or_exit_conf(md, lw->W_x_prev, lw->b_x_prev, h, lw->W_norm != nullptr, nullptr);
-    or_decide_given(md, l, topk, g, I, xi, s, Dhat, Dbar, pJ, last_exec, out);
+    // Predicted exit layer (Eq. 36) caps the look-ahead: layers >= L_hat are
+    // predicted not to run, so they add no cost-to-go.
+    int Lhat = md->N, cap = 1 << 30;
+    float cgap = kInf, cbest = 0.0f;
+    if (md->n_centroids > 0 && lw->centroids) {
+        Lhat = or_predict_exit(md, lw->centroids, lw->centroid_exit, h, &cbest, &cgap);
+        cap = Lhat - 1 - l;
+    }
+    or_decide_given_capped(md, l, topk, g, I, xi, s, Dhat, Dbar, pJ, last_exec, cap, out);
+    out->Lhat = Lhat;
     // Near-threshold flags for the comparison protocol.
     const float band = 1e-5f;
     int nr = 0;
+    if (cgap <= band * std::max(1.0f, std::fabs(cbest))) nr |= 32;
     if (std::fabs(I - md->theta[l]) <= band) nr |= 1;
     if (xi >= 0.0f && std::fabs(xi - pJ) <= band) nr |= 2;
     {
@@ -586,6 +636,7 @@ int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uin
             if (out->Gamma) out->Gamma[t] = D.Gamma;
             if (out->tot_exec) out->tot_exec[t] = D.tot_exec;
             if (out->tot_skip) out->tot_skip[t] = D.tot_skip;
+            if (out->lhat) out->lhat[t] = (int16_t)(D.action == A_DEAD ? -1 : D.Lhat);
             for (int j = 0; j < K; ++j) {
                 if (out->topk_idx) out->topk_idx[t * K + j] = D.action == A_DEAD ? -1 : D.topk[j];
                 if (out->topk_g) out->topk_g[t * K + j] = D.action == A_DEAD ? 0.0f : D.g[j];

@@ -34,17 +34,17 @@ class trimmoe_config(C.Structure):
     _fields_ = [(n, C.c_int) for n in ("N", "d", "E", "k", "F", "F_sh", "C", "M", "H", "act",
                                        "renorm_topk", "n_sub", "T_max")] + \
                [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref_ms", "phi_beta")] + \
-               [("profile", C.c_int), ("norm_eps", C.c_float)]
+               [("profile", C.c_int), ("norm_eps", C.c_float), ("n_centroids", C.c_int)]
 
 
 class trimmoe_weights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("W_r", "b_r", "W_x", "b_x", "W13", "W2", "W13_sh", "W2_sh",
-                                          "W_norm")]
+                                          "W_norm", "centroids")]
 
 
 class trimmoe_tables(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("place", "sim", "sub_thresh", "trans_ms", "comp_ms", "P",
-                                          "theta", "lambda_", "eps")]
+                                          "theta", "lambda_", "eps", "centroid_exit")]
 
 
 class trimmoe_tokens(C.Structure):
@@ -54,7 +54,7 @@ class trimmoe_tokens(C.Structure):
 
 class trimmoe_layer_out(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("topk_idx", "topk_g", "I", "xi", "action", "exp_sel",
-                                          "srv_sel", "perm", "group_off")]
+                                          "srv_sel", "perm", "group_off", "lhat")]
 
 
 class trimmoe_stats_t(C.Structure):
@@ -228,13 +228,15 @@ class Engine:
             "W13_sh": dt(experts["W13_sh"], torch.bfloat16) if cfg.F_sh else None,
             "W2_sh": dt(experts["W2_sh"], torch.bfloat16) if cfg.F_sh else None,
             "W_norm": dt(small["W_norm"], torch.bfloat16) if small.get("W_norm") is not None else None,
+            "centroids": dt(small["centroids"], torch.bfloat16) if cfg.n_centroids else None,
         }
         self.tables = {k: np.ascontiguousarray(v) for k, v in tables.items() if k != "d_ref"}
         self.c_cfg = trimmoe_config(
             N=cfg.N, d=cfg.d, E=cfg.E, k=cfg.k, F=cfg.F, F_sh=cfg.F_sh, C=cfg.C, M=cfg.M, H=cfg.H,
             act=cfg.act, renorm_topk=cfg.renorm_topk, n_sub=cfg.n_sub, T_max=T_max,
             omega_T=cfg.omega_T, omega_D=cfg.omega_D, d_ref_ms=float(tables["d_ref"]),
-            phi_beta=cfg.phi_beta, profile=1 if profile else 0, norm_eps=cfg.norm_eps)
+            phi_beta=cfg.phi_beta, profile=1 if profile else 0, norm_eps=cfg.norm_eps,
+            n_centroids=cfg.n_centroids)
         self.c_w = trimmoe_weights(**{k: _ptr(v) for k, v in self.w.items()})
         t = self.tables
         P = t["P"].astype(np.float32) if t["P"].size else None
@@ -245,6 +247,9 @@ class Engine:
             lambda_=_ptr(t["lam"]), eps=_ptr(t["eps"]))
         self._keep_place = t["place"].astype(np.uint16)
         self.c_tab.place = _ptr(self._keep_place)
+        if cfg.n_centroids:
+            self._cexit = np.ascontiguousarray(small["centroid_exit"], dtype=np.float32)
+            self.c_tab.centroid_exit = _ptr(self._cexit)
         self.T_max = T_max
         self.handle = trimmoe_create(self.c_cfg, self.c_w, self.c_tab)
 
@@ -291,7 +296,8 @@ class Engine:
             exp_sel=torch.empty(T * K, dtype=torch.uint8, device=dev),
             srv_sel=torch.empty(T * K, dtype=torch.uint8, device=dev),
             perm=torch.full((T * K + T,), -1, dtype=torch.int32, device=dev),
-            group_off=torch.empty(E + 2, dtype=torch.int32, device=dev))
+            group_off=torch.empty(E + 2, dtype=torch.int32, device=dev),
+            lhat=torch.empty(T, dtype=torch.int16, device=dev))
 
     def stream_ptr(self, stream=None) -> int:
         torch = self.torch

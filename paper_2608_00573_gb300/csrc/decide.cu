@@ -117,6 +117,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
                 p.action[t] = 3;
                 p.I_out[t] = 0.f;
                 p.xi_out[t] = -1.f;
+                if (p.lhat_out) p.lhat_out[t] = -1;
             }
             if (lane < K) {
                 p.topk_idx[t * K + lane] = -1;
@@ -203,6 +204,25 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         }
         const bool exit_ok = have_xi && (xi >= pJ);
 
+        // Token-similarity exit prediction (Eq. 36): nearest centroid by cosine
+        // (score h.c_j / |c_j|, ties to the lower index); layers >= L_hat are
+        // predicted not to run and leave the look-ahead.
+        int Lhat = p.N;
+        if (p.n_cent > 0) {
+            float bsc = -kInf;
+            int bj = 0x7fffffff;
+            for (int j = lane; j < p.n_cent; j += 32) {
+                float acc = 0.f;
+                for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + C + j]);
+                const float cn = p.cnorm[j];
+                const float sc = cn > 0.f ? __fdiv_rn(acc, cn) : -kInf;
+                if (sc > bsc || (sc == bsc && j < bj)) { bsc = sc; bj = j; }
+            }
+            warp_argmax(bsc, bj);
+            Lhat = p.lhat_tab[bj];
+        }
+        if (lane == 0 && p.lhat_out) p.lhat_out[t] = (int16_t)Lhat;
+
         // Transmission necessity (Eq. 35) over the budget-feasible candidates (Eq. 34).
         float Gamma = 0.f;
         for (int j = 0; j < K; ++j) {
@@ -222,7 +242,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
 
         // Look-ahead Phi^{(H-1)}_l over all (m, k), bottom-up (Eq. 39).
         const float R = __fsub_rn(Dbar, Dhat);
-        const int top = min(p.H - 1, p.N - 1 - l);
+        const int top = max(0, min(min(p.H - 1, p.N - 1 - l), Lhat - 1 - l));
         bool have_phi = false;
         for (int jj = top; jj >= 1; --jj) {
             const int lp = l + jj;

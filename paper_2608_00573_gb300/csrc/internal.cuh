@@ -57,7 +57,8 @@ struct RouterParams {
     int T, d;
     int n_out;                  // E + C logits per token
     int n_lo;                   // leading rows with a lo part (E)
-    int ng;                     // rows per pass (multiple of 8, <= 64)
+    int ng;                     // rows per pass (multiple of 8, <= 128)
+    int nl;                     // rows of the lo part staged per pass (multiple of 8, <= ng)
     int zs;                     // row stride of zpart
     int ksplit;                 // number of column ranges
     const __nv_bfloat16* h;
@@ -79,6 +80,10 @@ struct DecideParams {
     float norm_eps;
     float* rnorm;               // [T] RMS factor r (written when use_norm)
     int has_head;               // exit head of the previous layer available (layer > 0)
+    int n_cent;                 // K_c centroids (Eq. 36), 0 = no exit prediction
+    const float* cnorm;         // [K_c] centroid norms of this layer
+    const int16_t* lhat_tab;    // [K_c] rounded average exit layer of each centroid
+    int16_t* lhat_out;          // [T] predicted exit layer (may be NULL)
     uint8_t* s;
     float* Dhat;
     const float* Dbar;
@@ -151,7 +156,8 @@ struct FeedbackParams {
 
 // Launchers (one translation unit each).
 cudaError_t launch_router(const RouterParams& p, cudaStream_t st);
-size_t router_smem_bytes(int ng);
+size_t router_smem_bytes(int ng, int nl);
+int router_lo_rows(int n_lo, int ng);
 int router_pass_rows(int n_out);
 int router_ksplit(int T, int d, int num_sms);
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);

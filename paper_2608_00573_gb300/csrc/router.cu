@@ -18,7 +18,8 @@
 // outputs per token) and the kernel is bound by streaming h from HBM, so the
 // tensor cores only remove the per-element unpack/FMA instruction cost.
 // One block = 64 tokens (4 warps x 16), d streamed in 64-column slabs through
-// a 4-stage cp.async ring in padded shared memory, ldmatrix fragments.
+// a 4-stage cp.async ring in padded shared memory, ldmatrix fragments; up to
+// 128 output rows per pass over h.
 // Dead tokens are zero-filled without reading HBM.
 #include "internal.cuh"
 
@@ -30,7 +31,7 @@ constexpr int kTok = 64;
 constexpr int kKS = 64;
 constexpr int kPad = 72;          // padded smem row (bf16): conflict-free ldmatrix
 constexpr int kStages = 4;
-constexpr int kNG = 64;           // outputs per pass (8 n-tiles of 8)
+constexpr int kNG = 128;          // largest number of outputs per pass (16 n-tiles of 8)
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
@@ -60,9 +61,12 @@ __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
+// NT: n-tiles of 8 outputs held in registers per pass (8 or 16).
+template <int NT>
 __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
     extern __shared__ __align__(16) uint8_t sm[];
     const int NG = p.ng;                       // padded rows per pass (<= kNG, multiple of 8)
+    const int NL = p.nl;                       // padded rows with a lo part (<= NG)
     __nv_bfloat16* sA = reinterpret_cast<__nv_bfloat16*>(sm);
     __nv_bfloat16* sBh = sA + kStages * kTok * kPad;
     __nv_bfloat16* sBl = sBh + kStages * NG * kPad;
@@ -81,9 +85,9 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
         const int ntile = (nrows + 7) >> 3;
         const bool any_lo = ng0 < p.n_lo;
         float sq = 0.f;
-        float acc[kNG / 8][4];
+        float acc[NT][4];
 #pragma unroll
-        for (int j = 0; j < kNG / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+        for (int j = 0; j < NT; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
 
         auto load_slab = [&](int s) {
             const int buf = s % kStages;
@@ -100,9 +104,9 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
                 const bool ok = r < nrows;
                 const size_t off = (size_t)(ng0 + (ok ? r : 0)) * p.d + sg * kKS + c * 8;
                 cp_async16(smem_u32(sBh + (buf * NG + r) * kPad + c * 8), p.Bhi + off, ok ? 16 : 0);
-                if (any_lo) {
+                if (any_lo && r < NL) {
                     const bool okl = ok && (ng0 + r) < p.n_lo;
-                    cp_async16(smem_u32(sBl + (buf * NG + r) * kPad + c * 8), p.Blo + off, okl ? 16 : 0);
+                    cp_async16(smem_u32(sBl + (buf * NL + r) * kPad + c * 8), p.Blo + off, okl ? 16 : 0);
                 }
             }
         };
@@ -138,14 +142,14 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
                 const int br = (lane & 7);
                 const int bc = kk * 16 + ((lane >> 3) & 1) * 8;
 #pragma unroll
-                for (int j = 0; j < kNG / 8; ++j) {
+                for (int j = 0; j < NT; ++j) {
                     if (j < ntile) {
                         uint32_t b[2];
                         float part[4] = {0.f, 0.f, 0.f, 0.f};
                         ldmatrix_x2(b, smem_u32(sBh + (buf * NG + j * 8 + br) * kPad + bc));
                         mma_bf16_16816(part, a, b);
                         if (ng0 + j * 8 < p.n_lo) {
-                            ldmatrix_x2(b, smem_u32(sBl + (buf * NG + j * 8 + br) * kPad + bc));
+                            ldmatrix_x2(b, smem_u32(sBl + (buf * NL + j * 8 + br) * kPad + bc));
                             mma_bf16_16816(part, a, b);
                         }
 #pragma unroll
@@ -168,7 +172,7 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
             if (ng0 == 0 && tig == 0) sqpart[t] = ssq[r];
             float* zrow = zpart + (size_t)t * p.zs;
 #pragma unroll
-            for (int j = 0; j < kNG / 8; ++j) {
+            for (int j = 0; j < NT; ++j) {
                 if (j < ntile) {
 #pragma unroll
                     for (int q = 0; q < 2; ++q) {
@@ -184,8 +188,13 @@ __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
 
 }  // namespace
 
-size_t router_smem_bytes(int ng) {
-    return (size_t)kStages * (kTok + 2 * ng) * kPad * sizeof(__nv_bfloat16);
+size_t router_smem_bytes(int ng, int nl) {
+    return (size_t)kStages * (kTok + ng + nl) * kPad * sizeof(__nv_bfloat16);
+}
+
+int router_lo_rows(int n_lo, int ng) {
+    const int r = ((n_lo + 7) / 8) * 8;
+    return r < ng ? r : ng;
 }
 
 // Column ranges per launch: a power of two dividing d/64, chosen so that the
@@ -206,16 +215,20 @@ int router_pass_rows(int n_out) {
 cudaError_t launch_router(const RouterParams& p, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
     if (p.d % kKS || p.ksplit < 1 || (p.d / kKS) % p.ksplit) return cudaErrorInvalidValue;
-    const size_t smem = router_smem_bytes(p.ng);
+    const size_t smem = router_smem_bytes(p.ng, p.nl);
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(router_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)router_smem_bytes(kNG));
+        cudaError_t e = cudaFuncSetAttribute(router_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)router_smem_bytes(kNG, kNG));
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(router_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)router_smem_bytes(kNG, kNG));
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     const dim3 grid((p.T + kTok - 1) / kTok, p.ksplit);
-    router_kernel<<<grid, 128, smem, st>>>(p);
+    if (p.ng <= 64) router_kernel<8><<<grid, 128, smem, st>>>(p);
+    else router_kernel<16><<<grid, 128, smem, st>>>(p);
     return cudaGetLastError();
 }
 

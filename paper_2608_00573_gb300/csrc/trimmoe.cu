@@ -103,7 +103,9 @@ struct trimmoe {
     __nv_bfloat16* rt_hi = nullptr;   // [N][E+C][d] router (gamma folded, hi part) then exit head of layer-1
     __nv_bfloat16* rt_lo = nullptr;   // [N][E][d] lo part of gamma * W_r
     float* rt_bias = nullptr;         // [N][E+C]
-    float* zbuf = nullptr;            // [rows_part][E+C] partial logits
+    float* cnorm = nullptr;           // [N][K_c] centroid norms
+    int16_t* lhat = nullptr;          // [N][K_c] rounded average exit layers
+    float* zbuf = nullptr;            // [rows_part][E+C+K_c] partial logits
     float* sqbuf = nullptr;           // [rows_part] partial sums of squares
     size_t rows_part = 0;             // max over T <= T_max of ksplit(T) * T
     float* ctab = nullptr;
@@ -243,6 +245,7 @@ trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
     if (c->M * c->E > kMaxME) { why = "config: M*E > 1024"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->H > kMaxH) { why = "config: H > 6"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->n_sub > 3) { why = "config: n_sub > 3"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->n_centroids < 0 || c->n_centroids > 256) { why = "config: n_centroids must be in [0, 256]"; return TRIMMOE_ERR_UNSUPPORTED; }
     if ((long long)c->T_max * (c->k + 1) >= (1ll << 31)) { why = "config: T_max too large"; return TRIMMOE_ERR_UNSUPPORTED; }
     return TRIMMOE_OK;
 }
@@ -269,6 +272,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     const int n13 = c.act == 1 ? 2 : 1;
     if (!w->W_r || !w->b_r || !w->W_x || !w->b_x || !w->W13 || !w->W2)
         return create_fail(TRIMMOE_ERR_ARG, "create: NULL weight pointer");
+    if (c.n_centroids > 0 && (!w->centroids || !tab->centroid_exit || !aligned16(w->centroids)))
+        return create_fail(TRIMMOE_ERR_ARG, "create: n_centroids > 0 needs 16-byte aligned centroids and centroid_exit");
     if ((c.F_sh > 0) != (w->W13_sh != nullptr && w->W2_sh != nullptr))
         return create_fail(TRIMMOE_ERR_ARG, "create: shared-expert weights must be given iff F_sh > 0");
     if (!aligned16(w->W_r) || !aligned16(w->W_x) || !aligned16(w->W13) || !aligned16(w->W2) ||
@@ -368,8 +373,9 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     // layer, rows [0, E) hold gamma_l * W_r[l] split exactly into bf16 hi + lo
     // (a bf16 x bf16 product has at most 16 significant bits), rows [E, E+C) the
     // exit head of layer l-1 (zero at layer 0); biases likewise.
-    const int n_out = E + c.C;
-    std::vector<uint16_t> hWr((size_t)N * E * d), hWx((size_t)N * c.C * d), hG;
+    const int Kc = c.n_centroids;
+    const int n_out = E + c.C + Kc;
+    std::vector<uint16_t> hWr((size_t)N * E * d), hWx((size_t)N * c.C * d), hG, hCt((size_t)N * Kc * d);
     std::vector<float> hbr((size_t)N * E), hbx((size_t)N * c.C);
     {
         cudaError_t e1 = cudaMemcpy(hWr.data(), w->W_r, hWr.size() * 2, cudaMemcpyDeviceToHost);
@@ -380,6 +386,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
             hG.resize((size_t)N * d);
             e1 = cudaMemcpy(hG.data(), w->W_norm, hG.size() * 2, cudaMemcpyDeviceToHost);
         }
+        if (e1 == cudaSuccess && Kc > 0)
+            e1 = cudaMemcpy(hCt.data(), w->centroids, hCt.size() * 2, cudaMemcpyDeviceToHost);
         if (e1 != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, std::string("create: reading router weights: ") + cudaGetErrorString(e1));
     }
     std::vector<uint16_t> rhi((size_t)N * n_out * d, 0), rlo((size_t)N * E * d, 0);
@@ -401,7 +409,22 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
                 std::memcpy(&rhi[((size_t)l * n_out + E + cc) * d], &hWx[((size_t)(l - 1) * c.C + cc) * d], (size_t)d * 2);
                 rb[(size_t)l * n_out + E + cc] = hbx[(size_t)(l - 1) * c.C + cc];
             }
+        for (int j = 0; j < Kc; ++j)
+            std::memcpy(&rhi[((size_t)l * n_out + E + c.C + j) * d], &hCt[((size_t)l * Kc + j) * d], (size_t)d * 2);
     }
+    // Centroid norms (double sum, rounded to fp32) and rounded exit layers (Eq. 36).
+    std::vector<float> cn((size_t)N * std::max(Kc, 1), 0.f);
+    std::vector<int16_t> lh((size_t)N * std::max(Kc, 1), 0);
+    for (int l = 0; l < N; ++l)
+        for (int j = 0; j < Kc; ++j) {
+            double nn = 0.0;
+            for (int i = 0; i < d; ++i) {
+                const double v = bf16_to_float(hCt[((size_t)l * Kc + j) * d + i]);
+                nn += v * v;
+            }
+            cn[(size_t)l * Kc + j] = (float)std::sqrt(nn);
+            lh[(size_t)l * Kc + j] = (int16_t)std::floor((double)tab->centroid_exit[(size_t)l * Kc + j] + 0.5);
+        }
 
     for (int tt = 1; tt <= c.T_max; ++tt)
         h->rows_part = std::max(h->rows_part, (size_t)router_ksplit(tt, d, h->num_sms) * tt);
@@ -415,6 +438,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->cand_Q, cq.size()) && h->dalloc(&h->cand_off, coff.size()) &&
               h->dalloc(&h->ctab, ctab.size()) && h->dalloc(&h->rt_hi, rhi.size()) &&
               h->dalloc(&h->rt_lo, rlo.size()) && h->dalloc(&h->rt_bias, rb.size()) &&
+              h->dalloc(&h->cnorm, cn.size()) && h->dalloc(&h->lhat, lh.size()) &&
               h->dalloc(&h->zbuf, h->rows_part * (size_t)n_out) && h->dalloc(&h->sqbuf, h->rows_part) &&
               h->dalloc(&h->trans, (size_t)M * M) && h->dalloc(&h->comp, (size_t)N * M) &&
               h->dalloc(&h->P, (size_t)std::max(N - 1, 1) * E * E) && h->dalloc(&h->theta, N) &&
@@ -442,6 +466,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     up(h->rt_hi, rhi.data(), rhi.size() * 2);
     up(h->rt_lo, rlo.data(), rlo.size() * 2);
     up(h->rt_bias, rb.data(), rb.size() * 4);
+    up(h->cnorm, cn.data(), cn.size() * 4);
+    up(h->lhat, lh.data(), lh.size() * 2);
     up(h->trans, tab->trans_ms, (size_t)M * M * 4);
     up(h->comp, tab->comp_ms, (size_t)N * M * 4);
     if (N > 1) up(h->P, tab->P, (size_t)(N - 1) * E * E * 4);
@@ -508,13 +534,15 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     const __nv_bfloat16* hid = static_cast<const __nv_bfloat16*>(tok->hidden);
     const __nv_bfloat16* gamma =
         h->w.W_norm ? static_cast<const __nv_bfloat16*>(h->w.W_norm) + (size_t)layer * d : nullptr;
-    const int n_out = E + c.C;
+    const int Kc = c.n_centroids;
+    const int n_out = E + c.C + Kc;
     RouterParams rp;
     rp.T = T;
     rp.d = d;
     rp.n_out = n_out;
     rp.n_lo = E;
     rp.ng = router_pass_rows(n_out);
+    rp.nl = router_lo_rows(E, rp.ng);
     rp.zs = n_out;
     rp.ksplit = router_ksplit(T, d, h->num_sms);
     rp.h = hid;
@@ -534,6 +562,10 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.norm_eps = c.norm_eps;
     dp.rnorm = h->rnorm;
     dp.has_head = layer > 0;
+    dp.n_cent = Kc;
+    dp.cnorm = h->cnorm + (size_t)layer * Kc;
+    dp.lhat_tab = h->lhat + (size_t)layer * Kc;
+    dp.lhat_out = (out && out->lhat) ? out->lhat : nullptr;
     dp.s = tok->s;
     dp.Dhat = tok->Dhat;
     dp.Dbar = tok->Dbar;

@@ -82,6 +82,7 @@ class WorkloadConfig:
     exit_width: float = 2.0
     norm: bool = True                # pre-FFN RMSNorm of the MoE sublayer
     norm_eps: float = 1e-6
+    n_centroids: int = 0             # K_c centroids per layer for exit prediction (Eq. 36); 0 = off
     seed: int = 0
 
     @property
@@ -244,7 +245,26 @@ def make_small_weights(cfg: WorkloadConfig, calib: Optional[dict] = "auto") -> d
         b_x[:, 0] = np.asarray(calib["exit_bias"], dtype=np.float32)
     else:
         b_x[:, 0] = -30.0                                     # no exits
-    return dict(W_r=W_r, b_r=b_r, W_x=W_x, b_x=b_x, W_norm=W_norm)
+    out = dict(W_r=W_r, b_r=b_r, W_x=W_x, b_x=b_x, W_norm=W_norm)
+    if cfg.n_centroids:
+        out.update(make_centroids(cfg))
+    return out
+
+
+def make_centroids(cfg: WorkloadConfig) -> dict:
+    """Synthetic stand-in for the token-similarity reference set (Eq. 36): per
+    layer, K_c centroid directions ~ N(0, 1) in bf16 and, per centroid, an
+    average exit layer drawn around the workload's exit peak (uniform over the
+    remaining depth when it has none), never before the next layer."""
+    rng = np.random.default_rng([cfg.seed, 606])
+    N, K, d = cfg.N, cfg.n_centroids, cfg.d
+    cent = _normal_bf16(rng, (N, K, d), 1.0)
+    peak = cfg.exit_peak if cfg.exit_peak is not None else 0.75 * N
+    ex = np.zeros((N, K), np.float32)
+    for l in range(N):
+        v = rng.normal(peak, max(cfg.exit_width, 1.0) * 2.0, size=K)
+        ex[l] = np.clip(v, l + 1, N).astype(np.float32)
+    return dict(centroids=cent, centroid_exit=ex)
 
 
 def make_expert_weights_host(cfg: WorkloadConfig) -> dict:

@@ -79,7 +79,8 @@ def compare_layer(cfg, om, eng, l, dev_tok, experts, row_sample=None, check_perm
     mis = (rows_differ(g["action"], o["action"]) | rows_differ(g["topk_idx"], o["topk_idx"])
            | rows_differ(g["exp_sel"], o["exp_sel"]) | rows_differ(g["srv_sel"], o["srv_sel"])
            | (after["s"] != tok_or["s"]) | (after["alive"] != tok_or["alive"])
-           | (after["exit_layer"] != tok_or["exit_layer"]) | (after["last_exec"] != tok_or["last_exec"]))
+           | (after["exit_layer"] != tok_or["exit_layer"]) | (after["last_exec"] != tok_or["last_exec"])
+           | (g["lhat"] != o["lhat"]))
     near = o["near"] > 0
     live = before["alive"] > 0
     bad = mis & ~near

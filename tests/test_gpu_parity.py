@@ -246,3 +246,25 @@ def test_budget_edge_cases(budget):
     reports = _run_all_layers(cfg, mutate_tokens=mut, theta=0.95, exit_bias=1.0)
     if budget == 0.0:
         assert sum(r["skip"] for r in reports) == 0
+
+
+@pytest.mark.parametrize("name,kw", [
+    ("mixtral_like_kc64", dict(N=6, d=512, E=8, k=2, F=256, T=700, M=10, H=3, n_centroids=64, renorm_topk=1,
+                               exit_peak=3.0)),
+    ("qwen_like_kc32_shared", dict(N=4, d=256, E=60, k=4, F=128, F_sh=128, T=300, M=10, H=3, n_centroids=32)),
+])
+def test_layer_parity_with_exit_prediction(name, kw):
+    """Token-similarity exit prediction (Eq. 36) on: the predicted exit layer is
+    compared per token and the capped look-ahead through the decisions."""
+    import torch
+    cfg = small_cfg(name=name, seed=95, **kw)
+    eng, om, tables, small, experts = make_engine(cfg, theta=0.9, exit_bias=1.0)
+    dev = eng.tokens_to_device(W.make_tokens(cfg))
+    capped = 0
+    for l in range(cfg.N):
+        compare_layer(cfg, om, eng, l, dev, experts)
+        # tokens whose predicted exit shortens this layer's look-ahead (checked above)
+        capped += int((np.floor(small["centroid_exit"][l] + 0.5) < l + cfg.H).sum())
+    assert capped > 0
+    eng.close()
+    torch.cuda.synchronize()
