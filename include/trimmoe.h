@@ -266,6 +266,42 @@ typedef struct {
 trimmoe_status trimmoe_feedback(trimmoe_handle h, const trimmoe_feedback_cfg* fb, int T, trimmoe_tokens* tok,
                                 trimmoe_feedback_out* out, void* stream);
 
+/* Offline stage (Algorithm 1) on calibration runs.
+ * Between trimmoe_calibration_begin and trimmoe_calibration_end every layer step
+ * counts, per live token: activity (pi_l, Eq. 26), its server before the layer
+ * (rho_{m,l}), each routed slot (activation frequency a_l^k), each slot with
+ * I > theta_l (sigma_l^k, Eq. 27), and the transition of its slot-0 target from
+ * the previous layer (Eq. 38; a token's first layer only records its target).
+ * Results (host arrays owned by the caller, any may be NULL):
+ *  counts: trans [N-1][E][E], alive [N], resid [N][M], act [N][E], above [N][E];
+ *  P [N-1][E][E] = row-normalised transitions (uniform rows without data);
+ *  pi [N] = alive / T_cal; sigma [N][E] = above / act (0 without data);
+ *  act_freq [N][E] = act / (k * alive); lambda [N][E] = pi * sigma * act_freq;
+ *  rho [N][M] = resid / alive. */
+typedef struct {
+    uint64_t *trans, *alive, *resid, *act, *above;
+    float *P, *pi, *sigma, *act_freq, *lambda, *rho;
+} trimmoe_calibration_t;
+
+/* Zero the counts and start counting (synchronises). */
+trimmoe_status trimmoe_calibration_begin(trimmoe_handle h);
+
+/* Stop counting and write the counts and statistics; T_cal = number of
+ * calibration tokens that entered layer 0 (synchronises). */
+trimmoe_status trimmoe_calibration_end(trimmoe_handle h, long long T_cal, trimmoe_calibration_t* out);
+
+/* Greedy communication-aware replication (Algorithm 1, Eq. 28), host only.
+ * place [N][E] server masks (updated in place; every entry non-zero); lambda,
+ * rho as above; trans [M][M] delays; expert_bytes [N][E] memory of one copy;
+ * capacity [M] bytes.  The benefit of a copy of expert k of layer l on a server
+ * m without it is lambda_l^k * rho_{m,l} * mean over its current hosts m' of
+ * trans[m][m']; each step places the feasible copy (fits the residual memory
+ * of m, Eq. c.1) of largest benefit, ties to the lowest (m, l, k), until none is
+ * feasible.  *added receives the number of copies placed.  ERR_ARG on bad input,
+ * ERR_COVERAGE if an expert has no server on entry. */
+trimmoe_status trimmoe_replicate(int N, int E, int M, const float* lambda, const float* rho, const float* trans,
+                                 const double* expert_bytes, const double* capacity, uint16_t* place, int* added);
+
 /* Compaction of one layer's decisions without any device allocation (the
  * paper has no counterpart: this entry point exists for callers that cannot
  * call cudaMalloc, e.g. code running inside an allocator callback or in a

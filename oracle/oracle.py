@@ -112,6 +112,10 @@ def lib():
             L.or_max_threads.restype = i
             L.or_feedback.argtypes = [vp, i, i, vp, vp, vp, vp, vp, vp, C.c_double, C.c_double, f, f, vp]
             L.or_feedback.restype = i
+            L.or_calib_accumulate.argtypes = [vp, i, i, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+            L.or_calib_finalize.argtypes = [vp, C.c_longlong, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]
+            L.or_replicate.argtypes = [vp, vp, vp, vp, vp, vp]
+            L.or_replicate.restype = i
             _lib = L
     return _lib
 
@@ -327,3 +331,47 @@ def feedback(tok, N, user_size, eta, p_min, kappa, delay_sum_ms, ref_slots, d_re
     if rc:
         raise RuntimeError("or_feedback failed")
     return pJ, out
+
+
+class CalibCounts:
+    """Calibration counters of the offline stage (host, uint64)."""
+
+    def __init__(self, cfg):
+        N, E, M = cfg.N, cfg.E, cfg.M
+        self.cfg = cfg
+        self.trans = np.zeros((max(N - 1, 1), E, E), np.uint64)
+        self.alive = np.zeros(N, np.uint64)
+        self.resid = np.zeros((N, M), np.uint64)
+        self.act = np.zeros((N, E), np.uint64)
+        self.above = np.zeros((N, E), np.uint64)
+
+    def accumulate(self, om, l, out, s_before, prev_target):
+        T = len(s_before)
+        ti = np.ascontiguousarray(out["topk_idx"], np.int32)
+        I = np.ascontiguousarray(out["I"], np.float32)
+        a = np.ascontiguousarray(out["action"], np.uint8)
+        sb = np.ascontiguousarray(s_before, np.uint8)
+        lib().or_calib_accumulate(C.byref(om.m), l, T, _p(ti), _p(I), _p(a), _p(sb), _p(prev_target),
+                                  _p(self.trans), _p(self.alive), _p(self.resid), _p(self.act), _p(self.above))
+
+    def finalize(self, om, T_cal):
+        cfg = self.cfg
+        N, E, M = cfg.N, cfg.E, cfg.M
+        out = dict(P=np.zeros((max(N - 1, 1), E, E), np.float32), pi=np.zeros(N, np.float32),
+                   sigma=np.zeros((N, E), np.float32), act=np.zeros((N, E), np.float32),
+                   lam=np.zeros((N, E), np.float32), rho=np.zeros((N, M), np.float32))
+        lib().or_calib_finalize(C.byref(om.m), int(T_cal), _p(self.trans), _p(self.alive), _p(self.resid),
+                                _p(self.act), _p(self.above), _p(out["P"]), _p(out["pi"]), _p(out["sigma"]),
+                                _p(out["act"]), _p(out["lam"]), _p(out["rho"]))
+        return out
+
+
+def replicate(om, lam, rho, expert_bytes, capacity, place):
+    """Greedy replication (Eq. 28) on a copy of place; returns (new place, replicas added)."""
+    pl = np.array(place, dtype=np.uint16, copy=True)
+    lam = np.ascontiguousarray(lam, np.float32)
+    rho = np.ascontiguousarray(rho, np.float32)
+    eb = np.ascontiguousarray(expert_bytes, np.float64)
+    cap = np.ascontiguousarray(capacity, np.float64)
+    n = lib().or_replicate(C.byref(om.m), _p(lam), _p(rho), _p(eb), _p(cap), _p(pl))
+    return pl, int(n)

@@ -730,6 +730,110 @@ int or_feedback(const OrFeedbackCfg* fb, int T, int N, float* pJ, const uint8_t*
     return 0;
 }
 
+// ------------------------------------------------- offline stage (Algorithm 1)
+
+// Calibration counts of one layer from its decisions (Algorithm 1, statistics
+// behind Eq. 26-28 and 38).  For every token live at layer l: one active count
+// (pi_l), one residence count on its server before the layer (rho_{m,l}), one
+// activation count per routed slot (a_l^k), one above-threshold count per slot
+// when I > theta_l (sigma_l^k); and, when the token was live at l-1 too, one
+// transition count from its slot-0 target at l-1 to its slot-0 target at l
+// (Eq. 38).  prev_target[t] carries the slot-0 target between layers (-1 none).
+int or_calib_accumulate(const OrModel* md, int l, int T, const int32_t* topk_idx, const float* I,
+                        const uint8_t* action, const uint8_t* s_before, int16_t* prev_target,
+                        uint64_t* c_trans, uint64_t* c_alive, uint64_t* c_resid, uint64_t* c_act,
+                        uint64_t* c_above) {
+    const int E = md->E, K = md->k, M = md->M;
+    for (int t = 0; t < T; ++t) {
+        if (action[t] == A_DEAD) continue;
+        c_alive[l] += 1;
+        c_resid[(size_t)l * M + s_before[t]] += 1;
+        for (int j = 0; j < K; ++j) {
+            const int r = topk_idx[t * K + j];
+            c_act[(size_t)l * E + r] += 1;
+            if (I[t] > md->theta[l]) c_above[(size_t)l * E + r] += 1;
+        }
+        const int r0 = topk_idx[t * K];
+        if (l > 0 && prev_target[t] >= 0) c_trans[((size_t)(l - 1) * E + prev_target[t]) * E + r0] += 1;
+        prev_target[t] = (int16_t)r0;
+    }
+    return 0;
+}
+
+// Offline statistics from the counts over T_cal calibration tokens:
+// P_l(k -> k') = n_l(k -> k') / sum_k'' n_l(k -> k'') (Eq. 38; a row without
+// observations stays uniform), pi_l = active_l / T_cal (Eq. 26),
+// sigma_l^k = above_l^k / routed_l^k (Eq. 27; 0 without observations),
+// a_l^k = routed_l^k / (k * active_l), lambda_l^k = pi_l sigma_l^k a_l^k,
+// rho_{m,l} = resident_{m,l} / active_l.
+int or_calib_finalize(const OrModel* md, long long T_cal, const uint64_t* c_trans, const uint64_t* c_alive,
+                      const uint64_t* c_resid, const uint64_t* c_act, const uint64_t* c_above, float* P,
+                      float* pi, float* sigma, float* act, float* lam, float* rho) {
+    const int N = md->N, E = md->E, M = md->M, K = md->k;
+    for (int l = 0; l + 1 < N; ++l)
+        for (int k = 0; k < E; ++k) {
+            uint64_t tot = 0;
+            for (int kp = 0; kp < E; ++kp) tot += c_trans[((size_t)l * E + k) * E + kp];
+            for (int kp = 0; kp < E; ++kp)
+                P[((size_t)l * E + k) * E + kp] =
+                    tot ? (float)((double)c_trans[((size_t)l * E + k) * E + kp] / (double)tot) : (float)(1.0 / E);
+        }
+    for (int l = 0; l < N; ++l) {
+        const double a = (double)c_alive[l];
+        pi[l] = T_cal > 0 ? (float)(a / (double)T_cal) : 0.0f;
+        for (int k = 0; k < E; ++k) {
+            const double routed = (double)c_act[(size_t)l * E + k];
+            sigma[(size_t)l * E + k] = routed > 0 ? (float)((double)c_above[(size_t)l * E + k] / routed) : 0.0f;
+            act[(size_t)l * E + k] = a > 0 ? (float)(routed / (K * a)) : 0.0f;
+            lam[(size_t)l * E + k] = pi[l] * sigma[(size_t)l * E + k] * act[(size_t)l * E + k];
+        }
+        for (int m = 0; m < M; ++m) rho[(size_t)l * M + m] = a > 0 ? (float)((double)c_resid[(size_t)l * M + m] / a) : 0.0f;
+    }
+    return 0;
+}
+
+// Greedy communication-aware replication (Algorithm 1, Eq. 28, (c.1)-(c.3)).
+// Benefit of a replica of expert k of layer l on server m that does not hold
+// it: B = lambda_l^k * rho_{m,l} * mean over the servers m' holding it of
+// trans[m][m'] (the combined z/B + tau delay from m).  Each iteration evaluates
+// every feasible pair (not yet placed, fits the residual memory of m), places
+// the largest benefit (ties: lowest (m, l, k) in that order) and updates the
+// residual memory; it stops when no feasible pair remains.  place is updated
+// in place; returns the number of replicas added.
+int or_replicate(const OrModel* md, const float* lam, const float* rho, const double* expert_bytes,
+                 const double* capacity, uint16_t* place) {
+    const int N = md->N, E = md->E, M = md->M;
+    std::vector<double> used(M, 0.0);
+    for (int l = 0; l < N; ++l)
+        for (int k = 0; k < E; ++k)
+            for (int m = 0; m < M; ++m)
+                if ((place[(size_t)l * E + k] >> m) & 1u) used[m] += expert_bytes[(size_t)l * E + k];
+    int added = 0;
+    while (true) {
+        double best = -1.0;
+        int bm = -1, bl = -1, bk = -1;
+        for (int m = 0; m < M; ++m)
+            for (int l = 0; l < N; ++l)
+                for (int k = 0; k < E; ++k) {
+                    const uint16_t mask = place[(size_t)l * E + k];
+                    if ((mask >> m) & 1u) continue;
+                    if (used[m] + expert_bytes[(size_t)l * E + k] > capacity[m]) continue;
+                    double dsum = 0.0;
+                    int hosts = 0;
+                    for (int mp = 0; mp < M; ++mp)
+                        if ((mask >> mp) & 1u) { dsum += (double)md->trans[(size_t)m * M + mp]; ++hosts; }
+                    const double reach = hosts ? dsum / hosts : 0.0;
+                    const double B = (double)lam[(size_t)l * E + k] * (double)rho[(size_t)l * M + m] * reach;
+                    if (B > best) { best = B; bm = m; bl = l; bk = k; }
+                }
+        if (bm < 0) break;
+        place[(size_t)bl * E + bk] |= (uint16_t)(1u << bm);
+        used[bm] += expert_bytes[(size_t)bl * E + bk];
+        ++added;
+    }
+    return added;
+}
+
 int or_max_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();

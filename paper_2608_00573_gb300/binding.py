@@ -85,9 +85,15 @@ class trimmoe_feedback_out(C.Structure):
         return {n: getattr(self, n) for n, _ in self._fields_}
 
 
+class trimmoe_calibration_t(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in ("trans", "alive", "resid", "act", "above", "P", "pi", "sigma",
+                                          "act_freq", "lambda_", "rho")]
+
+
 EXPORTS = ("trimmoe_create", "trimmoe_layer_step", "trimmoe_forward", "trimmoe_forward_host",
            "trimmoe_stats", "trimmoe_reset_stats", "trimmoe_last_error", "trimmoe_destroy",
-           "trimmoe_compact_noalloc", "trimmoe_feedback")
+           "trimmoe_compact_noalloc", "trimmoe_feedback", "trimmoe_calibration_begin",
+           "trimmoe_calibration_end", "trimmoe_replicate")
 
 _lib = None
 _lock = threading.Lock()
@@ -122,6 +128,12 @@ def lib():
             L.trimmoe_compact_noalloc.argtypes = [vp, vp, i, i, i, i, vp, vp, vp, vp, vp]
             L.trimmoe_feedback.argtypes = [vp, vp, i, vp, vp, vp]
             L.trimmoe_feedback.restype = i
+            L.trimmoe_calibration_begin.argtypes = [vp]
+            L.trimmoe_calibration_begin.restype = i
+            L.trimmoe_calibration_end.argtypes = [vp, C.c_longlong, vp]
+            L.trimmoe_calibration_end.restype = i
+            L.trimmoe_replicate.argtypes = [i, i, i, vp, vp, vp, vp, vp, vp, vp]
+            L.trimmoe_replicate.restype = i
             L.trimmoe_compact_noalloc.restype = i
             _lib = L
     return _lib
@@ -180,6 +192,37 @@ def trimmoe_feedback(h, fb: trimmoe_feedback_cfg, T: int, tok: trimmoe_tokens, s
     out = trimmoe_feedback_out()
     _check(lib().trimmoe_feedback(h, C.byref(fb), T, C.byref(tok), C.byref(out), C.c_void_p(stream)), h)
     return out.as_dict()
+
+
+def trimmoe_calibration_begin(h):
+    _check(lib().trimmoe_calibration_begin(h), h)
+
+
+def trimmoe_calibration_end(h, T_cal: int, N: int, E: int, M: int) -> dict:
+    """Counts and statistics of the offline stage as numpy arrays."""
+    o = dict(trans=np.zeros((max(N - 1, 1), E, E), np.uint64), alive=np.zeros(N, np.uint64),
+             resid=np.zeros((N, M), np.uint64), act=np.zeros((N, E), np.uint64), above=np.zeros((N, E), np.uint64),
+             P=np.zeros((max(N - 1, 1), E, E), np.float32), pi=np.zeros(N, np.float32),
+             sigma=np.zeros((N, E), np.float32), act_freq=np.zeros((N, E), np.float32),
+             lam=np.zeros((N, E), np.float32), rho=np.zeros((N, M), np.float32))
+    st = trimmoe_calibration_t(trans=_ptr(o["trans"]), alive=_ptr(o["alive"]), resid=_ptr(o["resid"]),
+                               act=_ptr(o["act"]), above=_ptr(o["above"]), P=_ptr(o["P"]), pi=_ptr(o["pi"]),
+                               sigma=_ptr(o["sigma"]), act_freq=_ptr(o["act_freq"]), lambda_=_ptr(o["lam"]),
+                               rho=_ptr(o["rho"]))
+    _check(lib().trimmoe_calibration_end(h, int(T_cal), C.byref(st)), h)
+    return o
+
+
+def trimmoe_replicate(lam, rho, trans, expert_bytes, capacity, place):
+    """Greedy replication (Eq. 28) on a copy of place (host arrays); returns (place, added)."""
+    N, E = place.shape
+    M = trans.shape[0]
+    pl = np.array(place, dtype=np.uint16, copy=True)
+    arrs = [np.ascontiguousarray(a, dt) for a, dt in ((lam, np.float32), (rho, np.float32), (trans, np.float32),
+                                                        (expert_bytes, np.float64), (capacity, np.float64))]
+    added = C.c_int(0)
+    _check(lib().trimmoe_replicate(N, E, M, *[_ptr(a) for a in arrs], _ptr(pl), C.byref(added)))
+    return pl, added.value
 
 
 def trimmoe_compact_noalloc(action, exp_sel, T: int, k: int, E: int, has_shared: int, perm, group_off,
@@ -322,6 +365,12 @@ class Engine:
 
     def stats(self) -> dict:
         return trimmoe_stats(self.handle)
+
+    def calibration_begin(self):
+        trimmoe_calibration_begin(self.handle)
+
+    def calibration_end(self, T_cal: int) -> dict:
+        return trimmoe_calibration_end(self.handle, T_cal, self.cfg.N, self.cfg.E, self.cfg.M)
 
     def feedback(self, tok: dict, user_size: int, eta: float, p_min: float, kappa: float,
                  T: Optional[int] = None, stream=None) -> dict:

@@ -343,6 +343,18 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
             p.exp_sel[t * K + lane] = action == 0 ? (uint8_t)esel[lane] : 0xFF;
             p.srv_sel[t * K + lane] = action == 0 ? (uint8_t)msel[lane] : 0xFF;
         }
+        if (lane == 0 && p.calib) {
+            // Calibration counts of the offline stage (Eq. 26-28, 38).
+            atomicAdd(&p.c_alive[l], 1ull);
+            atomicAdd(&p.c_resid[l * M + s], 1ull);
+            for (int j = 0; j < K; ++j) {
+                atomicAdd(&p.c_act[l * E + topk[j]], 1ull);
+                if (I > p.tab.theta[l]) atomicAdd(&p.c_above[l * E + topk[j]], 1ull);
+            }
+            const int prev = p.prev_target[t];
+            if (l > 0 && prev >= 0) atomicAdd(&p.c_trans[((size_t)(l - 1) * E + prev) * E + topk[0]], 1ull);
+            p.prev_target[t] = (int16_t)topk[0];
+        }
         if (lane == 0) {
             p.action[t] = (uint8_t)action;
             p.I_out[t] = I;

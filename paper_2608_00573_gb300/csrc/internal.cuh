@@ -84,6 +84,14 @@ struct DecideParams {
     const float* cnorm;         // [K_c] centroid norms of this layer
     const int16_t* lhat_tab;    // [K_c] rounded average exit layer of each centroid
     int16_t* lhat_out;          // [T] predicted exit layer (may be NULL)
+    // Offline-stage calibration counts (Algorithm 1), accumulated when calib != 0.
+    int calib;
+    int16_t* prev_target;       // [T] slot-0 target at the previous layer, -1 none
+    unsigned long long* c_trans;   // [N-1][E][E]
+    unsigned long long* c_alive;   // [N]
+    unsigned long long* c_resid;   // [N][M]
+    unsigned long long* c_act;     // [N][E]
+    unsigned long long* c_above;   // [N][E]
     uint8_t* s;
     float* Dhat;
     const float* Dbar;

@@ -141,6 +141,12 @@ struct trimmoe {
     int* fb_updated = nullptr;
     double* fb_result = nullptr;
 
+    // offline-stage calibration counts
+    int calib = 0;
+    int16_t* prev_target = nullptr;
+    unsigned long long* c_counts = nullptr;   // trans | alive | resid | act | above
+    size_t n_counts = 0;
+
     // counters kept on the host
     uint64_t launches = 0, layer_calls = 0;
 
@@ -451,7 +457,10 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->blk_base, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
               h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, 1) && h->dalloc(&h->dev_err, 1) &&
-              h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2);
+              h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2) &&
+              h->dalloc(&h->prev_target, T);
+    h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
+    ok = ok && h->dalloc(&h->c_counts, h->n_counts);
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
     if (!ok) return bail(TRIMMOE_ERR_OOM, "create: device allocation failed");
     cudaError_t ce = cudaSuccess;
@@ -566,6 +575,13 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.cnorm = h->cnorm + (size_t)layer * Kc;
     dp.lhat_tab = h->lhat + (size_t)layer * Kc;
     dp.lhat_out = (out && out->lhat) ? out->lhat : nullptr;
+    dp.calib = h->calib;
+    dp.prev_target = h->prev_target;
+    dp.c_trans = h->c_counts;
+    dp.c_alive = dp.c_trans + (size_t)std::max(c.N - 1, 1) * E * E;
+    dp.c_resid = dp.c_alive + c.N;
+    dp.c_act = dp.c_resid + (size_t)c.N * c.M;
+    dp.c_above = dp.c_act + (size_t)c.N * E;
     dp.s = tok->s;
     dp.Dhat = tok->Dhat;
     dp.Dbar = tok->Dbar;
@@ -847,6 +863,116 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
     h->launches = h->layer_calls = h->n_gemm_up = h->n_gemm_down = 0;
     h->win_delay0 = 0.0;
     h->win_ref_slots = 0.0;
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_calibration_begin(trimmoe_handle h) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    DeviceGuard g(h->dev);
+    if (cudaStreamSynchronize(h->last_stream) != cudaSuccess ||
+        cudaMemset(h->c_counts, 0, h->n_counts * sizeof(unsigned long long)) != cudaSuccess ||
+        cudaMemset(h->prev_target, 0xFF, (size_t)h->cfg.T_max * sizeof(int16_t)) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, "calibration_begin: reset failed");
+    h->calib = 1;
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_calibration_end(trimmoe_handle h, long long T_cal, trimmoe_calibration_t* out) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    if (!out || T_cal < 0) return h->fail(TRIMMOE_ERR_ARG, "calibration_end: NULL output or negative T_cal");
+    DeviceGuard g(h->dev);
+    std::vector<unsigned long long> cnt(h->n_counts);
+    if (cudaStreamSynchronize(h->last_stream) != cudaSuccess ||
+        cudaMemcpy(cnt.data(), h->c_counts, cnt.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) !=
+            cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, "calibration_end: copy failed");
+    h->calib = 0;
+    const int N = h->cfg.N, E = h->cfg.E, M = h->cfg.M, K = h->cfg.k;
+    const size_t ntr = (size_t)std::max(N - 1, 1) * E * E;
+    const unsigned long long* trans = cnt.data();
+    const unsigned long long* alive = trans + ntr;
+    const unsigned long long* resid = alive + N;
+    const unsigned long long* act = resid + (size_t)N * M;
+    const unsigned long long* above = act + (size_t)N * E;
+    auto put = [](uint64_t* dst, const unsigned long long* src, size_t n) {
+        if (dst) for (size_t i = 0; i < n; ++i) dst[i] = src[i];
+    };
+    put(out->trans, trans, ntr);
+    put(out->alive, alive, N);
+    put(out->resid, resid, (size_t)N * M);
+    put(out->act, act, (size_t)N * E);
+    put(out->above, above, (size_t)N * E);
+    if (out->P)
+        for (int l = 0; l + 1 < N; ++l)
+            for (int k = 0; k < E; ++k) {
+                unsigned long long tot = 0;
+                for (int kp = 0; kp < E; ++kp) tot += trans[((size_t)l * E + k) * E + kp];
+                for (int kp = 0; kp < E; ++kp)
+                    out->P[((size_t)l * E + k) * E + kp] =
+                        tot ? (float)((double)trans[((size_t)l * E + k) * E + kp] / (double)tot) : (float)(1.0 / E);
+            }
+    for (int l = 0; l < N; ++l) {
+        const double a = (double)alive[l];
+        const float pi = T_cal > 0 ? (float)(a / (double)T_cal) : 0.0f;
+        if (out->pi) out->pi[l] = pi;
+        for (int k = 0; k < E; ++k) {
+            const double routed = (double)act[(size_t)l * E + k];
+            const float sg = routed > 0 ? (float)((double)above[(size_t)l * E + k] / routed) : 0.0f;
+            const float af = a > 0 ? (float)(routed / (K * a)) : 0.0f;
+            if (out->sigma) out->sigma[(size_t)l * E + k] = sg;
+            if (out->act_freq) out->act_freq[(size_t)l * E + k] = af;
+            if (out->lambda) out->lambda[(size_t)l * E + k] = pi * sg * af;
+        }
+        if (out->rho)
+            for (int m = 0; m < M; ++m)
+                out->rho[(size_t)l * M + m] = a > 0 ? (float)((double)resid[(size_t)l * M + m] / a) : 0.0f;
+    }
+    return TRIMMOE_OK;
+}
+
+extern "C" trimmoe_status trimmoe_replicate(int N, int E, int M, const float* lambda, const float* rho,
+                                            const float* trans, const double* expert_bytes, const double* capacity,
+                                            uint16_t* place, int* added) {
+    if (N < 1 || E < 1 || M < 1 || M > 16 || !lambda || !rho || !trans || !expert_bytes || !capacity || !place) {
+        tmoe::set_global_error("replicate: bad dimensions or NULL pointer");
+        return TRIMMOE_ERR_ARG;
+    }
+    const uint32_t mmask = (M >= 16) ? 0xFFFFu : ((1u << M) - 1u);
+    std::vector<double> used(M, 0.0);
+    for (int l = 0; l < N; ++l)
+        for (int k = 0; k < E; ++k) {
+            if ((place[(size_t)l * E + k] & mmask) == 0) {
+                tmoe::set_global_error("replicate: an expert has no server (Eq. 2)");
+                return TRIMMOE_ERR_COVERAGE;
+            }
+            for (int m = 0; m < M; ++m)
+                if ((place[(size_t)l * E + k] >> m) & 1u) used[m] += expert_bytes[(size_t)l * E + k];
+        }
+    int n_added = 0;
+    while (true) {
+        double best = -1.0;
+        int bm = -1, bl = -1, bk = -1;
+        for (int m = 0; m < M; ++m)
+            for (int l = 0; l < N; ++l)
+                for (int k = 0; k < E; ++k) {
+                    const uint16_t mask = place[(size_t)l * E + k];
+                    if ((mask >> m) & 1u) continue;
+                    if (used[m] + expert_bytes[(size_t)l * E + k] > capacity[m]) continue;
+                    double sum = 0.0;
+                    int hosts = 0;
+                    for (int mp = 0; mp < M; ++mp)
+                        if ((mask >> mp) & 1u) { sum += (double)trans[(size_t)m * M + mp]; ++hosts; }
+                    const double reach = hosts ? sum / hosts : 0.0;
+                    const double b = (double)lambda[(size_t)l * E + k] * (double)rho[(size_t)l * M + m] * reach;
+                    if (b > best) { best = b; bm = m; bl = l; bk = k; }
+                }
+        if (bm < 0) break;
+        place[(size_t)bl * E + bk] |= (uint16_t)(1u << bm);
+        used[bm] += expert_bytes[(size_t)bl * E + bk];
+        ++n_added;
+    }
+    if (added) *added = n_added;
     return TRIMMOE_OK;
 }
 

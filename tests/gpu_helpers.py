@@ -133,4 +133,4 @@ def compare_layer(cfg, om, eng, l, dev_tok, experts, row_sample=None, check_perm
     counts = np.bincount(g["action"], minlength=4)
     return dict(layer=l, live=n_live, near_mismatch=n_mis, near=int(near.sum()), max_rel_err=err,
                 exec=int(counts[0]), skip=int(counts[1]), exit=int(counts[2]), dead=int(counts[3]),
-                rows_checked=int(run.sum()))
+                rows_checked=int(run.sum()), oracle_out=o, s_before=before["s"])
