@@ -294,11 +294,13 @@ def run_ours(args):
     # Roofline of the dominant kernel (grouped FFN GEMM) from events recorded
     # around each launch on the launching stream during the timed region.
     peaks = load_peaks()
-    kinds = {"grouped_gemm_gate_up": (st["ms_gemm_up"], st["flops_gemm_up"], st["n_gemm_up"]),
-             "grouped_gemm_down": (st["ms_gemm_down"], st["flops_gemm_down"], st["n_gemm_down"])}
+    kinds = {"grouped_gemm_gate_up": (st["ms_gemm_up"], st["flops_gemm_up"], st["n_gemm_up"], st["bytes_gemm_up"]),
+             "grouped_gemm_down": (st["ms_gemm_down"], st["flops_gemm_down"], st["n_gemm_down"],
+                                   st["bytes_gemm_down"])}
     dom = max(kinds, key=lambda k: kinds[k][0])
-    ms_k, fl_k, n_k = kinds[dom]
+    ms_k, fl_k, n_k, by_k = kinds[dom]
     achieved = fl_k / (ms_k / 1e3) / 1e12 if ms_k > 0 else 0.0
+    achieved_bw = by_k / (ms_k / 1e3) / 1e9 if ms_k > 0 else 0.0
     traffic = None
     tp = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tp):
@@ -307,13 +309,23 @@ def run_ours(args):
         ent = tj.get(cfg.name, {}).get(dom)
         if ent and ent.get("kernel_rev") == KERNEL_REV:
             traffic = ent.get("bytes_per_launch")
-    roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peaks["bf16_sus"],
-            "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sus"], "traffic": traffic,
-            "peak_source": f"{peaks['source']} bf16 sustained",
-            "flops_per_launch": fl_k / max(n_k, 1), "ms_per_launch": ms_k / max(n_k, 1)}
-    # Whole-forward roofline: executed GEMM FLOPs at the bf16 peak vs bytes at HBM.
+    # The GEMM is tensor-bound when its FLOPs take longer at peak than its bytes.
+    tensor_bound = fl_k / (peaks["bf16_sus"] * 1e12) >= by_k / (peaks["hbm"] * 1e9)
+    if tensor_bound:
+        roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peaks["bf16_sus"],
+                "unit": "TFLOP/s", "frac": achieved / peaks["bf16_sus"], "traffic": traffic,
+                "peak_source": f"{peaks['source']} bf16 sustained"}
+    else:
+        roof = {"bound": "hbm", "kernel": dom, "achieved": achieved_bw, "peak": peaks["hbm"],
+                "unit": "GB/s", "frac": achieved_bw / peaks["hbm"], "traffic": traffic,
+                "peak_source": f"{peaks['source']} HBM copy"}
+    roof.update(flops_per_launch=fl_k / max(n_k, 1), bytes_per_launch=by_k / max(n_k, 1),
+                ms_per_launch=ms_k / max(n_k, 1))
+    # Whole-forward roofline: executed GEMM FLOPs at the bf16 peak vs the GEMMs'
+    # bytes at HBM, whichever is slower.
     per_fwd_flops = st["gemm_flops"] / args.steps
-    fwd_roof_ms = per_fwd_flops / (peaks["bf16_sus"] * 1e12) * 1e3
+    per_fwd_bytes = (st["bytes_gemm_up"] + st["bytes_gemm_down"]) / args.steps
+    fwd_roof_ms = max(per_fwd_flops / (peaks["bf16_sus"] * 1e12), per_fwd_bytes / (peaks["hbm"] * 1e9)) * 1e3
     kernel_ms = {k: st[f"ms_{k}"] / args.steps for k in
                  ("router", "decide", "compact", "gather", "gemm_up", "gemm_down", "combine")}
     line = {
@@ -325,8 +337,8 @@ def run_ours(args):
                    "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (expert weights and hidden states)"},
         "roofline": roof,
-        "forward_roofline": {"gemm_flops_per_forward": per_fwd_flops, "roofline_ms": fwd_roof_ms,
-                             "frac": fwd_roof_ms / ms_step},
+        "forward_roofline": {"gemm_flops_per_forward": per_fwd_flops, "gemm_bytes_per_forward": per_fwd_bytes,
+                             "roofline_ms": fwd_roof_ms, "frac": fwd_roof_ms / ms_step},
         "kernel_ms_per_step": kernel_ms,
         "decisions": {"layer_tokens": st["layer_tokens"] // args.steps,
                       "skip_share": st["skipped"] / max(st["layer_tokens"], 1),

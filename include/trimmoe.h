@@ -196,6 +196,13 @@ typedef struct {
     uint64_t n_gemm_up, n_gemm_down;
     double flops_gemm_up, flops_gemm_down;
     double ms_router;             /* router / exit-head logits kernel (profile != 0) */
+    /* Algorithmic HBM bytes of the grouped FFN GEMMs that ran: weights of the
+     * experts that received work once, activation rows in and out. */
+    double bytes_gemm_up, bytes_gemm_down;
+    /* Decisions whose look-ahead table (Eq. 39) was read from the per-layer
+     * tables shared by all tokens of equal budget instead of computed per token
+     * (the results are the same either way). */
+    uint64_t lookahead_shared;
 } trimmoe_stats_t;
 
 /* Validate, copy the tables, derive the candidate lists V_{l,r} and losses Q,

@@ -67,7 +67,9 @@ class trimmoe_stats_t(C.Structure):
                [(n, C.c_double) for n in ("ms_decide", "ms_compact", "ms_gather", "ms_gemm_up",
                                           "ms_gemm_down", "ms_combine")] + \
                [("n_gemm_up", C.c_uint64), ("n_gemm_down", C.c_uint64),
-                ("flops_gemm_up", C.c_double), ("flops_gemm_down", C.c_double), ("ms_router", C.c_double)]
+                ("flops_gemm_up", C.c_double), ("flops_gemm_down", C.c_double), ("ms_router", C.c_double),
+                ("bytes_gemm_up", C.c_double), ("bytes_gemm_down", C.c_double),
+                ("lookahead_shared", C.c_uint64)]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}

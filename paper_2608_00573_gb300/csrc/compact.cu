@@ -60,6 +60,10 @@ __global__ void __launch_bounds__(256) scan_kernel(const CompactParams p) {
         p.goff[nb] = acc;
         atomicAdd(&p.ctr->pairs_total, (unsigned long long)(acc - total[p.E]));
         atomicAdd(&p.ctr->shared_rows, (unsigned long long)total[p.E]);
+        unsigned long long touched = 0;
+        for (int e = 0; e < p.E; ++e) touched += total[e] > 0 ? 1ull : 0ull;
+        atomicAdd(&p.ctr->experts_touched, touched);
+        if (total[p.E] > 0) atomicAdd(&p.ctr->shared_touched, 1ull);
     }
 }
 

@@ -74,7 +74,7 @@ __device__ __forceinline__ float exec_cost(const DecideParams& p, const float* c
 
 struct WarpCounters {
     unsigned long long layer_tokens, exec_tokens, skipped, exited;
-    unsigned long long le, ls, re, rs, hops;
+    unsigned long long le, ls, re, rs, hops, shared_phi;
     double delay;
     float max_ratio;
 };
@@ -99,10 +99,10 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
     uint8_t* cok = reinterpret_cast<uint8_t*>(cph + MC);   // Q <= R
     uint8_t* cmv = cok + ((MC + 3) & ~3);                  // server of the candidate
 
-    __shared__ unsigned long long blk_cnt[9];
+    __shared__ unsigned long long blk_cnt[10];
     __shared__ double blk_delay;
     __shared__ unsigned int blk_ratio;
-    if (threadIdx.x < 9) blk_cnt[threadIdx.x] = 0ull;
+    if (threadIdx.x < 10) blk_cnt[threadIdx.x] = 0ull;
     if (threadIdx.x == 0) { blk_delay = 0.0; blk_ratio = 0u; }
     __syncthreads();
 
@@ -240,11 +240,26 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         const float Lambda = __fmul_rn(p.tab.lambda[l], I);
         const bool skip_ok = (Gamma > 0.f) && (I <= p.tab.theta[l]) && (__fadd_rn(Dhat, Lambda) <= Dbar);
 
-        // Look-ahead Phi^{(H-1)}_l over all (m, k), bottom-up (Eq. 39).
+        // Look-ahead Phi^{(H-1)}_l over all (m, k), bottom-up (Eq. 39).  Phi
+        // depends on the token only through Dbar and the tests Q <= R and
+        // eps <= R, so every R between two consecutive thresholds of the window
+        // gives the same table: with the layer's Dbar the token reads the table
+        // of its interval, computed once with the same operation order.
         const float R = __fsub_rn(Dbar, Dhat);
         const int top = max(0, min(min(p.H - 1, p.N - 1 - l), Lhat - 1 - l));
         bool have_phi = false;
-        for (int jj = top; jj >= 1; --jj) {
+        const float* phiP = bufPhi;
+        const bool use_shared = p.phi_tabs != nullptr && top >= p.dmin && top > 0 && Dbar == *p.dbar_shared;
+        if (use_shared) {
+            int lo = 0, hi = p.n_thr;       // interval = number of thresholds <= R
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (p.thr[mid] <= R) lo = mid + 1; else hi = mid;
+            }
+            phiP = p.phi_tabs + ((size_t)(top - p.dmin) * (p.n_thr + 1) + lo) * ME;
+            have_phi = true;
+        }
+        for (int jj = use_shared ? 0 : top; jj >= 1; --jj) {
             const int lp = l + jj;
             const float eps = p.tab.eps[lp];
             const int* coff = p.tab.cand_off + lp * (E + 1);
@@ -317,7 +332,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
                 const int m = p.tab.cand_m[c];
                 const float f = exec_cost(p, ct_s, m, Q, Dbar);
                 float v = f;
-                if (j == 0) v = __fadd_rn(f, have_phi ? bufPhi[m * E + p.tab.cand_k[c]] : 0.f);
+                if (j == 0) v = __fadd_rn(f, have_phi ? phiP[m * E + p.tab.cand_k[c]] : 0.f);
                 if (v < bv) { bv = v; bi = c; }
             }
             warp_argmin(bv, bi);
@@ -330,7 +345,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         float tot_skip = kInf;
         if (skip_ok)
             tot_skip = __fadd_rn(__fmul_rn(p.omega_D, __fdiv_rn(Lambda, Dbar)),
-                                 have_phi ? bufPhi[s * E + topk[0]] : 0.f);
+                                 have_phi ? phiP[s * E + topk[0]] : 0.f);
         int action = 0;
         float best = tot_exec;
         if (skip_ok && tot_skip < tot_exec) { action = 1; best = tot_skip; }
@@ -386,6 +401,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
                 ++wc.exited;
             }
             ++wc.layer_tokens;
+            if (use_shared) ++wc.shared_phi;
             if (Dbar > 0.f && Dbar < FLT_MAX) wc.max_ratio = fmaxf(wc.max_ratio, Dnew / Dbar);
         }
         __syncwarp();
@@ -400,6 +416,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         atomicAdd(&blk_cnt[6], wc.re);
         atomicAdd(&blk_cnt[7], wc.rs);
         atomicAdd(&blk_cnt[8], wc.hops);
+        atomicAdd(&blk_cnt[9], wc.shared_phi);
         atomicAdd(&blk_delay, wc.delay);
         atomicMax(&blk_ratio, __float_as_uint(fmaxf(wc.max_ratio, 0.f)));
     }
@@ -415,12 +432,101 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         atomicAdd(&c->pairs_remote_exact, blk_cnt[6]);
         atomicAdd(&c->pairs_remote_sub, blk_cnt[7]);
         atomicAdd(&c->remote_hops, blk_cnt[8]);
+        atomicAdd(&c->lookahead_shared, blk_cnt[9]);
         atomicAdd(&c->delay_ms, blk_delay);
         atomicMax(&c->max_budget_ratio_bits, blk_ratio);
     }
 }
 
+// The layer's look-ahead tables for Dbar = Dbar[0]: block (i, y) computes the
+// table of interval i (R = thr[i - 1], or -inf for i = 0) at depth dmin + y,
+// each entry by one thread with the same operation order as the per-token path
+// above.
+__global__ void __launch_bounds__(256) lookahead_shared_kernel(const DecideParams p) {
+    extern __shared__ float smem[];
+    const int E = p.E, M = p.M, l = p.layer;
+    const int ME = M * E;
+    const int MC = p.tab.max_layer_cand;
+    float* bufV = smem;
+    float* bufPhi = bufV + ME;
+    float* cqt = bufPhi + ME;
+    float* cph = cqt + MC;
+    uint8_t* cok = reinterpret_cast<uint8_t*>(cph + MC);
+    uint8_t* cmv = cok + ((MC + 3) & ~3);
+    const float Dbar = p.Dbar[0];
+    const int iv = blockIdx.x;
+    const float R = iv == 0 ? -kInf : p.thr[iv - 1];
+    const int top = p.dmin + blockIdx.y;
+    bool have_phi = false;
+    for (int jj = top; jj >= 1; --jj) {
+        const int lp = l + jj;
+        const float eps = p.tab.eps[lp];
+        const int* coff = p.tab.cand_off + lp * (E + 1);
+        const int cb = coff[0];
+        const int nc = coff[E] - cb;
+        for (int c = threadIdx.x; c < nc; c += blockDim.x) {
+            const float Q = p.tab.cand_Q[cb + c];
+            const int mm = p.tab.cand_m[cb + c];
+            cok[c] = (Q <= R) ? 1 : 0;
+            cqt[c] = (Q > 0.f) ? __fmul_rn(p.omega_D, __fdiv_rn(Q, Dbar)) : -1.f;
+            cph[c] = have_phi ? bufPhi[mm * E + p.tab.cand_k[cb + c]] : 0.f;
+            cmv[c] = (uint8_t)mm;
+        }
+        __syncthreads();
+        const float* ct = p.tab.ctab + (size_t)lp * M * M;
+        const float skip_cost = __fmul_rn(p.omega_D, __fdiv_rn(eps, Dbar));
+        const bool skip_budget = eps <= R;
+        for (int idx = threadIdx.x; idx < ME; idx += blockDim.x) {
+            const int m = idx / E, kp = idx - (idx / E) * E;
+            const int s0 = coff[kp] - cb, s1 = coff[kp + 1] - cb;
+            const float* ctm = ct + m * M;
+            float best = kInf;
+            bool local = false;
+            for (int c = s0; c < s1; ++c) {
+                if (!cok[c]) continue;
+                const int mm = cmv[c];
+                float v = ctm[mm];
+                const float q = cqt[c];
+                if (q >= 0.f) v = __fadd_rn(v, q);
+                if (have_phi) v = __fadd_rn(v, cph[c]);
+                best = fminf(best, v);
+                local |= (mm == m);
+            }
+            if (!local && skip_budget) {
+                float v = skip_cost;
+                if (have_phi) v = __fadd_rn(v, bufPhi[m * E + kp]);
+                best = fminf(best, v);
+            }
+            bufV[idx] = best;
+        }
+        __syncthreads();
+        const float* Pl = p.tab.P + (size_t)(lp - 1) * E * E;
+        for (int idx = threadIdx.x; idx < ME; idx += blockDim.x) {
+            const int m = idx / E, k = idx - (idx / E) * E;
+            const float* Prow = Pl + k * E;
+            const float* Vrow = bufV + m * E;
+            float acc = 0.f;
+            for (int kp = 0; kp < E; ++kp) acc = __fadd_rn(acc, __fmul_rn(__ldg(Prow + kp), Vrow[kp]));
+            bufPhi[idx] = acc;
+        }
+        __syncthreads();
+        have_phi = true;
+    }
+    float* out = p.phi_tabs_out + ((size_t)blockIdx.y * (p.n_thr + 1) + iv) * ME;
+    for (int idx = threadIdx.x; idx < ME; idx += blockDim.x) out[idx] = have_phi ? bufPhi[idx] : 0.f;
+    if (threadIdx.x == 0 && iv == 0 && blockIdx.y == 0) *p.dbar_shared_out = Dbar;
+}
+
 }  // namespace
+
+cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStream_t st) {
+    if (p.T <= 0 || n_depth <= 0) return cudaSuccess;
+    const size_t MC = (size_t)p.tab.max_layer_cand;
+    // At most 2 * 1024 + 2 * 1024 floats plus 2 KB of flags (M * E <= 1024): under 48 KB.
+    const size_t smem = (2 * (size_t)p.M * p.E + 2 * MC) * sizeof(float) + ((MC + 3) / 4) * 2 * sizeof(float);
+    lookahead_shared_kernel<<<dim3(p.n_thr + 1, n_depth), 256, smem, st>>>(p);
+    return cudaGetLastError();
+}
 
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand) {
     const size_t MC = (size_t)max_layer_cand;

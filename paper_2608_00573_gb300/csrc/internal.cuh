@@ -21,6 +21,8 @@ constexpr int kMaxH = 6;
 constexpr int kMaxC = 256;
 constexpr int kMaxCand = 64;        // (1 + n_sub) * M with n_sub <= 3, M <= 16
 constexpr int kMaxME = 1024;        // look-ahead table entries per token
+constexpr size_t kMaxIntervals = 4096;            // shared look-ahead tables per depth and layer
+constexpr size_t kMaxTabFloats = (size_t)16 << 20; // 64 MB of shared look-ahead tables
 constexpr int kGateUp = 128;        // W13 gate/up row interleave
 
 // Device error codes (first one wins).
@@ -31,6 +33,8 @@ struct DevCounters {
     unsigned long long layer_tokens, exec_tokens, skipped, exited;
     unsigned long long pairs_local_exact, pairs_local_sub, pairs_remote_exact, pairs_remote_sub;
     unsigned long long shared_rows, remote_hops, pairs_total;
+    unsigned long long experts_touched, shared_touched;   // (layer, expert) groups with work
+    unsigned long long lookahead_shared;                  // decisions that read a shared look-ahead table
     double delay_ms;
     unsigned int max_budget_ratio_bits;   // non-negative float bits, atomicMax-able
 };
@@ -84,6 +88,16 @@ struct DecideParams {
     const float* cnorm;         // [K_c] centroid norms of this layer
     const int16_t* lhat_tab;    // [K_c] rounded average exit layer of each centroid
     int16_t* lhat_out;          // [T] predicted exit layer (may be NULL)
+    // Shared look-ahead tables of the layer (Dbar = Dbar[0]): one per interval
+    // between consecutive thresholds thr[0..n_thr) of the window and per depth
+    // dmin..top_full, laid out [depth - dmin][interval][M*E].
+    const float* phi_tabs;      // NULL: every token computes its own table
+    const float* dbar_shared;
+    const float* thr;           // sorted distinct Q and eps of layers l+1 .. l+top_full
+    int n_thr;
+    int dmin;
+    float* phi_tabs_out;        // written by the shared-table kernel
+    float* dbar_shared_out;
     // Offline-stage calibration counts (Algorithm 1), accumulated when calib != 0.
     int calib;
     int16_t* prev_target;       // [T] slot-0 target at the previous layer, -1 none
@@ -170,6 +184,7 @@ int router_pass_rows(int n_out);
 int router_ksplit(int T, int d, int num_sms);
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand);
+cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStream_t st);
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);
 cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
                           const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,

@@ -7,6 +7,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <limits>
 #include <mutex>
 #include <string>
 #include <utility>
@@ -103,6 +104,15 @@ struct trimmoe {
     __nv_bfloat16* rt_hi = nullptr;   // [N][E+C][d] router (gamma folded, hi part) then exit head of layer-1
     __nv_bfloat16* rt_lo = nullptr;   // [N][E][d] lo part of gamma * W_r
     float* rt_bias = nullptr;         // [N][E+C]
+    // Shared look-ahead tables: per layer the sorted distinct thresholds (Q of
+    // the candidates and eps of the window's layers), the depths tabulated and
+    // the table workspace of the current layer.
+    std::vector<float> h_thr;         // flat, layer after layer
+    std::vector<int> thr_off;         // [N + 1]
+    std::vector<int> tab_depths;      // [N] depths tabulated (0: none)
+    float* thr = nullptr;
+    float* phi_tabs = nullptr;
+    float* dbar_shared = nullptr;     // [1]
     float* cnorm = nullptr;           // [N][K_c] centroid norms
     int16_t* lhat = nullptr;          // [N][K_c] rounded average exit layers
     float* zbuf = nullptr;            // [rows_part][E+C+K_c] partial logits
@@ -374,6 +384,32 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         return create_fail(TRIMMOE_ERR_UNSUPPORTED, "create: candidate lists too long for the decision kernel");
     }
     h->max_layer_cand = max_layer_cand;
+    // Look-ahead thresholds (Eq. 39): Phi of layer l depends on R only through
+    // Q <= R and eps <= R over layers l+1 .. l+top, so the sorted distinct
+    // values split R into intervals of equal tables.  Depths below the full
+    // window are tabulated only when exit prediction can shorten it.
+    h->thr_off.assign(N + 1, 0);
+    h->tab_depths.assign(N, 0);
+    size_t tab_floats = 0;
+    for (int l = 0; l < N; ++l) {
+        const int top = std::min(c.H - 1, N - 1 - l);
+        std::vector<float> v;
+        for (int j = 1; j <= top; ++j) {
+            const int lp = l + j;
+            v.push_back(tab->eps[lp]);
+            for (int i = coff[(size_t)lp * (E + 1)]; i < coff[(size_t)lp * (E + 1) + E]; ++i) v.push_back(cq[i]);
+        }
+        std::sort(v.begin(), v.end());
+        v.erase(std::unique(v.begin(), v.end()), v.end());
+        const int depths = top <= 0 ? 0 : (c.n_centroids > 0 ? top : 1);
+        const size_t need = (size_t)depths * (v.size() + 1) * M * E;
+        if (v.size() + 1 <= kMaxIntervals && need <= kMaxTabFloats) {
+            h->tab_depths[l] = depths;
+            tab_floats = std::max(tab_floats, need);
+        }
+        h->h_thr.insert(h->h_thr.end(), v.begin(), v.end());
+        h->thr_off[l + 1] = (int)h->h_thr.size();
+    }
 
     // Router tables of kernel a0 (built from the borrowed device weights): per
     // layer, rows [0, E) hold gamma_l * W_r[l] split exactly into bf16 hi + lo
@@ -458,7 +494,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
               h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, 1) && h->dalloc(&h->dev_err, 1) &&
               h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2) &&
-              h->dalloc(&h->prev_target, T);
+              h->dalloc(&h->prev_target, T) && h->dalloc(&h->phi_tabs, std::max<size_t>(tab_floats, 1)) &&
+              h->dalloc(&h->thr, std::max<size_t>(h->h_thr.size(), 1)) && h->dalloc(&h->dbar_shared, 1);
     h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
     ok = ok && h->dalloc(&h->c_counts, h->n_counts);
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
@@ -470,6 +507,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     up(h->cand_m, cm.data(), cm.size());
     up(h->cand_k, ck.data(), ck.size());
     up(h->cand_Q, cq.data(), cq.size() * 4);
+    if (!h->h_thr.empty()) up(h->thr, h->h_thr.data(), h->h_thr.size() * 4);
     up(h->cand_off, coff.data(), coff.size() * 4);
     up(h->ctab, ctab.data(), ctab.size() * 4);
     up(h->rt_hi, rhi.data(), rhi.size() * 2);
@@ -575,6 +613,18 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.cnorm = h->cnorm + (size_t)layer * Kc;
     dp.lhat_tab = h->lhat + (size_t)layer * Kc;
     dp.lhat_out = (out && out->lhat) ? out->lhat : nullptr;
+    // Shared tables pay off once the tokens outnumber the tables severalfold.
+    const int top_full = std::min(c.H - 1, c.N - 1 - layer);
+    const int n_thr = h->thr_off[layer + 1] - h->thr_off[layer];
+    const int n_depth = h->tab_depths[layer];
+    const bool shared_tabs = n_depth > 0 && (size_t)(n_thr + 1) * n_depth * 4 <= (size_t)T;
+    dp.phi_tabs = shared_tabs ? h->phi_tabs : nullptr;
+    dp.dbar_shared = h->dbar_shared;
+    dp.thr = h->thr + h->thr_off[layer];
+    dp.n_thr = n_thr;
+    dp.dmin = top_full - n_depth + 1;
+    dp.phi_tabs_out = h->phi_tabs;
+    dp.dbar_shared_out = h->dbar_shared;
     dp.calib = h->calib;
     dp.prev_target = h->prev_target;
     dp.c_trans = h->c_counts;
@@ -611,7 +661,11 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.tab.eps = h->eps;
     dp.ctr = h->ctr;
 
-    e = h->timed(K_DECIDE, st, [&] { return launch_decide(dp, h->num_sms, st); });
+    e = h->timed(K_DECIDE, st, [&] {
+        cudaError_t e2 = cudaSuccess;
+        if (shared_tabs) e2 = launch_lookahead_shared(dp, n_depth, st);
+        return e2 == cudaSuccess ? launch_decide(dp, h->num_sms, st) : e2;
+    });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("decide: ") + cudaGetErrorString(e));
 
     CompactParams cp;
@@ -667,7 +721,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm down: ") + cudaGetErrorString(e));
     h->n_gemm_up++;
     h->n_gemm_down++;
-    h->launches += 8;
+    h->launches += 8 + (shared_tabs ? 1 : 0);
     if (has_sh) {
         GemmLaunch s1 = g1;
         s1.tmB = &h->tmW13sh[layer];
@@ -837,6 +891,11 @@ extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) 
     out->flops_gemm_up = 2.0 * dc.pairs_total * n13F * c.d + 2.0 * dc.shared_rows * 2.0 * c.F_sh * c.d;
     out->flops_gemm_down = 2.0 * dc.pairs_total * (double)c.d * c.F + 2.0 * dc.shared_rows * (double)c.d * c.F_sh;
     out->gemm_flops = out->flops_gemm_up + out->flops_gemm_down;
+    const double dd = c.d, FF = c.F, Fs = c.F_sh;
+    out->bytes_gemm_up = 2.0 * ((double)dc.experts_touched * n13F * dd + (double)dc.shared_touched * 2.0 * Fs * dd +
+                                (double)dc.pairs_total * (dd + FF) + (double)dc.shared_rows * (dd + Fs));
+    out->bytes_gemm_down = 2.0 * ((double)dc.experts_touched * dd * FF + (double)dc.shared_touched * dd * Fs +
+                                  (double)dc.pairs_total * (FF + dd) + (double)dc.shared_rows * (Fs + dd));
     out->ms_decide = h->ms[K_DECIDE];
     out->ms_compact = h->ms[K_COMPACT];
     out->ms_gather = h->ms[K_GATHER];
@@ -844,6 +903,7 @@ extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) 
     out->ms_gemm_down = h->ms[K_GEMM_DOWN];
     out->ms_combine = h->ms[K_COMBINE];
     out->ms_router = h->ms[K_ROUTER];
+    out->lookahead_shared = dc.lookahead_shared;
     out->n_gemm_up = h->n_gemm_up;
     out->n_gemm_down = h->n_gemm_down;
     if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "stats: a kernel timed out waiting");

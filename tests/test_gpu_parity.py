@@ -268,3 +268,31 @@ def test_layer_parity_with_exit_prediction(name, kw):
     assert capped > 0
     eng.close()
     torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("n_centroids", [0, 32])
+def test_shared_lookahead_tables_with_mixed_budgets(n_centroids):
+    """Many tokens of one budget read the look-ahead table (Eq. 39) of their
+    remaining-budget interval, computed once per layer; tokens of another budget
+    compute their own.  Both must equal the oracle, which computes every table
+    per token.  Remaining budgets are spread over the whole range, and with exit
+    prediction the window is shortened for some tokens."""
+    import torch
+    cfg = small_cfg(name=f"shared_phi_{n_centroids}", N=4, d=256, E=60, k=4, F=128, F_sh=128, T=4096, M=10,
+                    H=3, zipf_s=1.0, seed=97, n_centroids=n_centroids)
+    eng, om, tables, small, experts = make_engine(cfg, theta=0.6, exit_bias=1.0)
+    tok = W.make_tokens(cfg)
+    rng = np.random.default_rng(7)
+    odd = np.arange(cfg.T) % 2 == 1
+    tok["Dbar"][odd] = np.float32(cfg.budget * 0.5)
+    tok["Dhat"] = (tok["Dbar"] * rng.random(cfg.T).astype(np.float32) ** 3).astype(np.float32)
+    dev = eng.tokens_to_device(tok)
+    eng.reset_stats()
+    sample = rng.choice(cfg.T, size=384, replace=False)
+    for l in range(cfg.N):
+        compare_layer(cfg, om, eng, l, dev, experts, row_sample=sample)
+    st = eng.stats()
+    print(n_centroids, st["lookahead_shared"], st["layer_tokens"])
+    assert 0 < st["lookahead_shared"] < st["layer_tokens"]
+    eng.close()
+    torch.cuda.synchronize()
