@@ -143,6 +143,8 @@ def workload_config(args):
     cfg = W.CONFIGS[args.config]
     if args.exit_prediction:
         cfg = cfg.replace(n_centroids=args.exit_prediction)
+    if args.budget:
+        cfg = cfg.replace(budget=args.budget)      # same calibrated thresholds, other Dbar
     if args.layers or args.tokens:
         over = {}
         if args.layers:
@@ -375,6 +377,7 @@ def main():
     ap.add_argument("--config", default="mixtral")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--budget", type=float, default=0.0, help="per-token quality budget Dbar (default: the workload's)")
     ap.add_argument("--layers", type=int, default=0, help="profiling only: first N layers of the workload")
     ap.add_argument("--tokens", type=int, default=0, help="profiling only: T tokens instead of the workload's")
     ap.add_argument("--exit-prediction", type=int, default=0,
