@@ -41,13 +41,15 @@ class OrModel(C.Structure):
                [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref", "phi_beta", "norm_eps")] + [
         ("place", C.c_void_p), ("sim", C.c_void_p), ("sub_thresh", C.c_void_p),
         ("trans", C.c_void_p), ("comp", C.c_void_p), ("P", C.c_void_p), ("theta", C.c_void_p),
-        ("lambda_", C.c_void_p), ("eps", C.c_void_p), ("n_centroids", C.c_int)]
+        ("lambda_", C.c_void_p), ("eps", C.c_void_p), ("n_centroids", C.c_int),
+        ("attn_heads", C.c_int), ("attn_kv_heads", C.c_int), ("head_dim", C.c_int), ("attn_seq", C.c_int),
+        ("rope_theta", C.c_float)]
 
 
 class OrLayerWeights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in
                 ("W_r", "b_r", "W_x_prev", "b_x_prev", "W13", "W2", "W13_sh", "W2_sh", "W_norm",
-                 "centroids", "centroid_exit")]
+                 "centroids", "centroid_exit", "W_attn_norm", "W_qkv", "W_o")]
 
 
 class OrTokens(C.Structure):
@@ -107,6 +109,11 @@ def lib():
             L.or_ffn_row.argtypes = [i, i, i, vp, vp, vp, vp]
             L.or_layer_step.argtypes = [vp, vp, i, i, vp, vp, vp, vp, i]
             L.or_layer_step.restype = i
+            L.or_layer_step_block.argtypes = [vp, vp, i, i, vp, vp, vp, vp, vp, i]
+            L.or_layer_step_block.restype = i
+            L.or_attention.argtypes = [vp, vp, i, vp, vp, vp, vp, i]
+            L.or_attention.restype = i
+            L.or_rope.argtypes = [vp, i, i, C.c_double, vp]
             L.or_forward.argtypes = [vp, vp, i, vp, vp, i]
             L.or_forward.restype = i
             L.or_max_threads.restype = i
@@ -145,7 +152,9 @@ class OracleModel:
             trans=_p(keep("trans", t["trans"], np.float32)), comp=_p(keep("comp", t["comp"], np.float32)),
             P=_p(keep("P", t["P"] if t["P"].size else np.zeros((1, cfg.E, cfg.E)), np.float32)),
             theta=_p(keep("theta", t["theta"], np.float32)), lambda_=_p(keep("lam", t["lam"], np.float32)),
-            eps=_p(keep("eps", t["eps"], np.float32)), n_centroids=cfg.n_centroids)
+            eps=_p(keep("eps", t["eps"], np.float32)), n_centroids=cfg.n_centroids,
+            attn_heads=cfg.attn_heads, attn_kv_heads=cfg.attn_kv_heads, head_dim=cfg.head_dim,
+            attn_seq=cfg.attn_seq, rope_theta=cfg.rope_theta)
         self.small = {k: (None if v is None else np.ascontiguousarray(v)) for k, v in small.items()}
         self.experts = experts   # dict of numpy arrays (bf16 bits) per layer or full, or None
 
@@ -165,11 +174,15 @@ class OracleModel:
         if self.cfg.n_centroids and s.get("centroids") is not None:
             cc = np.ascontiguousarray(s["centroids"][l], dtype=np.uint16)
             ce = np.ascontiguousarray(s["centroid_exit"][l], dtype=np.float32)
+        an = None
+        if self.cfg.attn_heads and s.get("W_attn_norm") is not None:
+            an = np.ascontiguousarray(s["W_attn_norm"][l], dtype=np.uint16)
         lw = OrLayerWeights(W_r=_p(wr), b_r=_p(br), W_x_prev=_p(wx), b_x_prev=_p(bx),
                             W13=_p(ex.get("W13")), W2=_p(ex.get("W2")),
                             W13_sh=_p(ex.get("W13_sh")), W2_sh=_p(ex.get("W2_sh")), W_norm=_p(wn),
-                            centroids=_p(cc), centroid_exit=_p(ce))
-        lw._keep = (wr, br, wx, bx, ex, wn, cc, ce)
+                            centroids=_p(cc), centroid_exit=_p(ce), W_attn_norm=_p(an),
+                            W_qkv=_p(ex.get("W_qkv")), W_o=_p(ex.get("W_o")))
+        lw._keep = (wr, br, wx, bx, ex, wn, cc, ce, an)
         return lw
 
 
@@ -200,19 +213,45 @@ def alloc_layer_out(T, cfg):
     return OrLayerOut(**{k: _p(v) for k, v in o.items()}), o
 
 
-def layer_step(om: OracleModel, l, h, tok, experts_l=None, row_mask=None, nthreads=0):
-    """Run one layer; returns (h_out, tokens_out, outputs). Inputs are not modified."""
+def layer_step(om: OracleModel, l, h, tok, experts_l=None, row_mask=None, nthreads=0, h_mid=None):
+    """Run one layer; returns (h_out, tokens_out, outputs). Inputs are not modified.
+    With an attention sublayer, h_mid (bf16 bits [T][d]) supplies the state after
+    attention; None computes it."""
     T = h.shape[0]
     h = np.array(h, dtype=np.uint16, copy=True, order="C")
     st, arrs = tokens_struct({k: np.array(v, copy=True) for k, v in tok.items()})
     out_s, out = alloc_layer_out(T, om.cfg)
     lw = om.layer_weights(l, experts_l)
     rm = None if row_mask is None else np.ascontiguousarray(row_mask, dtype=np.uint8)
-    rc = lib().or_layer_step(C.byref(om.m), C.byref(lw), l, T, _p(h), C.byref(st), C.byref(out_s),
-                             _p(rm), nthreads)
+    hm = None if h_mid is None else np.ascontiguousarray(h_mid, dtype=np.uint16)
+    rc = lib().or_layer_step_block(C.byref(om.m), C.byref(lw), l, T, _p(h), _p(hm), C.byref(st),
+                                   C.byref(out_s), _p(rm), nthreads)
     if rc:
         raise RuntimeError(f"or_layer_step failed: {rc}")
     return h, arrs, out
+
+
+def attention(om: OracleModel, l, h, alive, experts_l=None, row_mask=None, nthreads=0):
+    """State after the attention sublayer of layer l (bf16 bits [T][d]); rows of
+    tokens that are not live or not in row_mask are copies of h."""
+    T = h.shape[0]
+    h = np.ascontiguousarray(h, dtype=np.uint16)
+    out = np.zeros_like(h)
+    lw = om.layer_weights(l, experts_l)
+    al = np.ascontiguousarray(alive, dtype=np.uint8)
+    rm = None if row_mask is None else np.ascontiguousarray(row_mask, dtype=np.uint8)
+    rc = lib().or_attention(C.byref(om.m), C.byref(lw), T, _p(h), _p(al), _p(rm), _p(out), nthreads)
+    if rc:
+        raise RuntimeError(f"or_attention failed: {rc}")
+    return out
+
+
+def rope(x, pos, theta):
+    """Rotary embedding of one head vector (float64)."""
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.zeros_like(x)
+    lib().or_rope(_p(x), x.size, int(pos), float(theta), _p(y))
+    return y
 
 
 def forward(om: OracleModel, h, tok, nthreads=0):

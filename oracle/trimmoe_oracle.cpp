@@ -34,7 +34,11 @@
 //    is local and eps_l' <= R; exit is not modelled inside the look-ahead; zero
 //    beyond the last layer;
 //  * action choice (Eq. 40): ties go EXEC, then SKIP, then EXIT; exit only when the
-//    best alternative's total is > 0 (Sec. V-A).
+//    best alternative's total is > 0 (Sec. V-A);
+//  * full block (optional): the attention sublayer runs for every live token
+//    before the MoE decision (Sec. III-C: a skip bypasses only the FFN); the
+//    router reads its output, the exit head of layer l-1 the state entering
+//    layer l; a token exiting at layer l leaves with that entering state.
 #include <algorithm>
 #include <cmath>
 #include <cstdint>
@@ -93,6 +97,9 @@ typedef struct {
     const float* lambda_;      // [N] slope of Lambda = lambda * I (Eq. 5)
     const float* eps;          // [N] per-layer skip tolerance (Eq. 25)
     int n_centroids;           // K_c centroids per layer for Eq. (36); 0 = no exit prediction
+    // Attention sublayer of the full block (attn_heads = 0: the MoE step alone).
+    int attn_heads, attn_kv_heads, head_dim, attn_seq;
+    float rope_theta;
 } OrModel;
 
 // Weights of one layer (host, bf16 bits).
@@ -108,6 +115,9 @@ typedef struct {
     const uint16_t* W_norm;    // [d] RMSNorm weights of this layer, NULL = no normalisation
     const uint16_t* centroids; // [K_c][d] representations entering this layer (Eq. 36)
     const float* centroid_exit;// [K_c] average exit layer of each centroid's calibration tokens
+    const uint16_t* W_attn_norm; // [d] RMSNorm weights in front of the attention sublayer
+    const uint16_t* W_qkv;     // [(Hq + 2 Hkv) Dh][d]: query heads, then key heads, then value heads
+    const uint16_t* W_o;       // [d][Hq Dh]
 } OrLayerWeights;
 
 // Per-token state (host arrays of length T), updated in place.
@@ -477,12 +487,17 @@ void or_decide_given(const OrModel* md, int l, const int* topk, const float* g, 
 }
 
 // Full per-token decision: router + exit head + or_decide_given.
-void or_decide_token(const OrModel* md, const OrLayerWeights* lw, int l, const uint16_t* h, int s,
-                     float Dhat, float Dbar, float pJ, int last_exec, OrDecision* out, float* z_out) {
+// The router reads h_moe, the input of the MoE sublayer; the exit head of layer
+// l-1 and the exit prediction read h_in, the representation entering layer l.
+// Without an attention sublayer both are the same state.
+void or_decide_token2(const OrModel* md, const OrLayerWeights* lw, int l, const uint16_t* h_moe,
+                      const uint16_t* h_in, int s, float Dhat, float Dbar, float pJ, int last_exec,
+                      OrDecision* out, float* z_out) {
     std::vector<float> z(md->E), p(md->E);
     int topk[16];
     float g[16], I;
-    or_router(md, lw->W_r, lw->b_r, lw->W_norm, h, z.data(), p.data(), topk, g, &I);
+    or_router(md, lw->W_r, lw->b_r, lw->W_norm, h_moe, z.data(), p.data(), topk, g, &I);
+    const uint16_t* h = h_in;
     float xi = -1.0f;
     if (l > 0 && last_exec && lw->W_x_prev)
         xi = or_exit_conf(md, lw->W_x_prev, lw->b_x_prev, h, lw->W_norm != nullptr, nullptr);
@@ -518,6 +533,114 @@ void or_decide_token(const OrModel* md, const OrLayerWeights* lw, int l, const u
     if (z_out) for (int e = 0; e < md->E; ++e) z_out[e] = z[e];
 }
 
+void or_decide_token(const OrModel* md, const OrLayerWeights* lw, int l, const uint16_t* h, int s,
+                     float Dhat, float Dbar, float pJ, int last_exec, OrDecision* out, float* z_out) {
+    or_decide_token2(md, lw, l, h, h, s, Dhat, Dbar, pJ, last_exec, out, z_out);
+}
+
+// ------------------------------------------------------- attention sublayer
+//
+// The paper keeps attention local to the token's server and treats it as a fixed
+// per-layer term (Sec. III-C, attention placement): a skip bypasses only the FFN
+// sublayer, the attention sublayer still runs.  Its arithmetic follows the
+// model families of Sec. VI-A (pre-norm transformer blocks): RMSNorm, rotary
+// position embedding, grouped-query causal softmax attention, output projection
+// with the residual.
+
+// Rotary position embedding of one head vector of length Dh: element i pairs
+// with i + Dh/2 and turns by the angle pos * theta^(-2i/Dh).
+void or_rope(const double* x, int Dh, int pos, double theta, double* y) {
+    const int half = Dh / 2;
+    for (int i = 0; i < half; ++i) {
+        const double ang = (double)pos * std::pow(theta, -2.0 * i / Dh);
+        const double c = std::cos(ang), sn = std::sin(ang);
+        y[i] = x[i] * c - x[i + half] * sn;
+        y[i + half] = x[i + half] * c + x[i] * sn;
+    }
+}
+
+// h_mid = h + attention(h) for the live tokens with row_mask set (every live
+// token when row_mask is NULL); all other rows of h_mid are copies of h.
+//   a = bf16(h * r * gamma)                        (r: RMS factor of h)
+//   q | k | v = bf16(a W_qkv^T)
+//   q, k <- bf16(rope(q, pos)), bf16(rope(k, pos))  per head, pos = t mod S
+//   o_head = bf16( sum_j softmax_j(q . k_j / sqrt(Dh)) v_j )
+//            over the tokens j of t's sequence (t - pos .. t), query head
+//            hq reading key/value head hq / (Hq / Hkv)
+//   h_mid = bf16(h + o W_o^T)
+// Keys and values come from every token of the sequence, live or not: a token
+// that left keeps its last state, which later tokens still attend to.
+int or_attention(const OrModel* md, const OrLayerWeights* lw, int T, const uint16_t* h, const uint8_t* alive,
+                 const uint8_t* row_mask, uint16_t* h_mid, int nthreads) {
+    const int d = md->d, Hq = md->attn_heads, Hkv = md->attn_kv_heads, Dh = md->head_dim, S = md->attn_seq;
+    if (Hq <= 0 || Hkv <= 0 || Hq % Hkv || Dh <= 0 || Dh % 2 || S <= 0 || !lw->W_qkv || !lw->W_o ||
+        !lw->W_attn_norm)
+        return -1;
+    const int nq = Hq * Dh, nkv = Hkv * Dh, nqkv = nq + 2 * nkv, grp = Hq / Hkv;
+    std::memcpy(h_mid, h, (size_t)T * d * sizeof(uint16_t));
+    std::vector<char> query(T, 0), need(T, 0);
+    for (int t = 0; t < T; ++t) {
+        if (!alive[t] || (row_mask && !row_mask[t])) continue;
+        query[t] = 1;
+        for (int j = t - t % S; j <= t; ++j) need[j] = 1;
+    }
+    // Projections of the tokens needed, RoPE on query and key heads.
+    std::vector<uint16_t> qkv((size_t)T * nqkv, 0);
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#pragma omp parallel for schedule(dynamic, 4)
+#endif
+    for (int t = 0; t < T; ++t) {
+        if (!need[t]) continue;
+        const uint16_t* hr = h + (size_t)t * d;
+        const double r = or_rms_factor(hr, d, md->norm_eps);
+        std::vector<uint16_t> a(d);
+        for (int i = 0; i < d; ++i) a[i] = d2bf((double)bf2f(hr[i]) * r * (double)bf2f(lw->W_attn_norm[i]));
+        uint16_t* out = qkv.data() + (size_t)t * nqkv;
+        for (int o = 0; o < nqkv; ++o) out[o] = d2bf(dot_bf16(a.data(), lw->W_qkv + (size_t)o * d, d));
+        const int pos = t % S;
+        std::vector<double> x(Dh), y(Dh);
+        for (int hh = 0; hh < Hq + Hkv; ++hh) {          // query heads, then key heads
+            uint16_t* v = out + (size_t)hh * Dh;
+            for (int i = 0; i < Dh; ++i) x[i] = bf2f(v[i]);
+            or_rope(x.data(), Dh, pos, (double)md->rope_theta, y.data());
+            for (int i = 0; i < Dh; ++i) v[i] = d2bf(y[i]);
+        }
+    }
+    const double scale = 1.0 / std::sqrt((double)Dh);
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 4)
+#endif
+    for (int t = 0; t < T; ++t) {
+        if (!query[t]) continue;
+        const int j0 = t - t % S;
+        const uint16_t* qt = qkv.data() + (size_t)t * nqkv;
+        std::vector<uint16_t> o(nq);
+        std::vector<double> w(t - j0 + 1), acc(Dh);
+        for (int hq = 0; hq < Hq; ++hq) {
+            const int g = hq / grp;
+            double mx = -std::numeric_limits<double>::infinity();
+            for (int j = j0; j <= t; ++j) {
+                const uint16_t* kj = qkv.data() + (size_t)j * nqkv + nq + (size_t)g * Dh;
+                w[j - j0] = dot_bf16(qt + (size_t)hq * Dh, kj, Dh) * scale;
+                mx = std::max(mx, w[j - j0]);
+            }
+            double den = 0.0;
+            for (int j = j0; j <= t; ++j) { w[j - j0] = std::exp(w[j - j0] - mx); den += w[j - j0]; }
+            std::fill(acc.begin(), acc.end(), 0.0);
+            for (int j = j0; j <= t; ++j) {
+                const uint16_t* vj = qkv.data() + (size_t)j * nqkv + nq + nkv + (size_t)g * Dh;
+                for (int i = 0; i < Dh; ++i) acc[i] += w[j - j0] / den * (double)bf2f(vj[i]);
+            }
+            for (int i = 0; i < Dh; ++i) o[(size_t)hq * Dh + i] = d2bf(acc[i]);
+        }
+        const uint16_t* hr = h + (size_t)t * d;
+        for (int c = 0; c < d; ++c)
+            h_mid[(size_t)t * d + c] = d2bf((double)bf2f(hr[c]) + dot_bf16(o.data(), lw->W_o + (size_t)c * nq, nq));
+    }
+    return 0;
+}
+
 // ------------------------------------------------------------- expert FFN
 
 // One expert on one row: act = silu(x W1^T) * (x W3^T) (SwiGLU) or relu(x W1^T),
@@ -551,10 +674,26 @@ void or_ffn_row(int d, int F, int act, const uint16_t* W13, const uint16_t* W2, 
 // decisions gate).  h is bf16 [T][d], updated in place.  row_mask (may be NULL)
 // limits the FFN/combine to the selected tokens; decisions, state and
 // compaction are always computed for every token.
-int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uint16_t* h,
-                  OrTokens* tk, OrLayerOut* out, const uint8_t* row_mask, int nthreads) {
+//
+// With an attention sublayer (md->attn_heads > 0) the layer is the full block:
+// h_mid = h + attention(h) for the live tokens (computed here when h_mid_in is
+// NULL, else taken from h_mid_in), the router, the experts and the residual read
+// h_mid, the exit head reads h; executed and skipped tokens leave with
+// h_mid + FFN (h_mid alone for a skip without a shared expert), while a token
+// that exits at this layer keeps h (layers from l on do not run for it).
+int or_layer_step_block(const OrModel* md, const OrLayerWeights* lw, int l, int T, uint16_t* h,
+                        const uint16_t* h_mid_in, OrTokens* tk, OrLayerOut* out, const uint8_t* row_mask,
+                        int nthreads) {
     const int K = md->k, E = md->E, d = md->d;
     if (l < 0 || l >= md->N || T < 0) return -1;
+    const bool block = md->attn_heads > 0;
+    std::vector<uint16_t> hmid;
+    if (block) {
+        hmid.resize((size_t)T * d);
+        if (h_mid_in) std::memcpy(hmid.data(), h_mid_in, (size_t)T * d * sizeof(uint16_t));
+        else if (or_attention(md, lw, T, h, tk->alive, nullptr, hmid.data(), nthreads)) return -1;
+    }
+    const uint16_t* hm = block ? hmid.data() : h;
     std::vector<OrDecision> dec(T);
 #ifdef _OPENMP
     if (nthreads > 0) omp_set_num_threads(nthreads);
@@ -563,8 +702,8 @@ int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uin
     for (int t = 0; t < T; ++t) {
         OrDecision& D = dec[t];
         if (!tk->alive[t]) { std::memset(&D, 0, sizeof(D)); D.action = A_DEAD; D.xi = -1.0f; continue; }
-        or_decide_token(md, lw, l, h + (size_t)t * d, tk->s[t], tk->Dhat[t], tk->Dbar[t], tk->pJ[t],
-                        tk->last_exec[t], &D, nullptr);
+        or_decide_token2(md, lw, l, hm + (size_t)t * d, h + (size_t)t * d, tk->s[t], tk->Dhat[t], tk->Dbar[t],
+                         tk->pJ[t], tk->last_exec[t], &D, nullptr);
     }
     // Compaction: executed (token, slot) pairs stably ordered by expert, then
     // the tokens that run the shared expert (executed or skipped), by token.
@@ -587,7 +726,7 @@ int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uin
     for (size_t i = 0; i < shared_rows.size(); ++i) pos_sh[shared_rows[i]] = (int)i;
 
     // Expert FFN on selected rows, then the gate-weighted combine with residual.
-    std::vector<uint16_t> hin(h, h + (size_t)T * d);
+    std::vector<uint16_t> hin(hm, hm + (size_t)T * d);
 #ifdef _OPENMP
 #pragma omp parallel for schedule(dynamic, 1)
 #endif
@@ -658,11 +797,16 @@ int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uin
     return 0;
 }
 
+int or_layer_step(const OrModel* md, const OrLayerWeights* lw, int l, int T, uint16_t* h,
+                  OrTokens* tk, OrLayerOut* out, const uint8_t* row_mask, int nthreads) {
+    return or_layer_step_block(md, lw, l, T, h, nullptr, tk, out, row_mask, nthreads);
+}
+
 // Whole forward: layers 0..N-1 (the layer loop of Algorithm 2).
 int or_forward(const OrModel* md, const OrLayerWeights* lws, int T, uint16_t* h, OrTokens* tk,
                int nthreads) {
     for (int l = 0; l < md->N; ++l) {
-        int rc = or_layer_step(md, &lws[l], l, T, h, tk, nullptr, nullptr, nthreads);
+        int rc = or_layer_step_block(md, &lws[l], l, T, h, nullptr, tk, nullptr, nullptr, nthreads);
         if (rc) return rc;
     }
     return 0;

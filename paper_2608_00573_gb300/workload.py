@@ -9,10 +9,11 @@ Shapes stand in for the three models the paper evaluates (Sec. VI-A:
 Switch-Base-8E, Qwen-MoE-A2.7B, Mixtral-8x7B); the paper's weights, datasets
 and testbed are not available, so every value here is synthetic:
 
-* weights ~ N(0, 1/fan_in) stored as bf16; hidden states ~ N(0, 1) in bf16;
+* weights ~ N(0, 1/fan_in) stored as bf16 (attention projections included);
+  hidden states ~ N(0, 1) in bf16;
   RMSNorm weights of the MoE sublayer ~ N(1, 0.1^2) in bf16 (all three models
   are pre-norm; without the norm a random-weight SwiGLU stack overflows bf16
-  within about ten layers);
+  within about ten layers), and likewise for the attention sublayer;
 * router bias b_e = -s * ln(e + 1), which makes expert popularity Zipf(s);
 * users are blocks of 128 tokens; each user's access server a(i) (Eq. 12) is
   drawn Zipf(1.0) over the M servers, with p_J = 0.9 and a per-token budget
@@ -83,7 +84,17 @@ class WorkloadConfig:
     norm: bool = True                # pre-FFN RMSNorm of the MoE sublayer
     norm_eps: float = 1e-6
     n_centroids: int = 0             # K_c centroids per layer for exit prediction (Eq. 36); 0 = off
+    # Attention sublayer of the full block (0 heads = the MoE step alone).
+    attn_heads: int = 0              # query heads
+    attn_kv_heads: int = 0           # key/value heads (grouped-query attention)
+    head_dim: int = 0
+    attn_seq: int = 128              # tokens per sequence (one user's block)
+    rope_theta: float = 1.0e6
     seed: int = 0
+
+    @property
+    def n_qkv(self) -> int:
+        return (self.attn_heads + 2 * self.attn_kv_heads) * self.head_dim
 
     @property
     def n13(self) -> int:
@@ -125,6 +136,20 @@ CONFIGS = {
         renorm_topk=1, T=256, zipf_s=1.5, skip_target=0.11, exit_target=0.40,
         exit_peak=18.0, exit_width=4.0, phi_beta=PHI_BETA, seed=4),
 }
+
+
+# Attention shapes of the three model families (query heads, key/value heads,
+# head dimension): Switch-Base 12 x 64, Qwen-MoE-A2.7B 16 x 128, Mixtral-8x7B
+# 32 query / 8 key-value heads of 128.
+ATTN_SHAPES = {"switch": (12, 12, 64), "qwen": (16, 16, 128), "mixtral": (32, 8, 128)}
+
+
+def with_attention(cfg: WorkloadConfig) -> WorkloadConfig:
+    """The workload with the attention sublayer of its model family in front of
+    every MoE step (the full transformer block)."""
+    fam = next(k for k in ATTN_SHAPES if cfg.name.startswith(k))
+    hq, hkv, dh = ATTN_SHAPES[fam]
+    return cfg.replace(attn_heads=hq, attn_kv_heads=hkv, head_dim=dh)
 
 
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -246,6 +271,9 @@ def make_small_weights(cfg: WorkloadConfig, calib: Optional[dict] = "auto") -> d
     else:
         b_x[:, 0] = -30.0                                     # no exits
     out = dict(W_r=W_r, b_r=b_r, W_x=W_x, b_x=b_x, W_norm=W_norm)
+    if cfg.attn_heads:
+        out["W_attn_norm"] = f32_to_bf16_bits((1.0 + 0.1 * np.random.default_rng([cfg.seed, 707]).standard_normal(
+            (N, d))).astype(np.float32))
     if cfg.n_centroids:
         out.update(make_centroids(cfg))
     return out
@@ -278,6 +306,11 @@ def make_expert_weights_host(cfg: WorkloadConfig) -> dict:
     if cfg.F_sh:
         out["W13_sh"] = _normal_bf16(rng, (N, 2 * cfg.F_sh, d), 1.0 / math.sqrt(d))
         out["W2_sh"] = _normal_bf16(rng, (N, d, cfg.F_sh), 1.0 / math.sqrt(cfg.F_sh))
+    if cfg.attn_heads:
+        ra = np.random.default_rng([cfg.seed, 808])
+        hd = cfg.attn_heads * cfg.head_dim
+        out["W_qkv"] = _normal_bf16(ra, (N, cfg.n_qkv, d), 1.0 / math.sqrt(d))
+        out["W_o"] = _normal_bf16(ra, (N, d, hd), 1.0 / math.sqrt(hd))
     return out
 
 
@@ -300,6 +333,16 @@ def make_expert_weights_device(cfg: WorkloadConfig, device="cuda") -> dict:
             W13_sh[l].normal_(0.0, 1.0 / math.sqrt(d), generator=g)
             W2_sh[l].normal_(0.0, 1.0 / math.sqrt(cfg.F_sh), generator=g)
         out.update(W13_sh=W13_sh, W2_sh=W2_sh)
+    if cfg.attn_heads:
+        ga = torch.Generator(device=device)
+        ga.manual_seed(cfg.seed * 7919 + 808)
+        hd = cfg.attn_heads * cfg.head_dim
+        W_qkv = torch.empty((N, cfg.n_qkv, d), dtype=torch.bfloat16, device=device)
+        W_o = torch.empty((N, d, hd), dtype=torch.bfloat16, device=device)
+        for l in range(N):
+            W_qkv[l].normal_(0.0, 1.0 / math.sqrt(d), generator=ga)
+            W_o[l].normal_(0.0, 1.0 / math.sqrt(hd), generator=ga)
+        out.update(W_qkv=W_qkv, W_o=W_o)
     return out
 
 
