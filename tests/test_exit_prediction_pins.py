@@ -26,12 +26,13 @@ def test_nearest_centroid_by_cosine_and_rounding():
         cos = C @ hf / np.linalg.norm(C, axis=1) / np.linalg.norm(hf)
         j = int(np.argmax(cos))
         assert L == int(np.floor(ex[j] + 0.5))
-    # rounding of the average exit layer: halves go up
+    # rounding of the average exit layer: halves go up (a model with one centroid)
+    om1 = O.OracleModel(cfg.replace(n_centroids=1), tables, small)
     one = np.zeros((1, cfg.d), np.uint16)
     one[0] = W.f32_to_bf16_bits(np.ones(cfg.d, np.float32))
     h = one[0]
     for avg, want in [(2.5, 3), (2.49, 2), (3.0, 3), (1.51, 2)]:
-        L, _, _ = O.predict_exit(om, one, np.array([avg], np.float32), h)
+        L, _, _ = O.predict_exit(om1, one, np.array([avg], np.float32), h)
         assert L == want
 
 
