@@ -145,6 +145,8 @@ def workload_config(args):
         cfg = cfg.replace(n_centroids=args.exit_prediction)
     if args.budget:
         cfg = cfg.replace(budget=args.budget)      # same calibrated thresholds, other Dbar
+    if args.full_block:
+        cfg = W.with_attention(cfg)                # attention sublayer in front of every MoE step
     if args.layers or args.tokens:
         over = {}
         if args.layers:
@@ -327,9 +329,18 @@ def run_ours(args):
     # bytes at HBM, whichever is slower.
     per_fwd_flops = st["gemm_flops"] / args.steps
     per_fwd_bytes = (st["bytes_gemm_up"] + st["bytes_gemm_down"]) / args.steps
+    kinds_ms = ("router", "decide", "compact", "gather", "gemm_up", "gemm_down", "combine")
+    if cfg.attn_heads:
+        # Attention sublayer: its projections and attention FLOPs, and per layer the
+        # projection weights once plus the activations it must read and write.
+        hd = cfg.attn_heads * cfg.head_dim
+        per_fwd_flops += (st["flops_attn_gemm"] + st["flops_attn"]) / args.steps
+        per_layer = 2.0 * (cfg.n_qkv * cfg.d + cfg.d * hd) + 2.0 * T * (
+            2 * cfg.d + 2 * cfg.n_qkv + 2 * hd + 2 * cfg.d + cfg.d)
+        per_fwd_bytes += per_layer * cfg.N
+        kinds_ms = kinds_ms + ("attn", "attn_gemm")
     fwd_roof_ms = max(per_fwd_flops / (peaks["bf16_sus"] * 1e12), per_fwd_bytes / (peaks["hbm"] * 1e9)) * 1e3
-    kernel_ms = {k: st[f"ms_{k}"] / args.steps for k in
-                 ("router", "decide", "compact", "gather", "gemm_up", "gemm_down", "combine")}
+    kernel_ms = {k: st[f"ms_{k}"] / args.steps for k in kinds_ms}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
@@ -337,7 +348,10 @@ def run_ours(args):
         "config": {"workload": cfg.name, "T": T, "N": cfg.N, "d": cfg.d, "E": cfg.E, "k": cfg.k, "F": cfg.F,
                    "F_sh": cfg.F_sh, "H": cfg.H, "budget": cfg.budget, "exit_prediction_centroids": cfg.n_centroids,
                    "parallelism": f"replicas{world}",
-                   "l2": "inputs larger than L2 (expert weights and hidden states)"},
+                   "l2": "inputs larger than L2 (expert weights and hidden states)",
+                   "full_block": bool(cfg.attn_heads),
+                   **({"attn_heads": cfg.attn_heads, "attn_kv_heads": cfg.attn_kv_heads, "head_dim": cfg.head_dim,
+                       "attn_seq": cfg.attn_seq} if cfg.attn_heads else {})},
         "roofline": roof,
         "forward_roofline": {"gemm_flops_per_forward": per_fwd_flops, "gemm_bytes_per_forward": per_fwd_bytes,
                              "roofline_ms": fwd_roof_ms, "frac": fwd_roof_ms / ms_step},
@@ -366,7 +380,7 @@ def run_ours(args):
 
 # Revision tag of the timed GEMM kernel; a stored ncu traffic figure is used
 # only when it was taken on this revision.
-KERNEL_REV = "gemm-v1"
+KERNEL_REV = "gemm-v2"
 
 
 def main():
@@ -378,6 +392,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--budget", type=float, default=0.0, help="per-token quality budget Dbar (default: the workload's)")
+    ap.add_argument("--full-block", action="store_true",
+                    help="the full transformer block: the model family's attention sublayer in front of every MoE step")
     ap.add_argument("--layers", type=int, default=0, help="profiling only: first N layers of the workload")
     ap.add_argument("--tokens", type=int, default=0, help="profiling only: T tokens instead of the workload's")
     ap.add_argument("--exit-prediction", type=int, default=0,

@@ -64,10 +64,20 @@ enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
  *  then reports per-kernel device time);
  *  norm_eps: epsilon of the pre-FFN RMSNorm (used when W_norm != NULL);
  *  n_centroids: K_c centroids per layer for the token-similarity exit-point
- *  prediction of Eq. (36) (0 = off, at most 256).
+ *  prediction of Eq. (36) (0 = off, at most 256);
+ *  attn_heads, attn_kv_heads, head_dim, attn_seq, rope_theta: the attention
+ *  sublayer of the full transformer block (attn_heads = 0: the MoE step
+ *  alone).  With it every layer first runs, for every live token, pre-norm
+ *  grouped-query causal attention: attn_heads query heads and attn_kv_heads
+ *  key/value heads of head_dim, rotary embedding with base rope_theta, within
+ *  sequences of attn_seq consecutive tokens (token t sits at position
+ *  t mod attn_seq).  Attention stays local to the token's server (Sec. III-C,
+ *  attention placement): a skip bypasses only the MoE sublayer.
  * Supported: d % 256 == 0; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
  * F_sh % 128 == 0; E <= 128; k <= min(E, 8); C <= 256; M*E <= 1024; H <= 6;
- * n_sub <= 3. */
+ * n_sub <= 3; attention: head_dim 64 or 128, attn_heads % attn_kv_heads == 0,
+ * (attn_heads + 2 attn_kv_heads) * head_dim % 256 == 0, 1 <= attn_seq <= 128,
+ * W_norm required. */
 typedef struct {
     int N, d, E, k, F, F_sh, C, M, H;
     int act;
@@ -78,6 +88,8 @@ typedef struct {
     int profile;
     float norm_eps;
     int n_centroids;
+    int attn_heads, attn_kv_heads, head_dim, attn_seq;
+    float rope_theta;
 } trimmoe_config;
 
 /* Weights (device, bf16 except the biases, borrowed; 16-byte aligned).
@@ -93,7 +105,17 @@ typedef struct {
  *       the router reads h*r*gamma_l (fp32), the experts its bf16 rounding, the
  *       exit head h*r, and the combine adds to h itself (pre-norm residual).
  *  centroids [N][K_c][d] (n_centroids > 0): representations entering layer l
- *       of the token-similarity reference set (Eq. 36); read at create. */
+ *       of the token-similarity reference set (Eq. 36); read at create.
+ *  W_attn_norm [N][d], W_qkv [N][(Hq + 2 Hkv) Dh][d], W_o [N][d][Hq Dh]
+ *       (attn_heads > 0): RMSNorm weights of the attention sublayer, the fused
+ *       query/key/value projection (query heads, then key heads, then value
+ *       heads, Dh rows each) and the output projection.  Layer l then computes
+ *       a = bf16(h r' gamma'), q|k|v = bf16(a W_qkv^T), rotary embedding on q
+ *       and k, causal softmax attention (query head j reads key/value head
+ *       j / (Hq/Hkv)), h_mid = bf16(h + o W_o^T); the router, experts and
+ *       residual read h_mid, the exit head of layer l-1 and the exit prediction
+ *       read h (the state entering the layer), and a token that exits at layer
+ *       l keeps h. */
 typedef struct {
     const void* W_r;
     const float* b_r;
@@ -105,6 +127,9 @@ typedef struct {
     const void* W2_sh;
     const void* W_norm;
     const void* centroids;
+    const void* W_attn_norm;
+    const void* W_qkv;
+    const void* W_o;
 } trimmoe_weights;
 
 /* The paper's input tables (host, copied at create).
@@ -159,7 +184,9 @@ typedef struct {
  *  group_off int32 [E+2]: pairs of expert e are perm[group_off[e] ..
  *  group_off[e+1]), shared rows perm[group_off[E] .. group_off[E+1]);
  *  lhat int16 [T]: predicted exit layer (Eq. 36; N without prediction, -1 for
- *  dead tokens). */
+ *  dead tokens);
+ *  h_attn bf16 [T][d] (full block only): the state after the attention
+ *  sublayer, h_mid (rows of tokens that are not live are unspecified). */
 typedef struct {
     int32_t* topk_idx;
     float* topk_g;
@@ -171,6 +198,7 @@ typedef struct {
     int32_t* perm;
     int32_t* group_off;
     int16_t* lhat;
+    void* h_attn;
 } trimmoe_layer_out;
 
 /* Counters accumulated since create / the last reset (Fig. 5(b) categories). */
@@ -203,6 +231,12 @@ typedef struct {
      * tables shared by all tokens of equal budget instead of computed per token
      * (the results are the same either way). */
     uint64_t lookahead_shared;
+    /* Attention sublayer of the full block: device time (profile != 0) of the
+     * RMSNorm + attention kernels and of the two projection GEMMs, and their
+     * FLOPs (projections 2*T*d*(Hq+2Hkv)Dh + 2*T*Hq*Dh*d; attention
+     * 4*Dh*Hq*(causal query-key pairs)). */
+    double ms_attn, ms_attn_gemm;
+    double flops_attn, flops_attn_gemm;
 } trimmoe_stats_t;
 
 /* Validate, copy the tables, derive the candidate lists V_{l,r} and losses Q,

@@ -34,12 +34,14 @@ class trimmoe_config(C.Structure):
     _fields_ = [(n, C.c_int) for n in ("N", "d", "E", "k", "F", "F_sh", "C", "M", "H", "act",
                                        "renorm_topk", "n_sub", "T_max")] + \
                [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref_ms", "phi_beta")] + \
-               [("profile", C.c_int), ("norm_eps", C.c_float), ("n_centroids", C.c_int)]
+               [("profile", C.c_int), ("norm_eps", C.c_float), ("n_centroids", C.c_int)] + \
+               [(n, C.c_int) for n in ("attn_heads", "attn_kv_heads", "head_dim", "attn_seq")] + \
+               [("rope_theta", C.c_float)]
 
 
 class trimmoe_weights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("W_r", "b_r", "W_x", "b_x", "W13", "W2", "W13_sh", "W2_sh",
-                                          "W_norm", "centroids")]
+                                          "W_norm", "centroids", "W_attn_norm", "W_qkv", "W_o")]
 
 
 class trimmoe_tables(C.Structure):
@@ -54,7 +56,7 @@ class trimmoe_tokens(C.Structure):
 
 class trimmoe_layer_out(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("topk_idx", "topk_g", "I", "xi", "action", "exp_sel",
-                                          "srv_sel", "perm", "group_off", "lhat")]
+                                          "srv_sel", "perm", "group_off", "lhat", "h_attn")]
 
 
 class trimmoe_stats_t(C.Structure):
@@ -69,7 +71,9 @@ class trimmoe_stats_t(C.Structure):
                [("n_gemm_up", C.c_uint64), ("n_gemm_down", C.c_uint64),
                 ("flops_gemm_up", C.c_double), ("flops_gemm_down", C.c_double), ("ms_router", C.c_double),
                 ("bytes_gemm_up", C.c_double), ("bytes_gemm_down", C.c_double),
-                ("lookahead_shared", C.c_uint64)]
+                ("lookahead_shared", C.c_uint64),
+                ("ms_attn", C.c_double), ("ms_attn_gemm", C.c_double), ("flops_attn", C.c_double),
+                ("flops_attn_gemm", C.c_double)]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}
@@ -274,6 +278,9 @@ class Engine:
             "W2_sh": dt(experts["W2_sh"], torch.bfloat16) if cfg.F_sh else None,
             "W_norm": dt(small["W_norm"], torch.bfloat16) if small.get("W_norm") is not None else None,
             "centroids": dt(small["centroids"], torch.bfloat16) if cfg.n_centroids else None,
+            "W_attn_norm": dt(small["W_attn_norm"], torch.bfloat16) if cfg.attn_heads else None,
+            "W_qkv": dt(experts["W_qkv"], torch.bfloat16) if cfg.attn_heads else None,
+            "W_o": dt(experts["W_o"], torch.bfloat16) if cfg.attn_heads else None,
         }
         self.tables = {k: np.ascontiguousarray(v) for k, v in tables.items() if k != "d_ref"}
         self.c_cfg = trimmoe_config(
@@ -281,7 +288,8 @@ class Engine:
             act=cfg.act, renorm_topk=cfg.renorm_topk, n_sub=cfg.n_sub, T_max=T_max,
             omega_T=cfg.omega_T, omega_D=cfg.omega_D, d_ref_ms=float(tables["d_ref"]),
             phi_beta=cfg.phi_beta, profile=1 if profile else 0, norm_eps=cfg.norm_eps,
-            n_centroids=cfg.n_centroids)
+            n_centroids=cfg.n_centroids, attn_heads=cfg.attn_heads, attn_kv_heads=cfg.attn_kv_heads,
+            head_dim=cfg.head_dim, attn_seq=cfg.attn_seq, rope_theta=cfg.rope_theta)
         self.c_w = trimmoe_weights(**{k: _ptr(v) for k, v in self.w.items()})
         t = self.tables
         P = t["P"].astype(np.float32) if t["P"].size else None
@@ -342,7 +350,9 @@ class Engine:
             srv_sel=torch.empty(T * K, dtype=torch.uint8, device=dev),
             perm=torch.full((T * K + T,), -1, dtype=torch.int32, device=dev),
             group_off=torch.empty(E + 2, dtype=torch.int32, device=dev),
-            lhat=torch.empty(T, dtype=torch.int16, device=dev))
+            lhat=torch.empty(T, dtype=torch.int16, device=dev),
+            h_attn=(torch.empty((T, self.cfg.d), dtype=torch.bfloat16, device=dev) if self.cfg.attn_heads
+                    else None))
 
     def stream_ptr(self, stream=None) -> int:
         torch = self.torch

@@ -1,8 +1,12 @@
 // Kernel (d): un-permute and gate-weighted combine with the residual path.
 //
-//   EXEC:  h[t] = bf16( h[t] + sum_j w_j * Y[pos(t, j)] (+ Ysh[t]) )
-//   SKIP:  h[t] = bf16( h[t] + Ysh[t] )    (only with a shared expert)
+//   EXEC:  h[t] = bf16( b[t] + sum_j w_j * Y[pos(t, j)] (+ Ysh[t]) )
+//   SKIP:  h[t] = bf16( b[t] + Ysh[t] )
 //   EXIT / DEAD: untouched.
+// The residual base b is h itself (the MoE step alone: then a skip without a
+// shared expert is not touched either) or the post-attention state of the full
+// block, which executed and skipped tokens carry on while an exiting token
+// keeps the state that entered the layer.
 // w_j are the router gates of the top-k slots, renormalised over the top-k
 // when requested; a substitute expert takes its target's gate.  A skipped
 // layer is the identity (residual) path of Sec. III-B; the shared expert is
@@ -20,7 +24,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
     for (int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; t < p.T;
          t += (gridDim.x * blockDim.x) >> 5) {
         const int a = p.action[t];
-        if (a > 1 || (a == 1 && !p.has_shared)) continue;
+        if (a > 1 || (a == 1 && !p.has_shared && p.h_src == p.h)) continue;
         float w[kMaxK];
         int pos[kMaxK];
         int nj = 0;
@@ -36,8 +40,9 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
         }
         const int psh = p.has_shared ? p.pos_sh[t] : -1;
         uint4* hrow = reinterpret_cast<uint4*>(p.h + (size_t)t * p.d);
+        const uint4* brow = reinterpret_cast<const uint4*>(p.h_src + (size_t)t * p.d);
         for (int c = lane; c < nchunk; c += 32) {
-            const uint4 hv = hrow[c];
+            const uint4 hv = brow[c];
             float acc[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
                             bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
             for (int j = 0; j < nj; ++j) {

@@ -184,10 +184,18 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         float xi = -1.f;
         const bool have_xi = (l > 0) && last_exec && p.has_head;
         if (have_xi) {
+            // The exit head reads the state entering the layer; with an attention
+            // sublayer in front of the MoE step that state has its own RMS factor.
+            float rx = rn;
+            if (p.use_norm && p.sqpart_x) {
+                float sq = 0.f;
+                for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart_x[(size_t)ks * p.T + t]);
+                rx = rsqrtf(sq / (float)p.d + p.norm_eps);
+            }
             for (int c = lane; c < C; c += 32) {
                 float acc = 0.f;
                 for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + c]);
-                xs[c] = __fadd_rn(__fmul_rn(acc, rn), p.bias[E + c]);
+                xs[c] = __fadd_rn(__fmul_rn(acc, rx), p.bias[E + c]);
             }
             __syncwarp();
             if (C == 1) {

@@ -5,9 +5,12 @@
 // that group's weights B (bf16 [N][K], K contiguous):
 //     out[row, :] = epilogue(A[row, :] . B^T)
 // with epilogue = store (down projection), SwiGLU over the interleaved
-// gate/up columns (W13 of a SwiGLU expert) or ReLU (W1 of a ReLU expert).
-// This is the only dense contraction of the layer step (the expert FFN of the
-// executed layers, Sec. III-B/C and the execute branch of Algorithm 2).
+// gate/up columns (W13 of a SwiGLU expert), ReLU (W1 of a ReLU expert) or a
+// residual add (bf16 residual row + accumulator: the attention output
+// projection of the full block).
+// The expert FFN of the executed layers (Sec. III-B/C and the execute branch of
+// Algorithm 2) is the dense contraction of the MoE step; the full block also
+// runs its attention projections through this kernel as a single group.
 //
 // Design (one CTA per SM, persistent, 192 threads):
 //   warp 0      TMA producer (one lane); also owns the TMEM allocation
@@ -94,7 +97,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
                     int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
-                    __nv_bfloat16* __restrict__ out, int ldo, int* err) {
+                    __nv_bfloat16* __restrict__ out, int ldo, int* err,
+                    const __nv_bfloat16* __restrict__ res, int ldr) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -255,6 +259,22 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                             const float x = __uint_as_float(r[i]);
                             v[i] = epi_mode == EPI_RELU ? fmaxf(x, 0.f) : x;
                         }
+                        if (epi_mode == EPI_RESID) {
+                            const uint4* rr = reinterpret_cast<const uint4*>(
+                                res + (size_t)(ti.out_row + row) * ldr + ti.nt * BN + c);
+#pragma unroll
+                            for (int q4 = 0; q4 < 4; ++q4) {
+                                const uint4 w = __ldg(rr + q4);
+                                v[q4 * 8 + 0] += bf16_lo(w.x);
+                                v[q4 * 8 + 1] += bf16_hi(w.x);
+                                v[q4 * 8 + 2] += bf16_lo(w.y);
+                                v[q4 * 8 + 3] += bf16_hi(w.y);
+                                v[q4 * 8 + 4] += bf16_lo(w.z);
+                                v[q4 * 8 + 5] += bf16_hi(w.z);
+                                v[q4 * 8 + 6] += bf16_lo(w.w);
+                                v[q4 * 8 + 7] += bf16_hi(w.w);
+                            }
+                        }
                         store_row32(orow + ti.nt * BN + c, v);
                     }
                 }
@@ -288,7 +308,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     if (g.ngroups <= 0 || g.ngroups > kMaxGroups || g.K % BK != 0) return cudaErrorInvalidValue;
     grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
         *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err);
+        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr);
     return cudaGetLastError();
 }
 

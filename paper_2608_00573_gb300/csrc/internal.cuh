@@ -78,6 +78,7 @@ struct DecideParams {
     float omega_T, omega_D, d_ref;
     const float* zpart;         // [ksplit][T][zs] partial router then exit-head dot products
     const float* sqpart;        // [ksplit][T] partial sums of h^2
+    const float* sqpart_x;      // [ksplit][T] partial sums of the exit head's input^2 (NULL: sqpart)
     const float* bias;          // [E + C] router then exit-head biases of this layer
     int zs, ksplit;
     int use_norm;
@@ -147,13 +148,29 @@ struct GemmLaunch {
     __nv_bfloat16* out;
     int ldo;
     int* err;
+    const __nv_bfloat16* res;   // EPI_RESID: residual rows (same row index as out)
+    int ldr;
 };
 
-enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2 };
+enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2, EPI_RESID = 3 };
+
+// Attention sublayer of the full block (kernels e).
+struct AttnParams {
+    int T, d, S, Hq, Hkv, nqkv;
+    float norm_eps, scale;
+    const __nv_bfloat16* h;       // [T][d] state entering the layer
+    const __nv_bfloat16* gamma;   // [d] RMSNorm weights of the sublayer
+    __nv_bfloat16* a;             // [T][d] normalised input of the q/k/v projection
+    int* goff;                    // [2] {0, T}: the projections' single GEMM group
+    const __nv_bfloat16* qkv;     // [T][nqkv] query heads, key heads, value heads
+    const float2* rope;           // [S][Dh/2] (cos, sin) of the rotary embedding
+    __nv_bfloat16* out;           // [T][Hq*Dh] attention output
+};
 
 struct CombineParams {
     int T, d, k, renorm, has_shared;
-    __nv_bfloat16* h;
+    __nv_bfloat16* h;              // output rows (executed and skipped tokens)
+    const __nv_bfloat16* h_src;    // residual base: h itself, or the post-attention state
     const uint8_t* action;
     const float* topk_g;
     const int32_t* pos_pair;
@@ -192,6 +209,8 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st);
 size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
+cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);
+cudaError_t launch_attention(const AttnParams& p, int head_dim, cudaStream_t st);
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
 
 // Error text for calls made without a handle (read by trimmoe_last_error(NULL)).
@@ -353,6 +372,30 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// ldmatrix / mma.sync fragments (router and attention kernels).
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldmatrix_x2(uint32_t (&r)[2], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];"
+                 : "=r"(r[0]), "=r"(r[1])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
 }
 
 }  // namespace tmoe

@@ -54,7 +54,7 @@ bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_NUM };
+enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
 
 inline float bf16_to_float(uint16_t b) {
     uint32_t u = (uint32_t)b << 16;
@@ -140,6 +140,16 @@ struct trimmoe {
 
     CUtensorMap tmXp, tmAct, tmActSh;
     std::vector<CUtensorMap> tmW13, tmW2, tmW13sh, tmW2sh;
+
+    // attention sublayer of the full block
+    int nqkv = 0;
+    __nv_bfloat16 *qkv = nullptr, *attn_out = nullptr, *hm = nullptr;
+    int* goff_attn = nullptr;
+    float2* rope = nullptr;           // [attn_seq][head_dim/2] (cos, sin)
+    float* sqbuf_x = nullptr;         // [rows_part] partial sums of squares of the layer input
+    CUtensorMap tmAttn;
+    std::vector<CUtensorMap> tmWqkv, tmWo;
+    double flops_attn = 0.0, flops_attn_gemm = 0.0;
 
     // host-buffer forward
     trimmoe_tokens dtok = {};
@@ -263,6 +273,20 @@ trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
     if (c->n_sub > 3) { why = "config: n_sub > 3"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->n_centroids < 0 || c->n_centroids > 256) { why = "config: n_centroids must be in [0, 256]"; return TRIMMOE_ERR_UNSUPPORTED; }
     if ((long long)c->T_max * (c->k + 1) >= (1ll << 31)) { why = "config: T_max too large"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->attn_heads < 0) { why = "config: attn_heads must be >= 0"; return TRIMMOE_ERR_ARG; }
+    if (c->attn_heads > 0) {
+        if (c->attn_kv_heads < 1 || c->attn_heads % c->attn_kv_heads) {
+            why = "config: attn_heads must be a positive multiple of attn_kv_heads";
+            return TRIMMOE_ERR_ARG;
+        }
+        if (c->head_dim != 64 && c->head_dim != 128) { why = "config: head_dim must be 64 or 128"; return TRIMMOE_ERR_UNSUPPORTED; }
+        if (((long long)c->attn_heads + 2 * c->attn_kv_heads) * c->head_dim % 256) {
+            why = "config: (attn_heads + 2 attn_kv_heads) * head_dim must be a multiple of 256";
+            return TRIMMOE_ERR_UNSUPPORTED;
+        }
+        if (c->attn_seq < 1 || c->attn_seq > 128) { why = "config: attn_seq must be in [1, 128]"; return TRIMMOE_ERR_UNSUPPORTED; }
+        if (!(c->rope_theta > 1.f) || !std::isfinite(c->rope_theta)) { why = "config: rope_theta must be > 1"; return TRIMMOE_ERR_ARG; }
+    }
     return TRIMMOE_OK;
 }
 
@@ -290,6 +314,10 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         return create_fail(TRIMMOE_ERR_ARG, "create: NULL weight pointer");
     if (c.n_centroids > 0 && (!w->centroids || !tab->centroid_exit || !aligned16(w->centroids)))
         return create_fail(TRIMMOE_ERR_ARG, "create: n_centroids > 0 needs 16-byte aligned centroids and centroid_exit");
+    if (c.attn_heads > 0 && (!w->W_attn_norm || !w->W_qkv || !w->W_o || !w->W_norm))
+        return create_fail(TRIMMOE_ERR_ARG, "create: the attention sublayer needs W_attn_norm, W_qkv, W_o and W_norm");
+    if (c.attn_heads > 0 && (!aligned16(w->W_attn_norm) || !aligned16(w->W_qkv) || !aligned16(w->W_o)))
+        return create_fail(TRIMMOE_ERR_ARG, "create: weights must be 16-byte aligned");
     if ((c.F_sh > 0) != (w->W13_sh != nullptr && w->W2_sh != nullptr))
         return create_fail(TRIMMOE_ERR_ARG, "create: shared-expert weights must be given iff F_sh > 0");
     if (!aligned16(w->W_r) || !aligned16(w->W_x) || !aligned16(w->W13) || !aligned16(w->W2) ||
@@ -499,6 +527,13 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
     ok = ok && h->dalloc(&h->c_counts, h->n_counts);
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
+    const int has_attn = c.attn_heads > 0;
+    if (has_attn) {
+        h->nqkv = (c.attn_heads + 2 * c.attn_kv_heads) * c.head_dim;
+        ok = ok && h->dalloc(&h->qkv, T * h->nqkv) && h->dalloc(&h->attn_out, T * c.attn_heads * c.head_dim) &&
+             h->dalloc(&h->hm, T * d) && h->dalloc(&h->goff_attn, 2) &&
+             h->dalloc(&h->rope, (size_t)c.attn_seq * (c.head_dim / 2)) && h->dalloc(&h->sqbuf_x, h->rows_part);
+    }
     if (!ok) return bail(TRIMMOE_ERR_OOM, "create: device allocation failed");
     cudaError_t ce = cudaSuccess;
     auto up = [&](void* dst, const void* src, size_t bytes) {
@@ -521,6 +556,17 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     up(h->theta, tab->theta, N * 4);
     up(h->lambda, tab->lambda, N * 4);
     up(h->eps, tab->eps, N * 4);
+    if (has_attn) {
+        // Rotary table: angle pos * theta^(-2i/Dh), cos and sin in double, stored fp32.
+        const int half = c.head_dim / 2;
+        std::vector<float2> rt((size_t)c.attn_seq * half);
+        for (int pos = 0; pos < c.attn_seq; ++pos)
+            for (int i = 0; i < half; ++i) {
+                const double ang = (double)pos * std::pow((double)c.rope_theta, -2.0 * i / c.head_dim);
+                rt[(size_t)pos * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+            }
+        up(h->rope, rt.data(), rt.size() * sizeof(float2));
+    }
     if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters));
     if (ce == cudaSuccess) ce = cudaMemset(h->dev_err, 0, sizeof(int));
     if (ce == cudaSuccess) ce = cudaMemset(h->Xp, 0, (size_t)h->rows_xp * d * 2);
@@ -544,6 +590,17 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
             tm = make_tmap(&h->tmW13sh[l], W13s + (size_t)l * 2 * c.F_sh * d, d, (uint64_t)2 * c.F_sh, 256) &&
                  make_tmap(&h->tmW2sh[l], W2s + (size_t)l * d * c.F_sh, c.F_sh, (uint64_t)d, 256);
         }
+    }
+    if (tm && has_attn) {
+        const int hd = c.attn_heads * c.head_dim;
+        const __nv_bfloat16* Wqkv = static_cast<const __nv_bfloat16*>(w->W_qkv);
+        const __nv_bfloat16* Wo = static_cast<const __nv_bfloat16*>(w->W_o);
+        h->tmWqkv.resize(N);
+        h->tmWo.resize(N);
+        tm = make_tmap(&h->tmAttn, h->attn_out, hd, T, 128);
+        for (int l = 0; l < N && tm; ++l)
+            tm = make_tmap(&h->tmWqkv[l], Wqkv + (size_t)l * h->nqkv * d, d, (uint64_t)h->nqkv, 256) &&
+                 make_tmap(&h->tmWo[l], Wo + (size_t)l * d * hd, hd, (uint64_t)d, 256);
     }
     if (!tm) return bail(TRIMMOE_ERR_CUDA, "create: cuTensorMapEncodeTiled failed");
     *out = h;
@@ -578,11 +635,81 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.omega_T = c.omega_T;
     dp.omega_D = c.omega_D;
     dp.d_ref = c.d_ref_ms;
-    const __nv_bfloat16* hid = static_cast<const __nv_bfloat16*>(tok->hidden);
+    const __nv_bfloat16* hid_in = static_cast<const __nv_bfloat16*>(tok->hidden);
+    const __nv_bfloat16* hid = hid_in;     // input of the MoE sublayer
     const __nv_bfloat16* gamma =
         h->w.W_norm ? static_cast<const __nv_bfloat16*>(h->w.W_norm) + (size_t)layer * d : nullptr;
     const int Kc = c.n_centroids;
     const int n_out = E + c.C + Kc;
+    cudaError_t e = cudaSuccess;
+    const bool has_attn = c.attn_heads > 0;
+    if (has_attn) {
+        // Attention sublayer (Sec. III-C, attention placement): local, for every
+        // live token, in front of the MoE decision.
+        const int hd = c.attn_heads * c.head_dim;
+        AttnParams ap;
+        ap.T = T;
+        ap.d = d;
+        ap.S = c.attn_seq;
+        ap.Hq = c.attn_heads;
+        ap.Hkv = c.attn_kv_heads;
+        ap.nqkv = h->nqkv;
+        ap.norm_eps = c.norm_eps;
+        ap.scale = (float)(1.0 / std::sqrt((double)c.head_dim));
+        ap.h = hid_in;
+        ap.gamma = static_cast<const __nv_bfloat16*>(h->w.W_attn_norm) + (size_t)layer * d;
+        ap.a = h->Xp;
+        ap.goff = h->goff_attn;
+        ap.qkv = h->qkv;
+        ap.rope = h->rope;
+        ap.out = h->attn_out;
+        e = h->timed(K_ATTN, st, [&] { return launch_attn_norm(ap, h->num_sms, st); });
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention norm: ") + cudaGetErrorString(e));
+        GemmLaunch qg{};
+        qg.tmA = &h->tmXp;
+        qg.tmB = &h->tmWqkv[layer];
+        qg.goff = h->goff_attn;
+        qg.first_group = 0;
+        qg.ngroups = 1;
+        qg.K = d;
+        qg.n_tiles_n = h->nqkv / 256;
+        qg.b_rows_per_group = h->nqkv;
+        qg.epi_mode = EPI_STORE;
+        qg.out = h->qkv;
+        qg.ldo = h->nqkv;
+        qg.err = h->dev_err;
+        e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(qg, h->num_sms, st); });
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("qkv gemm: ") + cudaGetErrorString(e));
+        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, c.head_dim, st); });
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(e));
+        GemmLaunch og = qg;
+        og.tmA = &h->tmAttn;
+        og.tmB = &h->tmWo[layer];
+        og.K = hd;
+        og.n_tiles_n = d / 256;
+        og.b_rows_per_group = d;
+        og.epi_mode = EPI_RESID;
+        og.out = h->hm;
+        og.ldo = d;
+        og.res = hid_in;
+        og.ldr = d;
+        e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(og, h->num_sms, st); });
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("output projection: ") + cudaGetErrorString(e));
+        h->launches += 4;
+        h->flops_attn_gemm += 2.0 * T * d * (double)h->nqkv + 2.0 * T * (double)hd * d;
+        double pairs = 0.0;                      // causal (query, key) pairs
+        for (int t0 = 0; t0 < T; t0 += c.attn_seq) {
+            const double n = std::min(c.attn_seq, T - t0);
+            pairs += n * (n + 1) / 2;
+        }
+        h->flops_attn += 4.0 * c.head_dim * (double)c.attn_heads * pairs;
+        hid = h->hm;
+        if (out && out->h_attn) {
+            e = cudaMemcpyAsync(out->h_attn, h->hm, (size_t)T * d * 2, cudaMemcpyDeviceToDevice, st);
+            if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "copy h_attn failed");
+        }
+    }
+
     RouterParams rp;
     rp.T = T;
     rp.d = d;
@@ -598,10 +725,31 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     rp.Blo = h->rt_lo + (size_t)layer * E * d;
     rp.zpart = h->zbuf;
     rp.sqpart = h->sqbuf;
-    cudaError_t e = h->timed(K_ROUTER, st, [&] { return launch_router(rp, st); });
+    // With the attention sublayer the router rows read h_mid while the exit-head
+    // and centroid rows read the state entering the layer: two passes.
+    RouterParams rx = rp;
+    if (has_attn) {
+        rp.n_out = E;
+        rp.ng = router_pass_rows(E);
+        rp.nl = router_lo_rows(E, rp.ng);
+        rx.h = hid_in;
+        rx.n_out = n_out - E;
+        rx.n_lo = 0;
+        rx.ng = router_pass_rows(n_out - E);
+        rx.nl = 0;
+        rx.Bhi = rp.Bhi + (size_t)E * d;
+        rx.zpart = h->zbuf + E;
+        rx.sqpart = h->sqbuf_x;
+    }
+    e = h->timed(K_ROUTER, st, [&] {
+        cudaError_t e2 = launch_router(rp, st);
+        return (e2 == cudaSuccess && has_attn) ? launch_router(rx, st) : e2;
+    });
+    if (has_attn) h->launches += 1;
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("router: ") + cudaGetErrorString(e));
     dp.zpart = h->zbuf;
     dp.sqpart = h->sqbuf;
+    dp.sqpart_x = has_attn ? h->sqbuf_x : nullptr;
     dp.bias = h->rt_bias + (size_t)layer * n_out;
     dp.zs = n_out;
     dp.ksplit = rp.ksplit;
@@ -691,7 +839,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gather: ") + cudaGetErrorString(e));
 
-    GemmLaunch g1;
+    GemmLaunch g1{};
     g1.tmA = &h->tmXp;
     g1.tmB = &h->tmW13[layer];
     g1.goff = h->goff;
@@ -759,6 +907,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     bp.renorm = c.renorm_topk;
     bp.has_shared = has_sh;
     bp.h = static_cast<__nv_bfloat16*>(tok->hidden);  // combine writes h in place
+    bp.h_src = hid;                                    // residual base: h, or h_mid of the full block
     bp.action = dp.action;
     bp.topk_g = dp.topk_g;
     bp.pos_pair = h->pos_pair;
@@ -904,6 +1053,10 @@ extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) 
     out->ms_combine = h->ms[K_COMBINE];
     out->ms_router = h->ms[K_ROUTER];
     out->lookahead_shared = dc.lookahead_shared;
+    out->ms_attn = h->ms[K_ATTN];
+    out->ms_attn_gemm = h->ms[K_ATTN_GEMM];
+    out->flops_attn = h->flops_attn;
+    out->flops_attn_gemm = h->flops_attn_gemm;
     out->n_gemm_up = h->n_gemm_up;
     out->n_gemm_down = h->n_gemm_down;
     if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "stats: a kernel timed out waiting");
@@ -921,6 +1074,7 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
         return h->fail(TRIMMOE_ERR_CUDA, "reset: memset failed");
     for (double& m : h->ms) m = 0.0;
     h->launches = h->layer_calls = h->n_gemm_up = h->n_gemm_down = 0;
+    h->flops_attn = h->flops_attn_gemm = 0.0;
     h->win_delay0 = 0.0;
     h->win_ref_slots = 0.0;
     return TRIMMOE_OK;

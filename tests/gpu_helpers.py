@@ -64,14 +64,28 @@ def compare_layer(cfg, om, eng, l, dev_tok, experts, row_sample=None, check_perm
     eng.layer_step(l, dev_tok, out=out)
     torch.cuda.synchronize()
     after = B.Engine.tokens_to_host(dev_tok)
-    g = {k: v.cpu().numpy() for k, v in out.items()}
+    g = {k: (v.view(torch.int16).cpu().numpy().view(np.uint16) if v.dtype == torch.bfloat16 else v.cpu().numpy())
+         for k, v in out.items() if v is not None}
     h_in = before.pop("h")
     mask = None
     if row_sample is not None:
         mask = np.zeros(T, np.uint8)
         mask[np.asarray(row_sample)] = 1
-    h_or, tok_or, o = O.layer_step(om, l, h_in, before, experts_l=experts_layer_host(experts, l),
-                                   row_mask=mask)
+    ex_l = experts_layer_host(experts, l)
+    hm_gpu = None
+    attn_err = 0.0
+    if cfg.attn_heads:
+        # Attention sublayer: the GPU's h_mid against the oracle's on the live
+        # (sampled) rows; the MoE part of the oracle then reads the GPU's h_mid.
+        hm_gpu = g["h_attn"]
+        amask = (before["alive"] > 0) & (mask.astype(bool) if mask is not None else True)
+        hm_or = O.attention(om, l, h_in, before["alive"], experts_l=ex_l, row_mask=amask.astype(np.uint8))
+        if amask.any():
+            a = W.bf16_bits_to_f32(hm_gpu[amask]).astype(np.float64)
+            b = W.bf16_bits_to_f32(hm_or[amask]).astype(np.float64)
+            attn_err = float((np.abs(a - b).max(axis=1) / np.maximum(np.abs(b).max(axis=1), 1e-30)).max())
+            assert attn_err <= HIDDEN_TOL, f"layer {l}: attention rel err {attn_err}"
+    h_or, tok_or, o = O.layer_step(om, l, h_in, before, experts_l=ex_l, row_mask=mask, h_mid=hm_gpu)
 
     def rows_differ(a, b):
         return (np.asarray(a).reshape(T, -1) != np.asarray(b).reshape(T, -1)).any(axis=1)
@@ -128,9 +142,13 @@ def compare_layer(cfg, om, eng, l, dev_tok, experts, row_sample=None, check_perm
         den = np.maximum(np.abs(ho[run]).max(axis=1), 1e-30)
         err = float((num / den).max())
         assert err <= HIDDEN_TOL, f"layer {l}: hidden rel err {err}"
-    still = same & ((act == O.A_EXIT) | (act == O.A_DEAD) | ((act == O.A_SKIP) & (cfg.F_sh == 0)))
+    still = same & ((act == O.A_EXIT) | (act == O.A_DEAD))
     assert np.array_equal(after["h"][still], h_in[still]), "untouched rows changed"
+    bare_skip = same & (act == O.A_SKIP) & (cfg.F_sh == 0)
+    assert np.array_equal(after["h"][bare_skip], (hm_gpu if hm_gpu is not None else h_in)[bare_skip]), \
+        "skipped rows must carry the MoE input unchanged"
     counts = np.bincount(g["action"], minlength=4)
     return dict(layer=l, live=n_live, near_mismatch=n_mis, near=int(near.sum()), max_rel_err=err,
+                attn_rel_err=attn_err,
                 exec=int(counts[0]), skip=int(counts[1]), exit=int(counts[2]), dead=int(counts[3]),
                 rows_checked=int(run.sum()), oracle_out=o, s_before=before["s"])

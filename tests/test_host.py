@@ -107,6 +107,22 @@ def test_create_rejects_bad_arguments_on_host(lib):
     mis = B.trimmoe_weights.from_buffer_copy(w)
     mis.W13 = 0x1003                      # not 16-byte aligned
     assert _create(lib, c, mis, t)[0] == -1
+    # attention sublayer of the full block
+    bad = B.trimmoe_config.from_buffer_copy(c)
+    bad.attn_heads, bad.attn_kv_heads, bad.head_dim, bad.attn_seq, bad.rope_theta = 8, 3, 64, 128, 1e4
+    rc, _, msg = _create(lib, bad, w, t)
+    assert rc == -1 and "attn_kv_heads" in msg
+    bad.attn_kv_heads, bad.head_dim = 2, 96
+    rc, _, msg = _create(lib, bad, w, t)
+    assert rc == -2 and "head_dim" in msg
+    bad.head_dim, bad.attn_seq = 64, 129
+    rc, _, msg = _create(lib, bad, w, t)
+    assert rc == -2 and "attn_seq" in msg
+    bad.attn_seq, bad.attn_heads, bad.attn_kv_heads = 128, 5, 1         # (5 + 2) * 64 = 448
+    assert _create(lib, bad, w, t)[0] == -2
+    bad.attn_heads, bad.attn_kv_heads = 8, 2
+    rc, _, msg = _create(lib, bad, w, t)                                 # weights missing
+    assert rc == -1 and "W_qkv" in msg
     place = keep["place"].copy()
     place[2, 5] = 0
     t2 = B.trimmoe_tables.from_buffer_copy(t)
