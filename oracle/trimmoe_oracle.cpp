@@ -562,8 +562,8 @@ void or_rope(const double* x, int Dh, int pos, double theta, double* y) {
 // h_mid = h + attention(h) for the live tokens with row_mask set (every live
 // token when row_mask is NULL); all other rows of h_mid are copies of h.
 //   a = bf16(h * r * gamma)                        (r: RMS factor of h)
-//   q | k | v = bf16(a W_qkv^T)
-//   q, k <- bf16(rope(q, pos)), bf16(rope(k, pos))  per head, pos = t mod S
+//   q = bf16(rope(a W_q^T, pos)), k = bf16(rope(a W_k^T, pos)) per head,
+//   v = bf16(a W_v^T)                               pos = t mod S
 //   o_head = bf16( sum_j softmax_j(q . k_j / sqrt(Dh)) v_j )
 //            over the tokens j of t's sequence (t - pos .. t), query head
 //            hq reading key/value head hq / (Hq / Hkv)
@@ -596,16 +596,16 @@ int or_attention(const OrModel* md, const OrLayerWeights* lw, int T, const uint1
         const double r = or_rms_factor(hr, d, md->norm_eps);
         std::vector<uint16_t> a(d);
         for (int i = 0; i < d; ++i) a[i] = d2bf((double)bf2f(hr[i]) * r * (double)bf2f(lw->W_attn_norm[i]));
-        uint16_t* out = qkv.data() + (size_t)t * nqkv;
-        for (int o = 0; o < nqkv; ++o) out[o] = d2bf(dot_bf16(a.data(), lw->W_qkv + (size_t)o * d, d));
+        std::vector<double> z(nqkv);
+        for (int o = 0; o < nqkv; ++o) z[o] = dot_bf16(a.data(), lw->W_qkv + (size_t)o * d, d);
         const int pos = t % S;
-        std::vector<double> x(Dh), y(Dh);
+        std::vector<double> y(Dh);
         for (int hh = 0; hh < Hq + Hkv; ++hh) {          // query heads, then key heads
-            uint16_t* v = out + (size_t)hh * Dh;
-            for (int i = 0; i < Dh; ++i) x[i] = bf2f(v[i]);
-            or_rope(x.data(), Dh, pos, (double)md->rope_theta, y.data());
-            for (int i = 0; i < Dh; ++i) v[i] = d2bf(y[i]);
+            or_rope(z.data() + (size_t)hh * Dh, Dh, pos, (double)md->rope_theta, y.data());
+            std::copy(y.begin(), y.end(), z.begin() + (size_t)hh * Dh);
         }
+        uint16_t* out = qkv.data() + (size_t)t * nqkv;
+        for (int o = 0; o < nqkv; ++o) out[o] = d2bf(z[o]);
     }
     const double scale = 1.0 / std::sqrt((double)Dh);
 #ifdef _OPENMP

@@ -6,8 +6,9 @@
 // model families of Sec. VI-A:
 //
 //   a       = bf16(h * r * gamma_attn),  r = 1/sqrt(mean(h^2) + eps)   (attn_norm_kernel)
-//   q|k|v   = bf16(a W_qkv^T)                                         (grouped GEMM, one group)
-//   o       = softmax(rope(q) rope(k)^T / sqrt(Dh), causal) v          (attention_kernel)
+//   q, k    = bf16(rope(a W_q^T)), bf16(rope(a W_k^T)), v = bf16(a W_v^T)
+//                                  (grouped GEMM, one group, rotary epilogue)
+//   o       = softmax(q k^T / sqrt(Dh), causal) v                      (attention_kernel)
 //   h_mid   = bf16(h + o W_o^T)                                       (grouped GEMM, residual epilogue)
 //
 // Tokens are grouped into sequences of S consecutive tokens (one user's
@@ -16,10 +17,13 @@
 // keeps its state, which later tokens still read); outputs of tokens that are
 // not live are computed but never read.
 //
+// The rotary embedding (pairs i, i + Dh/2, angle pos * theta^(-2i/Dh) from a
+// host-made cos/sin table) is applied by the projection GEMM's epilogue to the
+// fp32 accumulators before their bf16 rounding.
+//
 // attention_kernel: one block per (query head, sequence), 4 warps.  Q, K and V
-// of the sequence (S <= 128 rows) are staged in padded shared memory with the
-// rotary embedding applied to Q and K on the way in (fp32 math from a host-made
-// cos/sin table, rounded to bf16).  Each warp owns two 16-row query blocks
+// of the sequence (S <= 128 rows) are staged in padded shared memory by
+// cp.async with every load in flight at once.  Each warp owns two 16-row query blocks
 // (mb and 7 - mb, which balances the causal work), computes the full causal
 // score rows with mma.sync m16n8k16 (bf16 in, fp32 accumulate), takes the
 // softmax in fp32 registers (quad shuffles), rounds the probabilities to bf16
@@ -91,8 +95,6 @@ __global__ void __launch_bounds__(256) attn_norm_kernel(const AttnParams p) {
 template <int DH>
 __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     constexpr int LD = DH + 8;                 // padded row (bf16): conflict-free ldmatrix
-    constexpr int HALF = DH / 2;
-    constexpr int HC = HALF / 8;               // 8-element chunks per half row
     constexpr int NTO = DH / 8;                // output n-tiles
     extern __shared__ __align__(16) uint8_t sm[];
     __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(sm);
@@ -109,37 +111,21 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
     const size_t koff = (size_t)(p.Hq + g) * DH;
     const size_t voff = (size_t)(p.Hq + p.Hkv + g) * DH;
 
-    // Stage Q and K with the rotary embedding (pairs i, i + Dh/2), and V.
-    for (int i = tid; i < 2 * n16 * HC; i += 128) {
-        const int which = i >= n16 * HC;       // 0: query head, 1: key head
-        const int rem = i - (which ? n16 * HC : 0);
-        const int r = rem / HC, c = (rem - r * HC) * 8;
-        __nv_bfloat16* dst = (which ? sK : sQ) + r * LD;
-        uint4 lo = make_uint4(0u, 0u, 0u, 0u), hi = lo;
-        if (r < n) {
-            const __nv_bfloat16* src = p.qkv + (size_t)(t0 + r) * p.nqkv + (which ? koff : qoff);
-            float x1[8], x2[8], y1[8], y2[8];
-            unpack8(*reinterpret_cast<const uint4*>(src + c), x1);
-            unpack8(*reinterpret_cast<const uint4*>(src + HALF + c), x2);
-            const float2* cs = p.rope + (size_t)r * HALF + c;
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const float2 w = __ldg(cs + u);
-                y1[u] = x1[u] * w.x - x2[u] * w.y;
-                y2[u] = x2[u] * w.x + x1[u] * w.y;
-            }
-            lo = pack8(y1);
-            hi = pack8(y2);
-        }
-        *reinterpret_cast<uint4*>(dst + c) = lo;
-        *reinterpret_cast<uint4*>(dst + HALF + c) = hi;
+    // Stage Q, K and V of the sequence (the projection's epilogue has already
+    // rotated Q and K) with every load in flight at once; rows >= n are zero.
+    constexpr int RC = DH / 8;                 // 16-byte chunks per row
+    for (int i = tid; i < 3 * n16 * RC; i += 128) {
+        const int which = i / (n16 * RC);      // 0: query head, 1: key head, 2: value head
+        const int rem = i - which * n16 * RC;
+        const int r = rem / RC, c = (rem - r * RC) * 8;
+        __nv_bfloat16* dst = (which == 0 ? sQ : which == 1 ? sK : sV) + r * LD + c;
+        const size_t off = which == 0 ? qoff : which == 1 ? koff : voff;
+        const bool ok = r < n;
+        const __nv_bfloat16* src = p.qkv + (size_t)(t0 + (ok ? r : 0)) * p.nqkv + off + c;
+        cp_async16(smem_u32(dst), src, ok ? 16 : 0);
     }
-    for (int i = tid; i < n16 * (DH / 8); i += 128) {
-        const int r = i / (DH / 8), c = (i - r * (DH / 8)) * 8;
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (r < n) v = *reinterpret_cast<const uint4*>(p.qkv + (size_t)(t0 + r) * p.nqkv + voff + c);
-        *reinterpret_cast<uint4*>(sV + r * LD + c) = v;
-    }
+    cp_async_commit();
+    cp_async_wait<0>();
     __syncthreads();
 
     const int gq = lane >> 2, tig = lane & 3;

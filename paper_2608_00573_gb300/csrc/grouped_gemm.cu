@@ -5,9 +5,10 @@
 // that group's weights B (bf16 [N][K], K contiguous):
 //     out[row, :] = epilogue(A[row, :] . B^T)
 // with epilogue = store (down projection), SwiGLU over the interleaved
-// gate/up columns (W13 of a SwiGLU expert), ReLU (W1 of a ReLU expert) or a
+// gate/up columns (W13 of a SwiGLU expert), ReLU (W1 of a ReLU expert), a
 // residual add (bf16 residual row + accumulator: the attention output
-// projection of the full block).
+// projection of the full block) or the rotary embedding of the query and key
+// heads (the q/k/v projection of the full block).
 // The expert FFN of the executed layers (Sec. III-B/C and the execute branch of
 // Algorithm 2) is the dense contraction of the MoE step; the full block also
 // runs its attention projections through this kernel as a single group.
@@ -98,7 +99,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
                     int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                     __nv_bfloat16* __restrict__ out, int ldo, int* err,
-                    const __nv_bfloat16* __restrict__ res, int ldr) {
+                    const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
+                    int rope_S, int rope_dh, int n_rot) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -246,6 +248,51 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                         store_row32(orow + ti.nt * (BN / 2) + c, v);
                     }
                 }
+            } else if (epi_mode == EPI_ROPE) {
+                // Rotary embedding of the query and key heads in the leading n_rot
+                // columns (pairs i, i + Dh/2 of each head; position = row mod S),
+                // the remaining (value) heads stored as they are.
+                const int pos = (ti.out_row + (valid ? row : 0)) % rope_S;
+                const int half = rope_dh >> 1;
+#pragma unroll 1
+                for (int h0 = 0; h0 < BN; h0 += rope_dh) {
+                    const int col0 = ti.nt * BN + h0;
+                    if (col0 < n_rot) {
+#pragma unroll 1
+                        for (int c = 0; c < half; c += 32) {
+                            uint32_t xa[32], xb[32];
+                            tmem_ld_32x32(tb + h0 + c, xa);
+                            tmem_ld_32x32(tb + h0 + half + c, xb);
+                            tmem_ld_wait();
+                            if (valid) {
+                                const float2* cs = rope + (size_t)pos * half + c;
+                                float ya[32], yb[32];
+#pragma unroll
+                                for (int i = 0; i < 32; ++i) {
+                                    const float2 w = __ldg(cs + i);
+                                    const float x1 = __uint_as_float(xa[i]), x2 = __uint_as_float(xb[i]);
+                                    ya[i] = x1 * w.x - x2 * w.y;
+                                    yb[i] = x2 * w.x + x1 * w.y;
+                                }
+                                store_row32(orow + col0 + c, ya);
+                                store_row32(orow + col0 + half + c, yb);
+                            }
+                        }
+                    } else {
+#pragma unroll 1
+                        for (int c = 0; c < rope_dh; c += 32) {
+                            uint32_t r[32];
+                            tmem_ld_32x32(tb + h0 + c, r);
+                            tmem_ld_wait();
+                            if (valid) {
+                                float v[32];
+#pragma unroll
+                                for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                                store_row32(orow + col0 + c, v);
+                            }
+                        }
+                    }
+                }
             } else {
 #pragma unroll 1
                 for (int c = 0; c < BN; c += 32) {
@@ -308,7 +355,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     if (g.ngroups <= 0 || g.ngroups > kMaxGroups || g.K % BK != 0) return cudaErrorInvalidValue;
     grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
         *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr);
+        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot);
     return cudaGetLastError();
 }
 

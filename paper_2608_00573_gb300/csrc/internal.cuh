@@ -150,9 +150,11 @@ struct GemmLaunch {
     int* err;
     const __nv_bfloat16* res;   // EPI_RESID: residual rows (same row index as out)
     int ldr;
+    const float2* rope;         // EPI_ROPE: (cos, sin) [rope_S][rope_dh/2]
+    int rope_S, rope_dh, n_rot; // sequence length, head dim, leading columns that rotate
 };
 
-enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2, EPI_RESID = 3 };
+enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2, EPI_RESID = 3, EPI_ROPE = 4 };
 
 // Attention sublayer of the full block (kernels e).
 struct AttnParams {
@@ -162,8 +164,7 @@ struct AttnParams {
     const __nv_bfloat16* gamma;   // [d] RMSNorm weights of the sublayer
     __nv_bfloat16* a;             // [T][d] normalised input of the q/k/v projection
     int* goff;                    // [2] {0, T}: the projections' single GEMM group
-    const __nv_bfloat16* qkv;     // [T][nqkv] query heads, key heads, value heads
-    const float2* rope;           // [S][Dh/2] (cos, sin) of the rotary embedding
+    const __nv_bfloat16* qkv;     // [T][nqkv] query heads, key heads (rotated), value heads
     __nv_bfloat16* out;           // [T][Hq*Dh] attention output
 };
 
@@ -374,7 +375,18 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// ldmatrix / mma.sync fragments (router and attention kernels).
+// cp.async (16 bytes, zero-filled past src_bytes), ldmatrix and mma.sync
+// fragments (router and attention kernels).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 __device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])

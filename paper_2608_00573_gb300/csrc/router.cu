@@ -33,16 +33,6 @@ constexpr int kPad = 72;          // padded smem row (bf16): conflict-free ldmat
 constexpr int kStages = 4;
 constexpr int kNG = 128;          // largest number of outputs per pass (16 n-tiles of 8)
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
 // NT: n-tiles of 8 outputs held in registers per pass (8 or 16).
 template <int NT>
 __global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {

@@ -661,7 +661,6 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         ap.a = h->Xp;
         ap.goff = h->goff_attn;
         ap.qkv = h->qkv;
-        ap.rope = h->rope;
         ap.out = h->attn_out;
         e = h->timed(K_ATTN, st, [&] { return launch_attn_norm(ap, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention norm: ") + cudaGetErrorString(e));
@@ -674,7 +673,11 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         qg.K = d;
         qg.n_tiles_n = h->nqkv / 256;
         qg.b_rows_per_group = h->nqkv;
-        qg.epi_mode = EPI_STORE;
+        qg.epi_mode = EPI_ROPE;
+        qg.rope = h->rope;
+        qg.rope_S = c.attn_seq;
+        qg.rope_dh = c.head_dim;
+        qg.n_rot = (c.attn_heads + c.attn_kv_heads) * c.head_dim;
         qg.out = h->qkv;
         qg.ldo = h->nqkv;
         qg.err = h->dev_err;
@@ -683,6 +686,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, c.head_dim, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(e));
         GemmLaunch og = qg;
+        og.rope = nullptr;
         og.tmA = &h->tmAttn;
         og.tmB = &h->tmWo[layer];
         og.K = hd;

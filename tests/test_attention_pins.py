@@ -155,7 +155,8 @@ def test_keys_of_tokens_that_left_still_count():
 
 def test_matches_torch_scaled_dot_product_attention():
     """The whole sublayer against torch: projections with matmul, the rotary
-    embedding as a complex rotation, causal attention by
+    embedding as a complex rotation of the projected query and key heads
+    (rounded to bf16 once, after the rotation), causal attention by
     scaled_dot_product_attention with the key/value heads repeated."""
     torch = pytest.importorskip("torch")
     cfg = _cfg(T=20)                     # a full sequence of 8 and a ragged 4
@@ -171,10 +172,10 @@ def test_matches_torch_scaled_dot_product_attention():
     def rnd(x):
         return torch.tensor(_bf(x.numpy()))
 
-    qkv = rnd(a @ Wqkv.T)
+    qkv = a @ Wqkv.T
     q = qkv[:, :Hq * Dh].reshape(-1, Hq, Dh)
     k = qkv[:, Hq * Dh:(Hq + Hkv) * Dh].reshape(-1, Hkv, Dh)
-    v = qkv[:, (Hq + Hkv) * Dh:].reshape(-1, Hkv, Dh)
+    v = rnd(qkv[:, (Hq + Hkv) * Dh:].reshape(-1, Hkv, Dh))
     pos = torch.arange(cfg.T, dtype=torch.float64) % S
     inv = cfg.rope_theta ** (-2.0 * torch.arange(Dh // 2, dtype=torch.float64) / Dh)
     rot = torch.polar(torch.ones(cfg.T, Dh // 2, dtype=torch.float64), pos[:, None] * inv[None, :])
