@@ -22,10 +22,14 @@
 //   warps 2-5   epilogue: tcgen05.ld 32 rows x 32 columns per warp, fused
 //               activation, bf16 stores
 // Operand tiles (A 128x64, B 256x64 per stage, 4 stages) arrive by TMA with
-// 128-byte swizzle.  Tiles are ordered expert-major, then output-column tile,
-// then row tile, so concurrent CTAs share one weight tile through L2.
+// 128-byte swizzle.  Tiles are ordered expert-major, then by blocks of row
+// tiles (about 48 MB of activations), then output-column tile, then row tile,
+// so concurrent CTAs share one weight tile through L2 and a block's
+// activations stay resident while the weights stream.
 // Every mbarrier wait is bounded (2 s); on expiry the kernel records an error
 // word, stops issuing work, frees its TMEM and returns.
+#include <algorithm>
+
 #include "internal.cuh"
 
 namespace tmoe {
@@ -59,8 +63,14 @@ struct Tile {
     int rows, a_row, out_row, b_row, nt;
 };
 
+// Tile t -> (group, row tile, column tile).  Within a group the row tiles are
+// taken in blocks of mblk (an activation block small enough to stay in L2);
+// inside a block the column tile is the slow index and the row tile the fast
+// one, so the CTAs running at the same time share one weight tile and the
+// block's activation rows are read from HBM once.
 __device__ __forceinline__ Tile map_tile(const GemmSmemTail* tl, int t, int ngroups, int n_tiles_n,
-                                         int base0, int a_rebase, int out_rebase, int b_rows_per_group) {
+                                         int base0, int a_rebase, int out_rebase, int b_rows_per_group,
+                                         int mblk) {
     int lo = 0, hi = ngroups - 1;
     while (lo < hi) {                      // largest g with tile_start[g] <= t
         const int mid = (lo + hi + 1) >> 1;
@@ -70,8 +80,20 @@ __device__ __forceinline__ Tile map_tile(const GemmSmemTail* tl, int t, int ngro
     const int cnt = tl->gcnt[g];
     const int mtc = (cnt + BM - 1) / BM;
     const int u = t - tl->tile_start[g];
-    const int nt = u / mtc;
-    const int mt = u - nt * mtc;
+    const int nfull = mtc / mblk;
+    const int full_tiles = nfull * mblk * n_tiles_n;
+    int nt, mt;
+    if (u < full_tiles) {
+        const int b = u / (mblk * n_tiles_n);
+        const int r = u - b * (mblk * n_tiles_n);
+        nt = r / mblk;
+        mt = b * mblk + (r - nt * mblk);
+    } else {
+        const int last = mtc - nfull * mblk;
+        const int r = u - full_tiles;
+        nt = r / last;
+        mt = nfull * mblk + (r - nt * last);
+    }
     Tile r;
     r.rows = min(BM, cnt - mt * BM);
     r.a_row = tl->gstart[g] - (a_rebase ? base0 : 0) + mt * BM;
@@ -100,7 +122,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                     __nv_bfloat16* __restrict__ out, int ldo, int* err,
                     const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
-                    int rope_S, int rope_dh, int n_rot) {
+                    int rope_S, int rope_dh, int n_rot, int mblk) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -161,7 +183,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             int it = 0;
             for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
                 const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
-                                         b_rows_per_group);
+                                         b_rows_per_group, mblk);
                 for (int kb = 0; kb < nkb; ++kb, ++it) {
                     const int s = it % STAGES;
                     const uint32_t ph = (it / STAGES) & 1;
@@ -218,7 +240,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         int tl_i = 0;
         for (int t = blockIdx.x; t < total; t += gridDim.x, ++tl_i) {
             const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
-                                     b_rows_per_group);
+                                     b_rows_per_group, mblk);
             const int buf = tl_i & 1;
             const uint32_t aph = (tl_i >> 1) & 1;
             int ok = 1;
@@ -353,9 +375,14 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
         attr_set = true;
     }
     if (g.ngroups <= 0 || g.ngroups > kMaxGroups || g.K % BK != 0) return cudaErrorInvalidValue;
+    // Row tiles per block: about 48 MB of activations (a third of L2), so that
+    // a block stays resident while the weight tiles stream past it.
+    const long long a_tile_bytes = (long long)BM * g.K * 2;
+    const int mblk = (int)std::max(1LL, (48LL << 20) / a_tile_bytes);
     grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
         *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot);
+        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot,
+        mblk);
     return cudaGetLastError();
 }
 
