@@ -61,7 +61,8 @@ enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
  *  omega_T, omega_D: weights of Eq. (21)/(31); d_ref_ms: d^ref of Eq. (31);
  *  phi_beta: Q = phi_beta * (1 - Sim)/2 (Eq. 3 with a linear phi);
  *  profile: 1 = record CUDA events around each kernel launch (trimmoe_stats
- *  then reports per-kernel device time);
+ *  then reports per-kernel device time); 2 = around the grouped GEMM launches
+ *  only (each event pair inside a replayed graph costs a few microseconds);
  *  norm_eps: epsilon of the pre-FFN RMSNorm (used when W_norm != NULL);
  *  n_centroids: K_c centroids per layer for the token-similarity exit-point
  *  prediction of Eq. (36) (0 = off, at most 256);
@@ -72,7 +73,15 @@ enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
  *  key/value heads of head_dim, rotary embedding with base rope_theta, within
  *  sequences of attn_seq consecutive tokens (token t sits at position
  *  t mod attn_seq).  Attention stays local to the token's server (Sec. III-C,
- *  attention placement): a skip bypasses only the MoE sublayer.
+ *  attention placement): a skip bypasses only the MoE sublayer;
+ *  graphs: 1 = trimmoe_forward / trimmoe_forward_host replay the whole
+ *  forward as a CUDA graph.  The first forward with a given (T, token
+ *  buffers, stream) runs as plain launches; the next one captures the layer
+ *  loop (twice, so profiling events of one replay can be read while the
+ *  other runs) and every later one launches the graph.  Results are those of
+ *  the plain launches.  Not used on the legacy or per-thread default stream,
+ *  or when the stream is already being captured (the launches then go into
+ *  the caller's capture); feedback and calibration calls drop the graph.
  * Supported: d % 256 == 0; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
  * F_sh % 128 == 0; E <= 128; k <= min(E, 8); C <= 256; M*E <= 1024; H <= 6;
  * n_sub <= 3; attention: head_dim 64 or 128, attn_heads % attn_kv_heads == 0,
@@ -90,6 +99,7 @@ typedef struct {
     int n_centroids;
     int attn_heads, attn_kv_heads, head_dim, attn_seq;
     float rope_theta;
+    int graphs;
 } trimmoe_config;
 
 /* Weights (device, bf16 except the biases, borrowed; 16-byte aligned).

@@ -36,7 +36,7 @@ class trimmoe_config(C.Structure):
                [(n, C.c_float) for n in ("omega_T", "omega_D", "d_ref_ms", "phi_beta")] + \
                [("profile", C.c_int), ("norm_eps", C.c_float), ("n_centroids", C.c_int)] + \
                [(n, C.c_int) for n in ("attn_heads", "attn_kv_heads", "head_dim", "attn_seq")] + \
-               [("rope_theta", C.c_float)]
+               [("rope_theta", C.c_float), ("graphs", C.c_int)]
 
 
 class trimmoe_weights(C.Structure):
@@ -255,7 +255,7 @@ class Engine:
     """Owns a trimmoe handle plus the torch tensors it borrows."""
 
     def __init__(self, cfg: W.WorkloadConfig, tables: dict, small: dict, experts: dict, T_max: int,
-                 device="cuda", profile: bool = False):
+                 device="cuda", profile=False, graphs: bool = False):
         import torch
         self.torch = torch
         self.cfg = cfg
@@ -287,9 +287,9 @@ class Engine:
             N=cfg.N, d=cfg.d, E=cfg.E, k=cfg.k, F=cfg.F, F_sh=cfg.F_sh, C=cfg.C, M=cfg.M, H=cfg.H,
             act=cfg.act, renorm_topk=cfg.renorm_topk, n_sub=cfg.n_sub, T_max=T_max,
             omega_T=cfg.omega_T, omega_D=cfg.omega_D, d_ref_ms=float(tables["d_ref"]),
-            phi_beta=cfg.phi_beta, profile=1 if profile else 0, norm_eps=cfg.norm_eps,
+            phi_beta=cfg.phi_beta, profile=int(profile), norm_eps=cfg.norm_eps,
             n_centroids=cfg.n_centroids, attn_heads=cfg.attn_heads, attn_kv_heads=cfg.attn_kv_heads,
-            head_dim=cfg.head_dim, attn_seq=cfg.attn_seq, rope_theta=cfg.rope_theta)
+            head_dim=cfg.head_dim, attn_seq=cfg.attn_seq, rope_theta=cfg.rope_theta, graphs=1 if graphs else 0)
         self.c_w = trimmoe_weights(**{k: _ptr(v) for k, v in self.w.items()})
         t = self.tables
         P = t["P"].astype(np.float32) if t["P"].size else None

@@ -88,6 +88,27 @@ void tmoe::set_global_error(const std::string& msg) {
     g_create_error = msg;
 }
 
+// A captured forward (all layers) replayed as one CUDA graph.  Two instances
+// alternate so that the profiling events of one replay can be read while the
+// next one runs.
+struct GraphInst {
+    cudaGraphExec_t exec = nullptr;
+    std::vector<std::pair<std::pair<cudaEvent_t, cudaEvent_t>, int>> evs;   // profile events inside the graph
+    bool pending = false;                                                   // replay not read yet
+};
+
+struct ForwardGraph {
+    int T = -1;
+    trimmoe_tokens tok = {};
+    cudaStream_t st = nullptr;
+    int eager_runs = 0;          // forwards run eagerly with this key (the first one is)
+    GraphInst inst[2];
+    int next = 0;
+    // host-side counters one replay adds
+    uint64_t launches = 0, layer_calls = 0, n_gemm_up = 0, n_gemm_down = 0;
+    double flops_attn = 0.0, flops_attn_gemm = 0.0;
+};
+
 struct trimmoe {
     trimmoe_config cfg;
     trimmoe_weights w;
@@ -170,6 +191,10 @@ struct trimmoe {
     // counters kept on the host
     uint64_t launches = 0, layer_calls = 0;
 
+    // CUDA graph of the forward (cfg.graphs), and the event list a capture fills
+    ForwardGraph fg;
+    std::vector<std::pair<std::pair<cudaEvent_t, cudaEvent_t>, int>>* cap_evs = nullptr;
+
     // profiling
     std::vector<cudaEvent_t> ev_free;
     std::vector<std::pair<std::pair<cudaEvent_t, cudaEvent_t>, int>> ev_pending;
@@ -209,20 +234,51 @@ struct trimmoe {
     template <class Fn>
     cudaError_t timed(int kind, cudaStream_t st, Fn fn) {
         cudaEvent_t a = nullptr, b = nullptr;
-        if (cfg.profile) {
+        // Inside a stream capture the events become event-record nodes of the
+        // graph (cudaEventRecordExternal), recorded at every replay.
+        const unsigned rec_flags = cap_evs ? cudaEventRecordExternal : 0u;
+        const bool rec = cfg.profile == 1 ||
+                         (cfg.profile == 2 && (kind == K_GEMM_UP || kind == K_GEMM_DOWN || kind == K_ATTN_GEMM));
+        if (rec) {
             a = get_event();
             b = get_event();
-            cudaEventRecord(a, st);
+            cudaEventRecordWithFlags(a, st, rec_flags);
         }
         cudaError_t e = fn();
-        if (cfg.profile) {
-            cudaEventRecord(b, st);
-            ev_pending.push_back({{a, b}, kind});
+        if (rec) {
+            cudaEventRecordWithFlags(b, st, rec_flags);
+            (cap_evs ? *cap_evs : ev_pending).push_back({{a, b}, kind});
         }
         return e;
     }
 
+    // Adds the kernel times of a finished graph replay (waits for it if needed).
+    void read_graph_inst(GraphInst& gi) {
+        if (!gi.pending) return;
+        if (!gi.evs.empty()) cudaEventSynchronize(gi.evs.back().first.second);
+        for (auto& pe : gi.evs) {
+            float t = 0.f;
+            if (cudaEventElapsedTime(&t, pe.first.first, pe.first.second) == cudaSuccess) ms[pe.second] += t;
+        }
+        gi.pending = false;
+    }
+
+    void drop_graph() {
+        for (GraphInst& gi : fg.inst) {
+            read_graph_inst(gi);
+            if (gi.exec) cudaGraphExecDestroy(gi.exec);
+            gi.exec = nullptr;
+            for (auto& pe : gi.evs) {
+                ev_free.push_back(pe.first.first);
+                ev_free.push_back(pe.first.second);
+            }
+            gi.evs.clear();
+        }
+        fg = ForwardGraph();
+    }
+
     void drain_events() {
+        for (GraphInst& gi : fg.inst) read_graph_inst(gi);
         for (auto& pe : ev_pending) {
             float t = 0.f;
             if (cudaEventElapsedTime(&t, pe.first.first, pe.first.second) == cudaSuccess) ms[pe.second] += t;
@@ -273,6 +329,8 @@ trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
     if (c->n_sub > 3) { why = "config: n_sub > 3"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->n_centroids < 0 || c->n_centroids > 256) { why = "config: n_centroids must be in [0, 256]"; return TRIMMOE_ERR_UNSUPPORTED; }
     if ((long long)c->T_max * (c->k + 1) >= (1ll << 31)) { why = "config: T_max too large"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->profile < 0 || c->profile > 2) { why = "config: profile must be 0, 1 or 2"; return TRIMMOE_ERR_ARG; }
+    if (c->graphs != 0 && c->graphs != 1) { why = "config: graphs must be 0 or 1"; return TRIMMOE_ERR_ARG; }
     if (c->attn_heads < 0) { why = "config: attn_heads must be >= 0"; return TRIMMOE_ERR_ARG; }
     if (c->attn_heads > 0) {
         if (c->attn_kv_heads < 1 || c->attn_heads % c->attn_kv_heads) {
@@ -617,6 +675,9 @@ static trimmoe_status check_tokens(trimmoe_handle h, const trimmoe_tokens* tok) 
 
 static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmoe_tokens* tok,
                                       trimmoe_layer_out* out, cudaStream_t st) {
+    // Launch errors are read with cudaGetLastError after each launch; clear a
+    // non-sticky error left behind by other code in this thread first.
+    cudaGetLastError();
     const trimmoe_config& c = h->cfg;
     const int E = c.E, K = c.k, d = c.d;
     const int has_sh = c.F_sh > 0;
@@ -949,6 +1010,98 @@ extern "C" trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T,
     return layer_step_impl(h, layer, T, tok, out, st);
 }
 
+static trimmoe_status forward_layers(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st) {
+    for (int l = 0; l < h->cfg.N; ++l) {
+        trimmoe_status s = layer_step_impl(h, l, T, tok, nullptr, st);
+        if (s != TRIMMOE_OK) return s;
+    }
+    return TRIMMOE_OK;
+}
+
+static bool same_tokens(const trimmoe_tokens& a, const trimmoe_tokens& b) {
+    return a.hidden == b.hidden && a.s == b.s && a.Dhat == b.Dhat && a.Dbar == b.Dbar && a.pJ == b.pJ &&
+           a.alive == b.alive && a.last_exec == b.last_exec && a.xi_last == b.xi_last && a.exit_layer == b.exit_layer;
+}
+
+// Captures the whole forward into gi (nothing runs); the host counters it
+// would add are kept per replay.
+static trimmoe_status capture_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st, GraphInst& gi) {
+    const uint64_t l0 = h->launches, c0 = h->layer_calls, u0 = h->n_gemm_up, d0 = h->n_gemm_down;
+    const double fa0 = h->flops_attn, fg0 = h->flops_attn_gemm;
+    h->cap_evs = &gi.evs;
+    cudaGraph_t graph = nullptr;
+    cudaError_t e = cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal);
+    trimmoe_status s = TRIMMOE_OK;
+    if (e == cudaSuccess) {
+        s = forward_layers(h, T, tok, st);
+        e = cudaStreamEndCapture(st, &graph);
+    }
+    h->cap_evs = nullptr;
+    ForwardGraph& fg = h->fg;
+    fg.launches = h->launches - l0;
+    fg.layer_calls = h->layer_calls - c0;
+    fg.n_gemm_up = h->n_gemm_up - u0;
+    fg.n_gemm_down = h->n_gemm_down - d0;
+    fg.flops_attn = h->flops_attn - fa0;
+    fg.flops_attn_gemm = h->flops_attn_gemm - fg0;
+    h->launches = l0;
+    h->layer_calls = c0;
+    h->n_gemm_up = u0;
+    h->n_gemm_down = d0;
+    h->flops_attn = fa0;
+    h->flops_attn_gemm = fg0;
+    if (e == cudaSuccess && s == TRIMMOE_OK) e = cudaGraphInstantiate(&gi.exec, graph, 0);
+    if (graph) cudaGraphDestroy(graph);
+    if (s != TRIMMOE_OK) return s;
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return h->fail(TRIMMOE_ERR_CUDA, std::string("forward: graph capture failed: ") + cudaGetErrorString(e));
+    }
+    return TRIMMOE_OK;
+}
+
+static trimmoe_status run_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const bool capturable = h->cfg.graphs && st != nullptr && st != cudaStreamLegacy && st != cudaStreamPerThread &&
+                            cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone;
+    if (!capturable) return forward_layers(h, T, tok, st);
+    ForwardGraph& fg = h->fg;
+    if (fg.T != T || fg.st != st || !same_tokens(fg.tok, *tok)) {
+        h->drop_graph();
+        fg.T = T;
+        fg.st = st;
+        fg.tok = *tok;
+    }
+    if (fg.eager_runs < 1) {            // the first forward of a key runs eagerly (lazy set-up happens there)
+        fg.eager_runs++;
+        return forward_layers(h, T, tok, st);
+    }
+    if (!fg.inst[0].exec) {
+        for (GraphInst& gi : fg.inst) {
+            trimmoe_status s = capture_forward(h, T, tok, st, gi);
+            if (s != TRIMMOE_OK) {
+                h->drop_graph();
+                return s;
+            }
+        }
+    }
+    GraphInst& gi = fg.inst[fg.next];
+    h->read_graph_inst(gi);
+    if (cudaGraphLaunch(gi.exec, st) != cudaSuccess) {
+        cudaGetLastError();
+        return h->fail(TRIMMOE_ERR_CUDA, "forward: graph launch failed");
+    }
+    gi.pending = h->cfg.profile != 0;
+    fg.next ^= 1;
+    h->launches += fg.launches;
+    h->layer_calls += fg.layer_calls;
+    h->n_gemm_up += fg.n_gemm_up;
+    h->n_gemm_down += fg.n_gemm_down;
+    h->flops_attn += fg.flops_attn;
+    h->flops_attn_gemm += fg.flops_attn_gemm;
+    return TRIMMOE_OK;
+}
+
 extern "C" trimmoe_status trimmoe_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream) {
     if (!h) return TRIMMOE_ERR_ARG;
     if (T < 0 || T > h->cfg.T_max) return h->fail(TRIMMOE_ERR_ARG, "forward: T outside [0, T_max]");
@@ -958,11 +1111,7 @@ extern "C" trimmoe_status trimmoe_forward(trimmoe_handle h, int T, trimmoe_token
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     h->last_stream = st;
     if (T == 0) return TRIMMOE_OK;
-    for (int l = 0; l < h->cfg.N; ++l) {
-        s = layer_step_impl(h, l, T, tok, nullptr, st);
-        if (s != TRIMMOE_OK) return s;
-    }
-    return TRIMMOE_OK;
+    return run_forward(h, T, tok, st);
 }
 
 extern "C" trimmoe_status trimmoe_forward_host(trimmoe_handle h, int T, trimmoe_tokens* tok, void* stream) {
@@ -996,8 +1145,8 @@ extern "C" trimmoe_status trimmoe_forward_host(trimmoe_handle h, int T, trimmoe_
     for (const Cp& c : in)
         if (cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
             return h->fail(TRIMMOE_ERR_CUDA, "forward_host: host-to-device copy failed");
-    for (int l = 0; l < h->cfg.N && T > 0; ++l) {
-        trimmoe_status s = layer_step_impl(h, l, T, &dt, nullptr, st);
+    if (T > 0) {
+        trimmoe_status s = run_forward(h, T, &dt, st);
         if (s != TRIMMOE_OK) return s;
     }
     for (const Cp& c : in)
@@ -1092,6 +1241,7 @@ extern "C" trimmoe_status trimmoe_calibration_begin(trimmoe_handle h) {
         cudaMemset(h->prev_target, 0xFF, (size_t)h->cfg.T_max * sizeof(int16_t)) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "calibration_begin: reset failed");
+    h->drop_graph();      // the decision kernel's parameters change
     h->calib = 1;
     return TRIMMOE_OK;
 }
@@ -1105,6 +1255,7 @@ extern "C" trimmoe_status trimmoe_calibration_end(trimmoe_handle h, long long T_
         cudaMemcpy(cnt.data(), h->c_counts, cnt.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) !=
             cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "calibration_end: copy failed");
+    h->drop_graph();
     h->calib = 0;
     const int N = h->cfg.N, E = h->cfg.E, M = h->cfg.M, K = h->cfg.k;
     const size_t ntr = (size_t)std::max(N - 1, 1) * E * E;
@@ -1245,6 +1396,7 @@ extern "C" trimmoe_status trimmoe_feedback(trimmoe_handle h, const trimmoe_feedb
     h->cfg = c2;
     h->win_delay0 = dc.delay_ms;
     h->win_ref_slots = 0.0;
+    h->drop_graph();      // omega enters the decision kernel by value
     out->omega_T = c2.omega_T;
     out->omega_D = c2.omega_D;
     out->T_norm = T_norm;
@@ -1268,6 +1420,7 @@ extern "C" void trimmoe_destroy(trimmoe_handle h) {
     DeviceGuard g(h->dev);
     cudaDeviceSynchronize();
     h->drain_events();
+    h->drop_graph();
     for (cudaEvent_t e : h->ev_free) cudaEventDestroy(e);
     for (void* p : h->allocs) cudaFree(p);
     delete h;
