@@ -32,47 +32,86 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
             nj = p.k;
             float gs = 0.f;
             for (int j = 0; j < nj; ++j) gs = __fadd_rn(gs, p.topk_g[t * p.k + j]);
-            for (int j = 0; j < nj; ++j) {
-                const float gj = p.topk_g[t * p.k + j];
-                w[j] = p.renorm ? __fdiv_rn(gj, gs) : gj;
-                pos[j] = p.pos_pair[t * p.k + j];
+#pragma unroll
+            for (int j = 0; j < kMaxK; ++j) {
+                if (j < nj) {
+                    const float gj = p.topk_g[t * p.k + j];
+                    w[j] = p.renorm ? __fdiv_rn(gj, gs) : gj;
+                    pos[j] = p.pos_pair[t * p.k + j];
+                }
             }
         }
         const int psh = p.has_shared ? p.pos_sh[t] : -1;
         uint4* hrow = reinterpret_cast<uint4*>(p.h + (size_t)t * p.d);
         const uint4* brow = reinterpret_cast<const uint4*>(p.h_src + (size_t)t * p.d);
-        for (int c = lane; c < nchunk; c += 32) {
-            const uint4 hv = brow[c];
-            float acc[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
-                            bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
-            for (int j = 0; j < nj; ++j) {
-                const uint4 y = __ldg(reinterpret_cast<const uint4*>(p.Y + (size_t)pos[j] * p.d) + c);
-                acc[0] = fmaf(w[j], bf16_lo(y.x), acc[0]);
-                acc[1] = fmaf(w[j], bf16_hi(y.x), acc[1]);
-                acc[2] = fmaf(w[j], bf16_lo(y.y), acc[2]);
-                acc[3] = fmaf(w[j], bf16_hi(y.y), acc[3]);
-                acc[4] = fmaf(w[j], bf16_lo(y.z), acc[4]);
-                acc[5] = fmaf(w[j], bf16_hi(y.z), acc[5]);
-                acc[6] = fmaf(w[j], bf16_lo(y.w), acc[6]);
-                acc[7] = fmaf(w[j], bf16_hi(y.w), acc[7]);
+        // kU chunks of 16 bytes per lane at a time: every load of a step is in
+        // flight before the first one is used.
+        constexpr int kU = 4;
+        for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
+            float acc[kU][8];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + 32 * u;
+                const uint4 hv = c < nchunk ? brow[c] : make_uint4(0u, 0u, 0u, 0u);
+                acc[u][0] = bf16_lo(hv.x); acc[u][1] = bf16_hi(hv.x);
+                acc[u][2] = bf16_lo(hv.y); acc[u][3] = bf16_hi(hv.y);
+                acc[u][4] = bf16_lo(hv.z); acc[u][5] = bf16_hi(hv.z);
+                acc[u][6] = bf16_lo(hv.w); acc[u][7] = bf16_hi(hv.w);
+            }
+#pragma unroll
+            for (int j = 0; j < kMaxK; ++j) {
+                if (j >= nj) break;
+                const uint4* yrow = reinterpret_cast<const uint4*>(p.Y + (size_t)pos[j] * p.d);
+                uint4 y[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int c = c0 + 32 * u;
+                    y[u] = c < nchunk ? __ldg(yrow + c) : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    acc[u][0] = fmaf(w[j], bf16_lo(y[u].x), acc[u][0]);
+                    acc[u][1] = fmaf(w[j], bf16_hi(y[u].x), acc[u][1]);
+                    acc[u][2] = fmaf(w[j], bf16_lo(y[u].y), acc[u][2]);
+                    acc[u][3] = fmaf(w[j], bf16_hi(y[u].y), acc[u][3]);
+                    acc[u][4] = fmaf(w[j], bf16_lo(y[u].z), acc[u][4]);
+                    acc[u][5] = fmaf(w[j], bf16_hi(y[u].z), acc[u][5]);
+                    acc[u][6] = fmaf(w[j], bf16_lo(y[u].w), acc[u][6]);
+                    acc[u][7] = fmaf(w[j], bf16_hi(y[u].w), acc[u][7]);
+                }
             }
             if (psh >= 0) {
-                const uint4 y = __ldg(reinterpret_cast<const uint4*>(p.Ysh + (size_t)psh * p.d) + c);
-                acc[0] += bf16_lo(y.x);
-                acc[1] += bf16_hi(y.x);
-                acc[2] += bf16_lo(y.y);
-                acc[3] += bf16_hi(y.y);
-                acc[4] += bf16_lo(y.z);
-                acc[5] += bf16_hi(y.z);
-                acc[6] += bf16_lo(y.w);
-                acc[7] += bf16_hi(y.w);
+                const uint4* yrow = reinterpret_cast<const uint4*>(p.Ysh + (size_t)psh * p.d);
+                uint4 y[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int c = c0 + 32 * u;
+                    y[u] = c < nchunk ? __ldg(yrow + c) : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    acc[u][0] += bf16_lo(y[u].x);
+                    acc[u][1] += bf16_hi(y[u].x);
+                    acc[u][2] += bf16_lo(y[u].y);
+                    acc[u][3] += bf16_hi(y[u].y);
+                    acc[u][4] += bf16_lo(y[u].z);
+                    acc[u][5] += bf16_hi(y[u].z);
+                    acc[u][6] += bf16_lo(y[u].w);
+                    acc[u][7] += bf16_hi(y[u].w);
+                }
             }
-            uint4 o;
-            o.x = pack_bf16x2(acc[0], acc[1]);
-            o.y = pack_bf16x2(acc[2], acc[3]);
-            o.z = pack_bf16x2(acc[4], acc[5]);
-            o.w = pack_bf16x2(acc[6], acc[7]);
-            hrow[c] = o;
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + 32 * u;
+                if (c < nchunk) {
+                    uint4 o;
+                    o.x = pack_bf16x2(acc[u][0], acc[u][1]);
+                    o.y = pack_bf16x2(acc[u][2], acc[u][3]);
+                    o.z = pack_bf16x2(acc[u][4], acc[u][5]);
+                    o.w = pack_bf16x2(acc[u][6], acc[u][7]);
+                    hrow[c] = o;
+                }
+            }
         }
     }
 }

@@ -140,23 +140,46 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
          r += (gridDim.x * blockDim.x) >> 5) {
         const int code = perm[r];
         const int t = r < routed ? code / k : code;
-        const uint4* src = reinterpret_cast<const uint4*>(h + (size_t)t * d);
-        uint4* dst = reinterpret_cast<uint4*>(Xp + (size_t)r * d);
+        const uint4* __restrict__ src = reinterpret_cast<const uint4*>(h + (size_t)t * d);
+        uint4* __restrict__ dst = reinterpret_cast<uint4*>(Xp + (size_t)r * d);
+        // kU chunks of 16 bytes per lane in flight at a time.
+        constexpr int kU = 4;
         if (!gamma) {
-            for (int c = lane; c < nchunk; c += 32) dst[c] = src[c];
+            for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
+                uint4 v[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u)
+                    if (c0 + 32 * u < nchunk) v[u] = src[c0 + 32 * u];
+#pragma unroll
+                for (int u = 0; u < kU; ++u)
+                    if (c0 + 32 * u < nchunk) dst[c0 + 32 * u] = v[u];
+            }
             continue;
         }
         const float rn = rnorm[t];
         const uint4* gv4 = reinterpret_cast<const uint4*>(gamma);
-        for (int c = lane; c < nchunk; c += 32) {
-            const uint4 hv = src[c];
-            const uint4 gv = __ldg(gv4 + c);
-            uint4 o;
-            o.x = pack_bf16x2(bf16_lo(hv.x) * rn * bf16_lo(gv.x), bf16_hi(hv.x) * rn * bf16_hi(gv.x));
-            o.y = pack_bf16x2(bf16_lo(hv.y) * rn * bf16_lo(gv.y), bf16_hi(hv.y) * rn * bf16_hi(gv.y));
-            o.z = pack_bf16x2(bf16_lo(hv.z) * rn * bf16_lo(gv.z), bf16_hi(hv.z) * rn * bf16_hi(gv.z));
-            o.w = pack_bf16x2(bf16_lo(hv.w) * rn * bf16_lo(gv.w), bf16_hi(hv.w) * rn * bf16_hi(gv.w));
-            dst[c] = o;
+        for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
+            uint4 hv[kU], gv[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + 32 * u;
+                if (c < nchunk) {
+                    hv[u] = src[c];
+                    gv[u] = __ldg(gv4 + c);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + 32 * u;
+                if (c < nchunk) {
+                    uint4 o;
+                    o.x = pack_bf16x2(bf16_lo(hv[u].x) * rn * bf16_lo(gv[u].x), bf16_hi(hv[u].x) * rn * bf16_hi(gv[u].x));
+                    o.y = pack_bf16x2(bf16_lo(hv[u].y) * rn * bf16_lo(gv[u].y), bf16_hi(hv[u].y) * rn * bf16_hi(gv[u].y));
+                    o.z = pack_bf16x2(bf16_lo(hv[u].z) * rn * bf16_lo(gv[u].z), bf16_hi(hv[u].z) * rn * bf16_hi(gv[u].z));
+                    o.w = pack_bf16x2(bf16_lo(hv[u].w) * rn * bf16_lo(gv[u].w), bf16_hi(hv[u].w) * rn * bf16_hi(gv[u].w));
+                    dst[c] = o;
+                }
+            }
         }
     }
 }

@@ -98,3 +98,37 @@ def test_graph_dropped_when_tokens_move():
     plain.close()
     graph.close()
     torch.cuda.synchronize()
+
+
+def test_graph_follows_feedback_updates():
+    """Runtime feedback changes omega (a kernel parameter): the replayed graph
+    is dropped and rebuilt, so forwards after the update equal those of plain
+    launches with the same window sequence."""
+    import torch
+    cfg = CASES["moe_shared_kc8"]
+    plain, om, tables, small, experts = make_engine(cfg, theta=0.9, exit_bias=1.0)
+    graph = B.Engine(cfg, tables, small, experts, T_max=cfg.T, graphs=True)
+    stream = torch.cuda.Stream()
+    tok = W.make_tokens(cfg)
+    with torch.cuda.stream(stream):
+        pristine = plain.tokens_to_device(tok)
+        buf_p = {k: v.clone() for k, v in pristine.items()}
+        buf_g = {k: v.clone() for k, v in pristine.items()}
+        for window in range(3):
+            for rep in range(3):
+                for k in pristine:
+                    if k != "pJ":                       # p_J carries the feedback across windows
+                        buf_p[k].copy_(pristine[k])
+                        buf_g[k].copy_(pristine[k])
+                plain.forward(buf_p, stream=stream)
+                graph.forward(buf_g, stream=stream)
+            op = plain.feedback(buf_p, user_size=128, eta=0.25, p_min=0.7, kappa=0.5, stream=stream)
+            og = graph.feedback(buf_g, user_size=128, eta=0.25, p_min=0.7, kappa=0.5, stream=stream)
+            assert op["omega_D"] == og["omega_D"] and op["omega_T"] == og["omega_T"], window
+            stream.synchronize()
+            a, b = B.Engine.tokens_to_host(buf_p), B.Engine.tokens_to_host(buf_g)
+            for k in a:
+                assert np.array_equal(a[k], b[k]), (window, k)
+    plain.close()
+    graph.close()
+    torch.cuda.synchronize()
