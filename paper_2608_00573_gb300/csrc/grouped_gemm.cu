@@ -122,7 +122,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                     __nv_bfloat16* __restrict__ out, int ldo, int* err,
                     const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
-                    int rope_S, int rope_dh, int n_rot, int mblk) {
+                    int rope_S, int rope_dh, int n_rot, int mblk, int ksplit, float* __restrict__ partial,
+                    int ldp, size_t pstride) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -152,10 +153,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         (void)base0;
     }
     __syncthreads();
-    const int total = tl->total_tiles;
+    const int ntiles = tl->total_tiles;
+    const int total = ntiles * ksplit;    // unit u: tile u % ntiles, K range u / ntiles
     if ((int)blockIdx.x >= total) return;
     const int base0 = tl->gstart[0];
     const int nkb = K / BK;
+    const int kbr = nkb / ksplit;         // k blocks per range
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -182,9 +185,10 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             // ---------------------------------------------------- producer
             int it = 0;
             for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
-                const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
+                const Tile ti = map_tile(tl, t % ntiles, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
                                          b_rows_per_group, mblk);
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                const int kb0 = (t / ntiles) * kbr;
+                for (int kb = kb0; kb < kb0 + kbr; ++kb, ++it) {
                     const int s = it % STAGES;
                     const uint32_t ph = (it / STAGES) & 1;
                     if (!mbar_wait_bounded(smem_u32(&tl->empty[s]), ph ^ 1, abort_flag, err,
@@ -213,7 +217,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                const int kb0 = (t / ntiles) * kbr;
+                for (int kb = kb0; kb < kb0 + kbr; ++kb, ++it) {
                     const int s = it % STAGES;
                     const uint32_t ph = (it / STAGES) & 1;
                     if (!mbar_wait_bounded(smem_u32(&tl->full[s]), ph, abort_flag, err, ERR_TIMEOUT_MMA)) {
@@ -226,7 +231,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk)
                         tc_mma_bf16(d_tmem, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + kk * 32),
-                                    idesc, (kb | kk) != 0 ? 1u : 0u);
+                                    idesc, (kb != kb0 || kk != 0) ? 1u : 0u);
                     tc_commit(smem_u32(&tl->empty[s]));
                 }
                 if (!ok) break;
@@ -239,7 +244,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         const int row = q * 32 + lane;
         int tl_i = 0;
         for (int t = blockIdx.x; t < total; t += gridDim.x, ++tl_i) {
-            const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
+            const Tile ti = map_tile(tl, t % ntiles, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
                                      b_rows_per_group, mblk);
             const int buf = tl_i & 1;
             const uint32_t aph = (tl_i >> 1) & 1;
@@ -252,7 +257,24 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
             const bool valid = row < ti.rows;
             __nv_bfloat16* orow = out + (size_t)(ti.out_row + (valid ? row : 0)) * ldo;
-            if (epi_mode == EPI_SWIGLU) {
+            if (ksplit > 1) {
+                // fp32 partial sums of this K range; the finish kernel adds the ranges.
+                float* prow = partial + (size_t)(t / ntiles) * pstride +
+                              (size_t)(ti.out_row + (valid ? row : 0)) * ldp + ti.nt * BN;
+#pragma unroll 1
+                for (int c = 0; c < BN; c += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32(tb + c, r);
+                    tmem_ld_wait();
+                    if (valid) {
+                        float4* d4 = reinterpret_cast<float4*>(prow + c);
+#pragma unroll
+                        for (int q4 = 0; q4 < 8; ++q4)
+                            d4[q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
+                                                 __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
+                    }
+                }
+            } else if (epi_mode == EPI_SWIGLU) {
 #pragma unroll 1
                 for (int c = 0; c < BN / 2; c += 32) {
                     uint32_t gr[32], ur[32];
@@ -382,7 +404,67 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
         *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
         g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot,
-        mblk);
+        mblk, g.ksplit > 1 ? g.ksplit : 1, g.partial, g.ldp, g.pstride);
+    return cudaGetLastError();
+}
+
+// K split for launches with few tiles (small batches): the power of two up to
+// 8 that fills the persistent CTAs' rounds best (ties to the smaller split),
+// keeping at least 8 k-blocks per range.
+int grouped_gemm_ksplit(int est_tiles, int nkb, int num_sms) {
+    if (est_tiles <= 0) return 1;
+    int best = 1;
+    double best_eff = 0.0;
+    for (int ks = 1; ks <= 8; ks *= 2) {
+        if (nkb % ks || nkb / ks < 8) break;
+        const long long units = (long long)est_tiles * ks;
+        const long long rounds = (units + num_sms - 1) / num_sms;
+        const double eff = (double)units / (double)(rounds * num_sms);
+        if (eff > best_eff + 1e-9) { best_eff = eff; best = ks; }
+    }
+    return best;
+}
+
+namespace {
+
+// out[row][col] = epilogue(sum over the K ranges, in order, of partial[ks][row][col]).
+__global__ void __launch_bounds__(256) splitk_finish_kernel(const int* __restrict__ goff, int first_group,
+                                                            int ngroups, int out_rebase, int ksplit,
+                                                            const float* __restrict__ partial, int ldp,
+                                                            size_t pstride, int epi_mode,
+                                                            __nv_bfloat16* __restrict__ out, int ldo) {
+    const int r0 = out_rebase ? 0 : goff[first_group];
+    const int r1 = goff[first_group + ngroups] - (out_rebase ? goff[first_group] : 0);
+    const int ncol = epi_mode == EPI_SWIGLU ? ldp / 2 : ldp;
+    const long long n = (long long)(r1 - r0) * ncol;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int r = r0 + (int)(i / ncol);
+        const int c = (int)(i % ncol);
+        if (epi_mode == EPI_SWIGLU) {
+            const int gcol = (c / (BN / 2)) * BN + (c % (BN / 2));
+            float gt = 0.f, up = 0.f;
+            for (int ks = 0; ks < ksplit; ++ks) {
+                const float* pr = partial + (size_t)ks * pstride + (size_t)r * ldp;
+                gt += pr[gcol];
+                up += pr[gcol + BN / 2];
+            }
+            out[(size_t)r * ldo + c] = __float2bfloat16_rn(gt / (1.f + __expf(-gt)) * up);
+        } else {
+            float v = 0.f;
+            for (int ks = 0; ks < ksplit; ++ks) v += partial[(size_t)ks * pstride + (size_t)r * ldp + c];
+            if (epi_mode == EPI_RELU) v = fmaxf(v, 0.f);
+            out[(size_t)r * ldo + c] = __float2bfloat16_rn(v);
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_splitk_finish(const GemmLaunch& g, int num_sms, cudaStream_t st) {
+    if (g.epi_mode != EPI_STORE && g.epi_mode != EPI_SWIGLU && g.epi_mode != EPI_RELU) return cudaErrorInvalidValue;
+    splitk_finish_kernel<<<num_sms * 2, 256, 0, st>>>(g.goff, g.first_group, g.ngroups, g.out_rebase, g.ksplit,
+                                                       g.partial, g.ldp, g.pstride, g.epi_mode, g.out, g.ldo);
     return cudaGetLastError();
 }
 

@@ -152,6 +152,13 @@ struct GemmLaunch {
     int ldr;
     const float2* rope;         // EPI_ROPE: (cos, sin) [rope_S][rope_dh/2]
     int rope_S, rope_dh, n_rot; // sequence length, head dim, leading columns that rotate
+    // Split over K (ksplit > 1): each (tile, range) writes its fp32 partial
+    // sums to partial[ks][row][col] (ldp columns, pstride floats per range) and
+    // splitk_finish adds the ranges in order and applies the epilogue.
+    int ksplit;
+    float* partial;
+    int ldp;
+    size_t pstride;
 };
 
 enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2, EPI_RESID = 3, EPI_ROPE = 4 };
@@ -208,6 +215,8 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
                           const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,
                           __nv_bfloat16* Xp, int max_rows, int num_sms, cudaStream_t st);
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st);
+cudaError_t launch_splitk_finish(const GemmLaunch& g, int num_sms, cudaStream_t st);
+int grouped_gemm_ksplit(int est_tiles, int nkb, int num_sms);
 size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
 cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);

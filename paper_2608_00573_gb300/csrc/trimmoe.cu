@@ -54,6 +54,9 @@ bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Small batches: routed GEMMs with at most kSplitKRows executed pairs may split K.
+constexpr int kSplitKMax = 8, kSplitKRows = 64;
+
 enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
 
 inline float bf16_to_float(uint16_t b) {
@@ -157,6 +160,7 @@ struct trimmoe {
     __nv_bfloat16 *Xp = nullptr, *act = nullptr, *act_sh = nullptr, *Y = nullptr, *Ysh = nullptr;
     DevCounters* ctr = nullptr;
     int* dev_err = nullptr;
+    float* splitk = nullptr;          // [8][64][max(n13 F, d)] partial sums of split-K GEMMs
     int rows_xp = 0;
 
     CUtensorMap tmXp, tmAct, tmActSh;
@@ -583,7 +587,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->prev_target, T) && h->dalloc(&h->phi_tabs, std::max<size_t>(tab_floats, 1)) &&
               h->dalloc(&h->thr, std::max<size_t>(h->h_thr.size(), 1)) && h->dalloc(&h->dbar_shared, 1);
     h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
-    ok = ok && h->dalloc(&h->c_counts, h->n_counts);
+    ok = ok && h->dalloc(&h->c_counts, h->n_counts) &&
+         h->dalloc(&h->splitk, (size_t)kSplitKMax * kSplitKRows * std::max<size_t>((size_t)h->n13 * c.F, (size_t)d));
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
     const int has_attn = c.attn_heads > 0;
     if (has_attn) {
@@ -919,7 +924,20 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     g1.out = h->act;
     g1.ldo = c.F;
     g1.err = h->dev_err;
-    e = h->timed(K_GEMM_UP, st, [&] { return launch_grouped_gemm(g1, h->num_sms, st); });
+    // Few executed pairs (decode-sized batches): few tiles would leave most
+    // CTAs idle, so the K range is split and a finish kernel adds the parts.
+    const bool small = (long long)T * K <= kSplitKRows;
+    const int est_groups = (int)std::min<long long>(E, (long long)T * K);
+    if (small) {
+        g1.ksplit = grouped_gemm_ksplit(est_groups * g1.n_tiles_n, d / 64, h->num_sms);
+        g1.partial = h->splitk;
+        g1.ldp = g1.n_tiles_n * 256;
+        g1.pstride = (size_t)kSplitKRows * g1.ldp;
+    }
+    e = h->timed(K_GEMM_UP, st, [&] {
+        cudaError_t e2 = launch_grouped_gemm(g1, h->num_sms, st);
+        return (e2 == cudaSuccess && g1.ksplit > 1) ? launch_splitk_finish(g1, h->num_sms, st) : e2;
+    });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm up: ") + cudaGetErrorString(e));
     GemmLaunch g2 = g1;
     g2.tmA = &h->tmAct;
@@ -930,13 +948,20 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     g2.epi_mode = EPI_STORE;
     g2.out = h->Y;
     g2.ldo = d;
-    e = h->timed(K_GEMM_DOWN, st, [&] { return launch_grouped_gemm(g2, h->num_sms, st); });
+    g2.ksplit = small ? grouped_gemm_ksplit(est_groups * g2.n_tiles_n, c.F / 64, h->num_sms) : 1;
+    g2.ldp = g2.n_tiles_n * 256;
+    g2.pstride = (size_t)kSplitKRows * g2.ldp;
+    e = h->timed(K_GEMM_DOWN, st, [&] {
+        cudaError_t e2 = launch_grouped_gemm(g2, h->num_sms, st);
+        return (e2 == cudaSuccess && g2.ksplit > 1) ? launch_splitk_finish(g2, h->num_sms, st) : e2;
+    });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm down: ") + cudaGetErrorString(e));
     h->n_gemm_up++;
     h->n_gemm_down++;
-    h->launches += 8 + (shared_tabs ? 1 : 0);
+    h->launches += 8 + (shared_tabs ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
     if (has_sh) {
         GemmLaunch s1 = g1;
+        s1.ksplit = 1;
         s1.tmB = &h->tmW13sh[layer];
         s1.first_group = E;
         s1.ngroups = 1;
