@@ -28,6 +28,16 @@
 // activations stay resident while the weights stream.
 // Every mbarrier wait is bounded (2 s); on expiry the kernel records an error
 // word, stops issuing work, frees its TMEM and returns.
+//
+// Pair variant (launches whose groups are large): clusters of two CTAs on two
+// SMs issue tcgen05.mma.cta_group::2 with M = 256, N = 256.  Each CTA stages
+// its own 128 rows of A and its own half (128 output columns) of B, 32 KB per
+// stage in 6 stages, and holds its 128 rows x 256 columns of the accumulator
+// in its own TMEM; the even CTA issues the MMAs for both.  Per SM this halves
+// the B bytes staged per FLOP, so the same shared memory keeps 5 stages
+// (~2500 tensor cycles) of loads in flight instead of 3.  A row-pair tile
+// covers 256 rows of one group (the odd CTA's rows may lie past the group:
+// loaded, computed and masked).
 #include <algorithm>
 
 #include "internal.cuh"
@@ -40,13 +50,17 @@ constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int P_STAGES = 6;                       // pair variant
+constexpr int PB_BYTES = (BN / 2) * BK * 2;        // this CTA's half of the B tile
+constexpr int P_STAGE_BYTES = A_BYTES + PB_BYTES;
 constexpr int kThreads = 192;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int kMaxGroups = kMaxE + 1;
 
-struct __align__(8) GemmSmemTail {
-    uint64_t full[STAGES];
-    uint64_t empty[STAGES];
+template <int NST>
+struct __align__(8) SmemTail {
+    uint64_t full[NST];
+    uint64_t empty[NST];
     uint64_t tfull[2];
     uint64_t tempty[2];
     uint32_t tmem_base;
@@ -56,21 +70,45 @@ struct __align__(8) GemmSmemTail {
     int gstart[kMaxGroups];
     int gcnt[kMaxGroups];
 };
+using GemmSmemTail = SmemTail<STAGES>;
+using PairSmemTail = SmemTail<P_STAGES>;
 
 constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + sizeof(GemmSmemTail);
+constexpr size_t kPairSmemBytes = 1024 + (size_t)P_STAGES * P_STAGE_BYTES + sizeof(PairSmemTail);
 
 struct Tile {
     int rows, a_row, out_row, b_row, nt;
 };
 
+// Per-group tile counts from the device-side group offsets (tile_rows rows per
+// row tile); one thread.
+template <class Tail>
+__device__ __forceinline__ void build_tile_table(Tail* tl, const int* goff, int first_group, int ngroups,
+                                                 int n_tiles_n, int tile_rows) {
+    int acc = 0;
+    for (int g = 0; g < ngroups; ++g) {
+        const int st = goff[first_group + g];
+        const int cnt = goff[first_group + g + 1] - st;
+        tl->gstart[g] = st;
+        tl->gcnt[g] = cnt;
+        tl->tile_start[g] = acc;
+        acc += ((cnt + tile_rows - 1) / tile_rows) * n_tiles_n;
+    }
+    tl->tile_start[ngroups] = acc;
+    tl->total_tiles = acc;
+    tl->abort_flag = 0;
+}
+
 // Tile t -> (group, row tile, column tile).  Within a group the row tiles are
 // taken in blocks of mblk (an activation block small enough to stay in L2);
 // inside a block the column tile is the slow index and the row tile the fast
 // one, so the CTAs running at the same time share one weight tile and the
-// block's activation rows are read from HBM once.
-__device__ __forceinline__ Tile map_tile(const GemmSmemTail* tl, int t, int ngroups, int n_tiles_n,
-                                         int base0, int a_rebase, int out_rebase, int b_rows_per_group,
-                                         int mblk) {
+// block's activation rows are read from HBM once.  A row tile has tile_rows
+// rows; this CTA takes the 128 from sub_row on and B rows from b_sub on.
+template <class Tail>
+__device__ __forceinline__ Tile map_tile(const Tail* tl, int t, int ngroups, int n_tiles_n, int base0,
+                                         int a_rebase, int out_rebase, int b_rows_per_group, int mblk,
+                                         int tile_rows, int sub_row, int b_sub) {
     int lo = 0, hi = ngroups - 1;
     while (lo < hi) {                      // largest g with tile_start[g] <= t
         const int mid = (lo + hi + 1) >> 1;
@@ -78,7 +116,7 @@ __device__ __forceinline__ Tile map_tile(const GemmSmemTail* tl, int t, int ngro
     }
     const int g = lo;
     const int cnt = tl->gcnt[g];
-    const int mtc = (cnt + BM - 1) / BM;
+    const int mtc = (cnt + tile_rows - 1) / tile_rows;
     const int u = t - tl->tile_start[g];
     const int nfull = mtc / mblk;
     const int full_tiles = nfull * mblk * n_tiles_n;
@@ -94,11 +132,12 @@ __device__ __forceinline__ Tile map_tile(const GemmSmemTail* tl, int t, int ngro
         nt = r / last;
         mt = nfull * mblk + (r - nt * last);
     }
+    const int r0 = mt * tile_rows + sub_row;
     Tile r;
-    r.rows = min(BM, cnt - mt * BM);
-    r.a_row = tl->gstart[g] - (a_rebase ? base0 : 0) + mt * BM;
-    r.out_row = tl->gstart[g] - (out_rebase ? base0 : 0) + mt * BM;
-    r.b_row = g * b_rows_per_group + nt * BN;
+    r.rows = max(0, min(BM, cnt - r0));
+    r.a_row = tl->gstart[g] - (a_rebase ? base0 : 0) + r0;
+    r.out_row = tl->gstart[g] - (out_rebase ? base0 : 0) + r0;
+    r.b_row = g * b_rows_per_group + nt * BN + b_sub;
     r.nt = nt;
     return r;
 }
@@ -116,6 +155,130 @@ __device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float (&v)
     }
 }
 
+// Epilogue of one tile for one warp: TMEM lane quarter q (rows q*32 + lane),
+// all BN accumulator columns at tb; K range kr when the K dimension is split.
+__device__ __forceinline__ void epilogue_tile(uint32_t tb, int row, const Tile& ti, int kr, int ksplit,
+                                              int epi_mode, __nv_bfloat16* __restrict__ out, int ldo,
+                                              const __nv_bfloat16* __restrict__ res, int ldr,
+                                              const float2* __restrict__ rope, int rope_S, int rope_dh,
+                                              int n_rot, float* __restrict__ partial, int ldp,
+                                              size_t pstride) {
+    const bool valid = row < ti.rows;
+    __nv_bfloat16* orow = out + (size_t)(ti.out_row + (valid ? row : 0)) * ldo;
+    if (ksplit > 1) {
+        // fp32 partial sums of this K range; the finish kernel adds the ranges.
+        float* prow = partial + (size_t)kr * pstride + (size_t)(ti.out_row + (valid ? row : 0)) * ldp +
+                      ti.nt * BN;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+            uint32_t r[32];
+            tmem_ld_32x32(tb + c, r);
+            tmem_ld_wait();
+            if (valid) {
+                float4* d4 = reinterpret_cast<float4*>(prow + c);
+#pragma unroll
+                for (int q4 = 0; q4 < 8; ++q4)
+                    d4[q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
+                                         __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
+            }
+        }
+    } else if (epi_mode == EPI_SWIGLU) {
+#pragma unroll 1
+        for (int c = 0; c < BN / 2; c += 32) {
+            uint32_t gr[32], ur[32];
+            tmem_ld_32x32(tb + c, gr);
+            tmem_ld_32x32(tb + BN / 2 + c, ur);
+            tmem_ld_wait();
+            if (valid) {
+                float v[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float gt = __uint_as_float(gr[i]);
+                    const float up = __uint_as_float(ur[i]);
+                    v[i] = gt / (1.f + __expf(-gt)) * up;
+                }
+                store_row32(orow + ti.nt * (BN / 2) + c, v);
+            }
+        }
+    } else if (epi_mode == EPI_ROPE) {
+        // Rotary embedding of the query and key heads in the leading n_rot
+        // columns (pairs i, i + Dh/2 of each head; position = row mod S),
+        // the remaining (value) heads stored as they are.
+        const int pos = (ti.out_row + (valid ? row : 0)) % rope_S;
+        const int half = rope_dh >> 1;
+#pragma unroll 1
+        for (int h0 = 0; h0 < BN; h0 += rope_dh) {
+            const int col0 = ti.nt * BN + h0;
+            if (col0 < n_rot) {
+#pragma unroll 1
+                for (int c = 0; c < half; c += 32) {
+                    uint32_t xa[32], xb[32];
+                    tmem_ld_32x32(tb + h0 + c, xa);
+                    tmem_ld_32x32(tb + h0 + half + c, xb);
+                    tmem_ld_wait();
+                    if (valid) {
+                        const float2* cs = rope + (size_t)pos * half + c;
+                        float ya[32], yb[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            const float2 w = __ldg(cs + i);
+                            const float x1 = __uint_as_float(xa[i]), x2 = __uint_as_float(xb[i]);
+                            ya[i] = x1 * w.x - x2 * w.y;
+                            yb[i] = x2 * w.x + x1 * w.y;
+                        }
+                        store_row32(orow + col0 + c, ya);
+                        store_row32(orow + col0 + half + c, yb);
+                    }
+                }
+            } else {
+#pragma unroll 1
+                for (int c = 0; c < rope_dh; c += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32(tb + h0 + c, r);
+                    tmem_ld_wait();
+                    if (valid) {
+                        float v[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                        store_row32(orow + col0 + c, v);
+                    }
+                }
+            }
+        }
+    } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+            uint32_t r[32];
+            tmem_ld_32x32(tb + c, r);
+            tmem_ld_wait();
+            if (valid) {
+                float v[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float x = __uint_as_float(r[i]);
+                    v[i] = epi_mode == EPI_RELU ? fmaxf(x, 0.f) : x;
+                }
+                if (epi_mode == EPI_RESID) {
+                    const uint4* rr = reinterpret_cast<const uint4*>(
+                        res + (size_t)(ti.out_row + row) * ldr + ti.nt * BN + c);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        const uint4 w = __ldg(rr + q4);
+                        v[q4 * 8 + 0] += bf16_lo(w.x);
+                        v[q4 * 8 + 1] += bf16_hi(w.x);
+                        v[q4 * 8 + 2] += bf16_lo(w.y);
+                        v[q4 * 8 + 3] += bf16_hi(w.y);
+                        v[q4 * 8 + 4] += bf16_lo(w.z);
+                        v[q4 * 8 + 5] += bf16_hi(w.z);
+                        v[q4 * 8 + 6] += bf16_lo(w.w);
+                        v[q4 * 8 + 7] += bf16_hi(w.w);
+                    }
+                }
+                store_row32(orow + ti.nt * BN + c, v);
+            }
+        }
+    }
+}
 __global__ void __launch_bounds__(kThreads, 1)
 grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
@@ -136,22 +299,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     const int lane = threadIdx.x & 31;
 
     // Tile table from the device-side group offsets.
-    if (threadIdx.x == 0) {
-        const int base0 = goff[first_group];
-        int acc = 0;
-        for (int g = 0; g < ngroups; ++g) {
-            const int st = goff[first_group + g];
-            const int cnt = goff[first_group + g + 1] - st;
-            tl->gstart[g] = st;
-            tl->gcnt[g] = cnt;
-            tl->tile_start[g] = acc;
-            acc += ((cnt + BM - 1) / BM) * n_tiles_n;
-        }
-        tl->tile_start[ngroups] = acc;
-        tl->total_tiles = acc;
-        tl->abort_flag = 0;
-        (void)base0;
-    }
+    if (threadIdx.x == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, BM);
     __syncthreads();
     const int ntiles = tl->total_tiles;
     const int total = ntiles * ksplit;    // unit u: tile u % ntiles, K range u / ntiles
@@ -186,7 +334,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             int it = 0;
             for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
                 const Tile ti = map_tile(tl, t % ntiles, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
-                                         b_rows_per_group, mblk);
+                                         b_rows_per_group, mblk, BM, 0, 0);
                 const int kb0 = (t / ntiles) * kbr;
                 for (int kb = kb0; kb < kb0 + kbr; ++kb, ++it) {
                     const int s = it % STAGES;
@@ -245,7 +393,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         int tl_i = 0;
         for (int t = blockIdx.x; t < total; t += gridDim.x, ++tl_i) {
             const Tile ti = map_tile(tl, t % ntiles, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
-                                     b_rows_per_group, mblk);
+                                     b_rows_per_group, mblk, BM, 0, 0);
             const int buf = tl_i & 1;
             const uint32_t aph = (tl_i >> 1) & 1;
             int ok = 1;
@@ -255,121 +403,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             if (!ok) break;
             tc_fence_after();
             const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
-            const bool valid = row < ti.rows;
-            __nv_bfloat16* orow = out + (size_t)(ti.out_row + (valid ? row : 0)) * ldo;
-            if (ksplit > 1) {
-                // fp32 partial sums of this K range; the finish kernel adds the ranges.
-                float* prow = partial + (size_t)(t / ntiles) * pstride +
-                              (size_t)(ti.out_row + (valid ? row : 0)) * ldp + ti.nt * BN;
-#pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    uint32_t r[32];
-                    tmem_ld_32x32(tb + c, r);
-                    tmem_ld_wait();
-                    if (valid) {
-                        float4* d4 = reinterpret_cast<float4*>(prow + c);
-#pragma unroll
-                        for (int q4 = 0; q4 < 8; ++q4)
-                            d4[q4] = make_float4(__uint_as_float(r[4 * q4]), __uint_as_float(r[4 * q4 + 1]),
-                                                 __uint_as_float(r[4 * q4 + 2]), __uint_as_float(r[4 * q4 + 3]));
-                    }
-                }
-            } else if (epi_mode == EPI_SWIGLU) {
-#pragma unroll 1
-                for (int c = 0; c < BN / 2; c += 32) {
-                    uint32_t gr[32], ur[32];
-                    tmem_ld_32x32(tb + c, gr);
-                    tmem_ld_32x32(tb + BN / 2 + c, ur);
-                    tmem_ld_wait();
-                    if (valid) {
-                        float v[32];
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float gt = __uint_as_float(gr[i]);
-                            const float up = __uint_as_float(ur[i]);
-                            v[i] = gt / (1.f + __expf(-gt)) * up;
-                        }
-                        store_row32(orow + ti.nt * (BN / 2) + c, v);
-                    }
-                }
-            } else if (epi_mode == EPI_ROPE) {
-                // Rotary embedding of the query and key heads in the leading n_rot
-                // columns (pairs i, i + Dh/2 of each head; position = row mod S),
-                // the remaining (value) heads stored as they are.
-                const int pos = (ti.out_row + (valid ? row : 0)) % rope_S;
-                const int half = rope_dh >> 1;
-#pragma unroll 1
-                for (int h0 = 0; h0 < BN; h0 += rope_dh) {
-                    const int col0 = ti.nt * BN + h0;
-                    if (col0 < n_rot) {
-#pragma unroll 1
-                        for (int c = 0; c < half; c += 32) {
-                            uint32_t xa[32], xb[32];
-                            tmem_ld_32x32(tb + h0 + c, xa);
-                            tmem_ld_32x32(tb + h0 + half + c, xb);
-                            tmem_ld_wait();
-                            if (valid) {
-                                const float2* cs = rope + (size_t)pos * half + c;
-                                float ya[32], yb[32];
-#pragma unroll
-                                for (int i = 0; i < 32; ++i) {
-                                    const float2 w = __ldg(cs + i);
-                                    const float x1 = __uint_as_float(xa[i]), x2 = __uint_as_float(xb[i]);
-                                    ya[i] = x1 * w.x - x2 * w.y;
-                                    yb[i] = x2 * w.x + x1 * w.y;
-                                }
-                                store_row32(orow + col0 + c, ya);
-                                store_row32(orow + col0 + half + c, yb);
-                            }
-                        }
-                    } else {
-#pragma unroll 1
-                        for (int c = 0; c < rope_dh; c += 32) {
-                            uint32_t r[32];
-                            tmem_ld_32x32(tb + h0 + c, r);
-                            tmem_ld_wait();
-                            if (valid) {
-                                float v[32];
-#pragma unroll
-                                for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-                                store_row32(orow + col0 + c, v);
-                            }
-                        }
-                    }
-                }
-            } else {
-#pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    uint32_t r[32];
-                    tmem_ld_32x32(tb + c, r);
-                    tmem_ld_wait();
-                    if (valid) {
-                        float v[32];
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) {
-                            const float x = __uint_as_float(r[i]);
-                            v[i] = epi_mode == EPI_RELU ? fmaxf(x, 0.f) : x;
-                        }
-                        if (epi_mode == EPI_RESID) {
-                            const uint4* rr = reinterpret_cast<const uint4*>(
-                                res + (size_t)(ti.out_row + row) * ldr + ti.nt * BN + c);
-#pragma unroll
-                            for (int q4 = 0; q4 < 4; ++q4) {
-                                const uint4 w = __ldg(rr + q4);
-                                v[q4 * 8 + 0] += bf16_lo(w.x);
-                                v[q4 * 8 + 1] += bf16_hi(w.x);
-                                v[q4 * 8 + 2] += bf16_lo(w.y);
-                                v[q4 * 8 + 3] += bf16_hi(w.y);
-                                v[q4 * 8 + 4] += bf16_lo(w.z);
-                                v[q4 * 8 + 5] += bf16_hi(w.z);
-                                v[q4 * 8 + 6] += bf16_lo(w.w);
-                                v[q4 * 8 + 7] += bf16_hi(w.w);
-                            }
-                        }
-                        store_row32(orow + ti.nt * BN + c, v);
-                    }
-                }
-            }
+            epilogue_tile(tb, row, ti, t / ntiles, ksplit, epi_mode, out, ldo, res, ldr, rope, rope_S, rope_dh,
+                          n_rot, partial, ldp, pstride);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&tl->tempty[buf]));
@@ -384,9 +419,190 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     }
 }
 
+// Pair variant: one cluster of two CTAs per row-pair tile of 256 rows x 256
+// columns.  The tile sequence is shared by both CTAs; CTA rank r takes rows
+// [r * 128, r * 128 + 128) of the tile and B rows (output columns)
+// [r * 128, r * 128 + 128) of the column tile.
+//   full[s]   (even CTA)  both CTAs' TMA loads of stage s complete on it
+//   empty[s]  (each CTA)  released by the even CTA's MMA commit, multicast
+//   tfull[b]  (each CTA)  accumulator b ready, multicast commit
+//   tempty[b] (even CTA)  8 arrivals: the 4 epilogue warps of each CTA
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                         const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
+                         int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
+                         __nv_bfloat16* __restrict__ out, int ldo, int* err,
+                         const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
+                         int rope_S, int rope_dh, int n_rot, int mblk) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
+    uint8_t* smem = smem_raw + pad;
+    const uint32_t sA = smem_u32(smem);
+    const uint32_t sB = sA + P_STAGES * A_BYTES;
+    PairSmemTail* tl = reinterpret_cast<PairSmemTail*>(smem + (size_t)P_STAGES * P_STAGE_BYTES);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();      // 0: issues the MMAs, 1: peer
+    const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
+    const int sub = (int)rank * (BM);             // this CTA's rows / B rows within the tile
+
+    if (threadIdx.x == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, 2 * BM);
+    __syncthreads();
+    const int ntiles = tl->total_tiles;
+    if (cid >= ntiles) return;                    // both CTAs of the pair leave together
+    const int base0 = tl->gstart[0];
+    const int nkb = K / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < P_STAGES; ++s) {
+            mbar_init(smem_u32(&tl->full[s]), 1);
+            mbar_init(smem_u32(&tl->empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&tl->tfull[b]), 1);
+            mbar_init(smem_u32(&tl->tempty[b]), 8);
+        }
+        fence_barrier_init();
+        prefetch_tmap(&tmA);
+        prefetch_tmap(&tmB);
+    }
+    if (warp == 0) tmem_alloc_pair(smem_u32(&tl->tmem_base), TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();                               // both CTAs' barriers are initialised
+    tc_fence_after();
+    const uint32_t tmem_base = tl->tmem_base;
+    volatile int* abort_flag = &tl->abort_flag;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------------------------------------------- producer (both CTAs)
+            int it = 0;
+            for (int t = cid; t < ntiles && !*abort_flag; t += ncl) {
+                const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
+                                         b_rows_per_group, mblk, 2 * BM, sub, sub);
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % P_STAGES;
+                    const uint32_t ph = (it / P_STAGES) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&tl->empty[s]), ph ^ 1, abort_flag, err,
+                                           ERR_TIMEOUT_PRODUCER))
+                        break;
+                    if (rank == 0) mbar_arrive_expect_tx(smem_u32(&tl->full[s]), 2 * P_STAGE_BYTES);
+                    const uint32_t fb = mapa_shared(smem_u32(&tl->full[s]), 0);
+                    tma_load_2d_pair(sA + s * A_BYTES, &tmA, kb * BK, ti.a_row, fb);
+                    tma_load_2d_pair(sB + s * PB_BYTES, &tmB, kb * BK, ti.b_row, fb);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) {
+            // ---------------------------------------------------- MMA issuer (even CTA)
+            constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
+            int it = 0, tl_i = 0;
+            bool ok = true;
+            for (int t = cid; t < ntiles && ok; t += ncl, ++tl_i) {
+                const int buf = tl_i & 1;
+                const uint32_t aph = (tl_i >> 1) & 1;
+                if (!mbar_wait_bounded(smem_u32(&tl->tempty[buf]), aph ^ 1, abort_flag, err,
+                                       ERR_TIMEOUT_MMA)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % P_STAGES;
+                    const uint32_t ph = (it / P_STAGES) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&tl->full[s]), ph, abort_flag, err, ERR_TIMEOUT_MMA)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = sA + s * A_BYTES;
+                    const uint32_t b0 = sB + s * PB_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        tc_mma_bf16_pair(d_tmem, smem_desc_sw128(a0 + kk * 32), smem_desc_sw128(b0 + kk * 32),
+                                         idesc, (kb != 0 || kk != 0) ? 1u : 0u);
+                    tc_commit_pair_mc(smem_u32(&tl->empty[s]), 0x3);
+                }
+                if (!ok) break;
+                tc_commit_pair_mc(smem_u32(&tl->tfull[buf]), 0x3);
+            }
+        }
+    } else {
+        // -------------------------------------------------------- epilogue (both CTAs)
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        int tl_i = 0;
+        for (int t = cid; t < ntiles; t += ncl, ++tl_i) {
+            const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
+                                     b_rows_per_group, mblk, 2 * BM, sub, sub);
+            const int buf = tl_i & 1;
+            const uint32_t aph = (tl_i >> 1) & 1;
+            int ok = 1;
+            if (lane == 0)
+                ok = mbar_wait_bounded(smem_u32(&tl->tfull[buf]), aph, abort_flag, err, ERR_TIMEOUT_EPI);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            tc_fence_after();
+            const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
+            epilogue_tile(tb, row, ti, 0, 1, epi_mode, out, ldo, res, ldr, rope, rope_S, rope_dh, n_rot, nullptr,
+                          0, 0);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                if (rank == 0) mbar_arrive(smem_u32(&tl->tempty[buf]));
+                else mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tempty[buf]), 0));
+            }
+        }
+    }
+
+    // A CTA that gave up tells its peer, so that the peer stops waiting on it.
+    __syncthreads();
+    if (threadIdx.x == 0 && *abort_flag)
+        st_shared_cluster_u32(mapa_shared(smem_u32(&tl->abort_flag), rank ^ 1u), 1u);
+    cluster_sync();                               // no access to the peer's memory remains in flight
+    if (warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    }
+}
+
 }  // namespace
 
 size_t grouped_gemm_smem_bytes() { return kSmemBytes; }
+
+namespace {
+
+// Clusters of two that fit on the device at once (the pair kernel is
+// persistent, so it launches no more than that); 0 if none.
+int pair_clusters(int num_sms) {
+    static int n = -1;
+    if (n >= 0) return n;
+    n = 0;
+    if (cudaFuncSetAttribute(grouped_gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kPairSmemBytes) != cudaSuccess)
+        return n;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(num_sms & ~1), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kPairSmemBytes;
+    int ncl = 0;
+    if (cudaOccupancyMaxActiveClusters(&ncl, grouped_gemm_pair_kernel, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return n;
+    }
+    n = std::min(ncl, num_sms / 2);
+    return n;
+}
+
+}  // namespace
+
+int grouped_gemm_pair_clusters(int num_sms) { return pair_clusters(num_sms); }
 
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st) {
     static bool attr_set = false;
@@ -400,6 +616,14 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     // Row tiles per block: about 48 MB of activations (a third of L2), so that
     // a block stays resident while the weight tiles stream past it.
     const long long a_tile_bytes = (long long)BM * g.K * 2;
+    if (g.tmB_pair && (g.ksplit <= 1) && pair_clusters(num_sms) > 0) {
+        const int mblk2 = (int)std::max(1LL, (48LL << 20) / (2 * a_tile_bytes));
+        grouped_gemm_pair_kernel<<<2 * pair_clusters(num_sms), kThreads, kPairSmemBytes, st>>>(
+            *g.tmA, *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
+            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh,
+            g.n_rot, mblk2);
+        return cudaGetLastError();
+    }
     const int mblk = (int)std::max(1LL, (48LL << 20) / a_tile_bytes);
     grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
         *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,

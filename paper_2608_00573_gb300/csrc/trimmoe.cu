@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <limits>
 #include <mutex>
@@ -56,6 +57,12 @@ bool make_tmap(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer
 
 // Small batches: routed GEMMs with at most kSplitKRows executed pairs may split K.
 constexpr int kSplitKMax = 8, kSplitKRows = 64;
+// GEMM launches whose groups average at least kPairMinRows rows run on CTA
+// pairs (256-row tiles): below that the extra padding of a 256-row tail tile
+// outweighs the pair's faster main loop.
+constexpr int kPairMinRows = 2048;
+
+inline bool pair_gemm(long long rows_per_group) { return rows_per_group >= kPairMinRows; }
 
 enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
 
@@ -165,6 +172,8 @@ struct trimmoe {
 
     CUtensorMap tmXp, tmAct, tmActSh;
     std::vector<CUtensorMap> tmW13, tmW2, tmW13sh, tmW2sh;
+    // the same weights in 128-row boxes (each CTA's half of a B tile in the pair kernel)
+    std::vector<CUtensorMap> tmW13p, tmW2p, tmW13shp, tmW2shp;
 
     // attention sublayer of the full block
     int nqkv = 0;
@@ -173,7 +182,7 @@ struct trimmoe {
     float2* rope = nullptr;           // [attn_seq][head_dim/2] (cos, sin)
     float* sqbuf_x = nullptr;         // [rows_part] partial sums of squares of the layer input
     CUtensorMap tmAttn;
-    std::vector<CUtensorMap> tmWqkv, tmWo;
+    std::vector<CUtensorMap> tmWqkv, tmWo, tmWqkvp, tmWop;
     double flops_attn = 0.0, flops_attn_gemm = 0.0;
 
     // host-buffer forward
@@ -641,17 +650,25 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     if (has_sh) tm = tm && make_tmap(&h->tmActSh, h->act_sh, c.F_sh, T, 128);
     h->tmW13.resize(N);
     h->tmW2.resize(N);
-    if (has_sh) { h->tmW13sh.resize(N); h->tmW2sh.resize(N); }
+    h->tmW13p.resize(N);
+    h->tmW2p.resize(N);
+    if (has_sh) { h->tmW13sh.resize(N); h->tmW2sh.resize(N); h->tmW13shp.resize(N); h->tmW2shp.resize(N); }
     const __nv_bfloat16* W13 = static_cast<const __nv_bfloat16*>(w->W13);
     const __nv_bfloat16* W2 = static_cast<const __nv_bfloat16*>(w->W2);
     for (int l = 0; l < N && tm; ++l) {
-        tm = make_tmap(&h->tmW13[l], W13 + (size_t)l * E * F13 * d, d, (uint64_t)E * F13, 256) &&
-             make_tmap(&h->tmW2[l], W2 + (size_t)l * E * d * c.F, c.F, (uint64_t)E * d, 256);
-        if (tm && has_sh) {
-            const __nv_bfloat16* W13s = static_cast<const __nv_bfloat16*>(w->W13_sh);
-            const __nv_bfloat16* W2s = static_cast<const __nv_bfloat16*>(w->W2_sh);
-            tm = make_tmap(&h->tmW13sh[l], W13s + (size_t)l * 2 * c.F_sh * d, d, (uint64_t)2 * c.F_sh, 256) &&
-                 make_tmap(&h->tmW2sh[l], W2s + (size_t)l * d * c.F_sh, c.F_sh, (uint64_t)d, 256);
+        for (uint32_t box : {256u, 128u}) {
+            CUtensorMap* m13 = box == 256 ? &h->tmW13[l] : &h->tmW13p[l];
+            CUtensorMap* m2 = box == 256 ? &h->tmW2[l] : &h->tmW2p[l];
+            tm = tm && make_tmap(m13, W13 + (size_t)l * E * F13 * d, d, (uint64_t)E * F13, box) &&
+                 make_tmap(m2, W2 + (size_t)l * E * d * c.F, c.F, (uint64_t)E * d, box);
+            if (tm && has_sh) {
+                const __nv_bfloat16* W13s = static_cast<const __nv_bfloat16*>(w->W13_sh);
+                const __nv_bfloat16* W2s = static_cast<const __nv_bfloat16*>(w->W2_sh);
+                tm = make_tmap(box == 256 ? &h->tmW13sh[l] : &h->tmW13shp[l], W13s + (size_t)l * 2 * c.F_sh * d, d,
+                               (uint64_t)2 * c.F_sh, box) &&
+                     make_tmap(box == 256 ? &h->tmW2sh[l] : &h->tmW2shp[l], W2s + (size_t)l * d * c.F_sh, c.F_sh,
+                               (uint64_t)d, box);
+            }
         }
     }
     if (tm && has_attn) {
@@ -660,10 +677,14 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         const __nv_bfloat16* Wo = static_cast<const __nv_bfloat16*>(w->W_o);
         h->tmWqkv.resize(N);
         h->tmWo.resize(N);
+        h->tmWqkvp.resize(N);
+        h->tmWop.resize(N);
         tm = make_tmap(&h->tmAttn, h->attn_out, hd, T, 128);
         for (int l = 0; l < N && tm; ++l)
             tm = make_tmap(&h->tmWqkv[l], Wqkv + (size_t)l * h->nqkv * d, d, (uint64_t)h->nqkv, 256) &&
-                 make_tmap(&h->tmWo[l], Wo + (size_t)l * d * hd, hd, (uint64_t)d, 256);
+                 make_tmap(&h->tmWo[l], Wo + (size_t)l * d * hd, hd, (uint64_t)d, 256) &&
+                 make_tmap(&h->tmWqkvp[l], Wqkv + (size_t)l * h->nqkv * d, d, (uint64_t)h->nqkv, 128) &&
+                 make_tmap(&h->tmWop[l], Wo + (size_t)l * d * hd, hd, (uint64_t)d, 128);
     }
     if (!tm) return bail(TRIMMOE_ERR_CUDA, "create: cuTensorMapEncodeTiled failed");
     *out = h;
@@ -747,6 +768,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         qg.out = h->qkv;
         qg.ldo = h->nqkv;
         qg.err = h->dev_err;
+        qg.tmB_pair = pair_gemm(T) ? &h->tmWqkvp[layer] : nullptr;
         e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(qg, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("qkv gemm: ") + cudaGetErrorString(e));
         e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, c.head_dim, st); });
@@ -755,6 +777,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         og.rope = nullptr;
         og.tmA = &h->tmAttn;
         og.tmB = &h->tmWo[layer];
+        og.tmB_pair = pair_gemm(T) ? &h->tmWop[layer] : nullptr;
         og.K = hd;
         og.n_tiles_n = d / 256;
         og.b_rows_per_group = d;
@@ -912,6 +935,8 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     GemmLaunch g1{};
     g1.tmA = &h->tmXp;
     g1.tmB = &h->tmW13[layer];
+    const bool pair_routed = pair_gemm((long long)T * K / E);
+    g1.tmB_pair = pair_routed ? &h->tmW13p[layer] : nullptr;
     g1.goff = h->goff;
     g1.first_group = 0;
     g1.ngroups = E;
@@ -942,6 +967,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     GemmLaunch g2 = g1;
     g2.tmA = &h->tmAct;
     g2.tmB = &h->tmW2[layer];
+    g2.tmB_pair = pair_routed ? &h->tmW2p[layer] : nullptr;
     g2.K = c.F;
     g2.n_tiles_n = d / 256;
     g2.b_rows_per_group = d;
@@ -963,6 +989,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         GemmLaunch s1 = g1;
         s1.ksplit = 1;
         s1.tmB = &h->tmW13sh[layer];
+        s1.tmB_pair = pair_gemm(T) ? &h->tmW13shp[layer] : nullptr;
         s1.first_group = E;
         s1.ngroups = 1;
         s1.out_rebase = 1;
@@ -976,6 +1003,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         GemmLaunch s2 = s1;
         s2.tmA = &h->tmActSh;
         s2.tmB = &h->tmW2sh[layer];
+        s2.tmB_pair = pair_gemm(T) ? &h->tmW2shp[layer] : nullptr;
         s2.a_rebase = 1;
         s2.K = c.F_sh;
         s2.n_tiles_n = d / 256;

@@ -36,12 +36,16 @@ BLOCKS = {
     "relu_c64_s37_kc16": small_cfg(name="b3", N=4, d=256, E=8, k=1, F=256, C=64, act=W.ACT_RELU, T=300, M=10,
                                    attn_heads=4, attn_kv_heads=4, head_dim=64, attn_seq=37, n_centroids=16,
                                    seed=43),
+    # 4200 tokens: the attention projections and the routed experts (2100 rows
+    # per group on average) run on CTA pairs, 256-row tiles with a ragged tail
+    "gqa_pair_T4200": small_cfg(name="b5", N=2, d=512, E=4, k=2, F=256, T=4200, M=10, H=3, renorm_topk=1,
+                                attn_heads=8, attn_kv_heads=2, head_dim=64, attn_seq=128, seed=44),
 }
 
 
 # exit-head bias per configuration: the 64-class head's max-softmax confidence
 # needs a larger bias than the sigmoid head to reach p_J = 0.9
-EXIT_BIAS = {"gqa_h64_s128": 1.0, "mha_h128_s100_shared": 1.0, "relu_c64_s37_kc16": 5.0}
+EXIT_BIAS = {"gqa_h64_s128": 1.0, "mha_h128_s100_shared": 1.0, "relu_c64_s37_kc16": 5.0, "gqa_pair_T4200": 1.0}
 
 
 @pytest.mark.parametrize("name", list(BLOCKS))

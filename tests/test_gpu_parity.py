@@ -236,6 +236,21 @@ def test_layer_parity_at_maximum_dimensions(name, kw):
     assert tot["exec"] > 0
 
 
+@pytest.mark.parametrize("name,kw", [
+    ("swiglu_shared_k2", dict(N=2, d=256, E=4, k=2, F=384, F_sh=256, T=4500, M=10, H=3)),
+    ("relu_k1_c64", dict(N=2, d=512, E=2, k=1, F=512, C=64, act=W.ACT_RELU, T=4400, M=10)),
+])
+def test_layer_parity_pair_gemm(name, kw):
+    """Groups averaging >= 2048 rows (and the shared expert's T rows) run the
+    grouped GEMM on CTA pairs (256-row tiles, tcgen05 cta_group::2); ragged
+    group tails leave the odd CTA's rows partly or wholly past the group."""
+    cfg = small_cfg(name=name, seed=98, **kw)
+    reports = _run_all_layers(cfg, theta=0.9, exit_bias=1.0 if cfg.C == 1 else 5.0)
+    tot = {k: sum(r[k] for r in reports) for k in ("exec", "skip", "exit")}
+    print(name, tot, [round(r["max_rel_err"], 5) for r in reports])
+    assert tot["exec"] > 0
+
+
 @pytest.mark.parametrize("budget", [0.0, float("inf")])
 def test_budget_edge_cases(budget):
     """Dbar = 0: only exact execution fits (Q = 0), no skip; Dbar = inf: every
