@@ -82,7 +82,7 @@ enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
  *  the plain launches.  Not used on the legacy or per-thread default stream,
  *  or when the stream is already being captured (the launches then go into
  *  the caller's capture); feedback and calibration calls drop the graph.
- * Supported: d % 256 == 0; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
+ * Supported: d % 256 == 0, d <= 16384; SwiGLU F % 128 == 0, ReLU F % 256 == 0;
  * F_sh % 128 == 0; E <= 128; k <= min(E, 8); C <= 256; M*E <= 1024; H <= 6;
  * n_sub <= 3; attention: head_dim 64 or 128, attn_heads % attn_kv_heads == 0,
  * (attn_heads + 2 attn_kv_heads) * head_dim % 256 == 0, 1 <= attn_seq <= 128,

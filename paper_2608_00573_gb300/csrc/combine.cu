@@ -11,118 +11,116 @@
 // when requested; a substitute expert takes its target's gate.  A skipped
 // layer is the identity (residual) path of Sec. III-B; the shared expert is
 // local and runs for every token that is still active (Sec. III-B).
-// One warp per token, 16-byte loads and stores, fp32 accumulation in slot order.
+// One warp per token, 16-byte loads and stores, fp32 accumulation in slot order
+// (residual base, then w_j * Y_j for j ascending, then the shared row).
 #include "internal.cuh"
 
 namespace tmoe {
 
 namespace {
 
+// KT: slots held in registers (k <= KT).  All loads of one step (the residual
+// base, every slot's Y row and the shared expert's row, kU chunks of 16 bytes
+// per lane each) are issued before the first one is used.
+template <int KT>
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
+    constexpr int kU = KT <= 2 ? 4 : 2;
     const int lane = threadIdx.x & 31;
     const int nchunk = p.d >> 3;
     for (int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; t < p.T;
          t += (gridDim.x * blockDim.x) >> 5) {
         const int a = p.action[t];
         if (a > 1 || (a == 1 && !p.has_shared && p.h_src == p.h)) continue;
-        float w[kMaxK];
-        int pos[kMaxK];
-        int nj = 0;
+        float w[KT];
+        const uint4* yrow[KT];
+        const int nj = a == 0 ? p.k : 0;
         if (a == 0) {
-            nj = p.k;
             float gs = 0.f;
             for (int j = 0; j < nj; ++j) gs = __fadd_rn(gs, p.topk_g[t * p.k + j]);
 #pragma unroll
-            for (int j = 0; j < kMaxK; ++j) {
+            for (int j = 0; j < KT; ++j) {
                 if (j < nj) {
                     const float gj = p.topk_g[t * p.k + j];
                     w[j] = p.renorm ? __fdiv_rn(gj, gs) : gj;
-                    pos[j] = p.pos_pair[t * p.k + j];
+                    yrow[j] = reinterpret_cast<const uint4*>(p.Y + (size_t)p.pos_pair[t * p.k + j] * p.d);
                 }
             }
         }
         const int psh = p.has_shared ? p.pos_sh[t] : -1;
+        const uint4* srow = reinterpret_cast<const uint4*>(p.Ysh + (size_t)(psh >= 0 ? psh : 0) * p.d);
         uint4* hrow = reinterpret_cast<uint4*>(p.h + (size_t)t * p.d);
         const uint4* brow = reinterpret_cast<const uint4*>(p.h_src + (size_t)t * p.d);
-        // kU chunks of 16 bytes per lane at a time: every load of a step is in
-        // flight before the first one is used.
-        constexpr int kU = 4;
         for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
-            float acc[kU][8];
+            uint4 hv[kU], yv[KT][kU], sv[kU];
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const int c = c0 + 32 * u;
-                const uint4 hv = c < nchunk ? brow[c] : make_uint4(0u, 0u, 0u, 0u);
-                acc[u][0] = bf16_lo(hv.x); acc[u][1] = bf16_hi(hv.x);
-                acc[u][2] = bf16_lo(hv.y); acc[u][3] = bf16_hi(hv.y);
-                acc[u][4] = bf16_lo(hv.z); acc[u][5] = bf16_hi(hv.z);
-                acc[u][6] = bf16_lo(hv.w); acc[u][7] = bf16_hi(hv.w);
+                hv[u] = c < nchunk ? brow[c] : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
-            for (int j = 0; j < kMaxK; ++j) {
-                if (j >= nj) break;
-                const uint4* yrow = reinterpret_cast<const uint4*>(p.Y + (size_t)pos[j] * p.d);
-                uint4 y[kU];
+            for (int j = 0; j < KT; ++j)
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
                     const int c = c0 + 32 * u;
-                    y[u] = c < nchunk ? __ldg(yrow + c) : make_uint4(0u, 0u, 0u, 0u);
+                    yv[j][u] = (j < nj && c < nchunk) ? __ldg(yrow[j] + c) : make_uint4(0u, 0u, 0u, 0u);
                 }
 #pragma unroll
-                for (int u = 0; u < kU; ++u) {
-                    acc[u][0] = fmaf(w[j], bf16_lo(y[u].x), acc[u][0]);
-                    acc[u][1] = fmaf(w[j], bf16_hi(y[u].x), acc[u][1]);
-                    acc[u][2] = fmaf(w[j], bf16_lo(y[u].y), acc[u][2]);
-                    acc[u][3] = fmaf(w[j], bf16_hi(y[u].y), acc[u][3]);
-                    acc[u][4] = fmaf(w[j], bf16_lo(y[u].z), acc[u][4]);
-                    acc[u][5] = fmaf(w[j], bf16_hi(y[u].z), acc[u][5]);
-                    acc[u][6] = fmaf(w[j], bf16_lo(y[u].w), acc[u][6]);
-                    acc[u][7] = fmaf(w[j], bf16_hi(y[u].w), acc[u][7]);
-                }
-            }
-            if (psh >= 0) {
-                const uint4* yrow = reinterpret_cast<const uint4*>(p.Ysh + (size_t)psh * p.d);
-                uint4 y[kU];
-#pragma unroll
-                for (int u = 0; u < kU; ++u) {
-                    const int c = c0 + 32 * u;
-                    y[u] = c < nchunk ? __ldg(yrow + c) : make_uint4(0u, 0u, 0u, 0u);
-                }
-#pragma unroll
-                for (int u = 0; u < kU; ++u) {
-                    acc[u][0] += bf16_lo(y[u].x);
-                    acc[u][1] += bf16_hi(y[u].x);
-                    acc[u][2] += bf16_lo(y[u].y);
-                    acc[u][3] += bf16_hi(y[u].y);
-                    acc[u][4] += bf16_lo(y[u].z);
-                    acc[u][5] += bf16_hi(y[u].z);
-                    acc[u][6] += bf16_lo(y[u].w);
-                    acc[u][7] += bf16_hi(y[u].w);
-                }
+            for (int u = 0; u < kU; ++u) {
+                const int c = c0 + 32 * u;
+                sv[u] = (psh >= 0 && c < nchunk) ? __ldg(srow + c) : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const int c = c0 + 32 * u;
-                if (c < nchunk) {
-                    uint4 o;
-                    o.x = pack_bf16x2(acc[u][0], acc[u][1]);
-                    o.y = pack_bf16x2(acc[u][2], acc[u][3]);
-                    o.z = pack_bf16x2(acc[u][4], acc[u][5]);
-                    o.w = pack_bf16x2(acc[u][6], acc[u][7]);
-                    hrow[c] = o;
+                if (c >= nchunk) continue;
+                const uint32_t hw[4] = {hv[u].x, hv[u].y, hv[u].z, hv[u].w};
+                uint32_t ow[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float lo = bf16_lo(hw[q]), hi = bf16_hi(hw[q]);
+#pragma unroll
+                    for (int j = 0; j < KT; ++j) {
+                        if (j < nj) {
+                            const uint32_t yw = q == 0 ? yv[j][u].x : q == 1 ? yv[j][u].y : q == 2 ? yv[j][u].z : yv[j][u].w;
+                            lo = fmaf(w[j], bf16_lo(yw), lo);
+                            hi = fmaf(w[j], bf16_hi(yw), hi);
+                        }
+                    }
+                    if (psh >= 0) {
+                        const uint32_t sw = q == 0 ? sv[u].x : q == 1 ? sv[u].y : q == 2 ? sv[u].z : sv[u].w;
+                        lo += bf16_lo(sw);
+                        hi += bf16_hi(sw);
+                    }
+                    ow[q] = pack_bf16x2(lo, hi);
                 }
+                hrow[c] = make_uint4(ow[0], ow[1], ow[2], ow[3]);
             }
         }
     }
+}
+
+template <int KT>
+int combine_grid(int T, int num_sms) {
+    static int per_sm = 0;
+    if (per_sm == 0) {
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, combine_kernel<KT>, 256, 0) != cudaSuccess || n < 1)
+            n = 1;
+        per_sm = n;
+    }
+    const int want = (T + 7) / 8;
+    const int cap = num_sms * per_sm;
+    return want < cap ? want : cap;
 }
 
 }  // namespace
 
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    int blocks = (p.T + 7) / 8;
-    blocks = blocks < num_sms * 8 ? blocks : num_sms * 8;
-    combine_kernel<<<blocks, 256, 0, st>>>(p);
+    if (p.k <= 1) combine_kernel<1><<<combine_grid<1>(p.T, num_sms), 256, 0, st>>>(p);
+    else if (p.k <= 2) combine_kernel<2><<<combine_grid<2>(p.T, num_sms), 256, 0, st>>>(p);
+    else if (p.k <= 4) combine_kernel<4><<<combine_grid<4>(p.T, num_sms), 256, 0, st>>>(p);
+    else combine_kernel<kMaxK><<<combine_grid<kMaxK>(p.T, num_sms), 256, 0, st>>>(p);
     return cudaGetLastError();
 }
 

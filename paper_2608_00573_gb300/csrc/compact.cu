@@ -8,8 +8,9 @@
 // pairs reach the expert FFN.
 //
 // Three passes over chunks of kChunk tokens: per-chunk bucket counts, one
-// scan over chunks and buckets, and a scatter in which one warp walks its
-// chunk in order and ranks equal buckets with __match_any_sync.
+// scan over chunks and buckets, and a scatter in which each warp of a chunk's
+// block walks its 32 tokens in order and ranks equal buckets with
+// __match_any_sync.
 #include <mutex>
 #include <string>
 
@@ -37,48 +38,101 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const CompactParams p) {
     for (int i = threadIdx.x; i < nb; i += blockDim.x) p.blk_counts[blockIdx.x * nb + i] = cnt[i];
 }
 
-// One block: per bucket, exclusive prefix over chunks; then bucket offsets.
-__global__ void __launch_bounds__(256) scan_kernel(const CompactParams p) {
+// One block of 1024 threads: each warp takes buckets e = warp, warp + 32, ...
+// and scans the chunks' counts of that bucket (32 chunks per step); then one
+// warp turns the bucket totals into group offsets.
+__global__ void __launch_bounds__(1024) scan_kernel(const CompactParams p) {
     __shared__ int total[kMaxE + 1];
     const int nb = p.E + 1;
-    for (int e = threadIdx.x; e < nb; e += blockDim.x) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int e = warp; e < nb; e += 32) {
         int run = 0;
-        for (int b = 0; b < p.nblk; ++b) {
-            const int c = p.blk_counts[b * nb + e];
-            p.blk_base[b * nb + e] = run;
-            run += c;
+        for (int b0 = 0; b0 < p.nblk; b0 += 32) {
+            const int b = b0 + lane;
+            const int c = b < p.nblk ? p.blk_counts[b * nb + e] : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            if (b < p.nblk) p.blk_base[b * nb + e] = run + incl - c;
+            run += __shfl_sync(0xffffffffu, incl, 31);
         }
-        total[e] = run;
+        if (lane == 0) total[e] = run;
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        int acc = 0;
-        for (int e = 0; e < nb; ++e) {
-            p.goff[e] = acc;
-            acc += total[e];
-        }
-        p.goff[nb] = acc;
-        atomicAdd(&p.ctr->pairs_total, (unsigned long long)(acc - total[p.E]));
-        atomicAdd(&p.ctr->shared_rows, (unsigned long long)total[p.E]);
+    if (warp == 0) {
+        int base = 0;
         unsigned long long touched = 0;
-        for (int e = 0; e < p.E; ++e) touched += total[e] > 0 ? 1ull : 0ull;
-        atomicAdd(&p.ctr->experts_touched, touched);
-        if (total[p.E] > 0) atomicAdd(&p.ctr->shared_touched, 1ull);
+        for (int e0 = 0; e0 < nb; e0 += 32) {
+            const int e = e0 + lane;
+            const int c = e < nb ? total[e] : 0;
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            if (e < nb) p.goff[e] = base + incl - c;
+            touched += __popc(__ballot_sync(0xffffffffu, e < p.E && c > 0));
+            base += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        if (lane == 0) {
+            p.goff[nb] = base;
+            atomicAdd(&p.ctr->pairs_total, (unsigned long long)(base - total[p.E]));
+            atomicAdd(&p.ctr->shared_rows, (unsigned long long)total[p.E]);
+            atomicAdd(&p.ctr->experts_touched, touched);
+            if (total[p.E] > 0) atomicAdd(&p.ctr->shared_touched, 1ull);
+        }
     }
 }
 
-// One warp per chunk walks the chunk's pairs in (t, j) order, 32 at a time.
-__global__ void __launch_bounds__(32) scatter_kernel(const CompactParams p) {
-    __shared__ int run[kMaxE + 1];
-    const int lane = threadIdx.x;
+// One block per chunk, one warp per 32 consecutive tokens of it.  Each warp
+// counts its pairs per bucket, the block turns the counts into per-warp
+// starting positions (the chunk's base plus the earlier warps' counts), and
+// each warp then walks its pairs in (t, j) order, 32 at a time, ranking equal
+// buckets with __match_any_sync.
+constexpr int kScatWarps = kChunk / 32;
+
+__global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) {
+    __shared__ int run[kScatWarps][kMaxE + 1];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.E + 1;
-    for (int e = lane; e < nb; e += 32) run[e] = p.goff[e] + p.blk_base[blockIdx.x * nb + e];
-    __syncwarp();
-    const int t0 = blockIdx.x * kChunk;
-    const int tn = min(kChunk, p.T - t0);
+    for (int i = threadIdx.x; i < kScatWarps * nb; i += blockDim.x) run[i / nb][i % nb] = 0;
+    __syncthreads();
+    const int t0 = blockIdx.x * kChunk + warp * 32;
+    const int tn = max(0, min(32, p.T - t0));
     const unsigned lt_mask = (1u << lane) - 1u;
-    // Routed pairs.
     const int npairs = tn * p.k;
+    // Pass 1: this warp's count per bucket.
+    for (int q0 = 0; q0 < npairs; q0 += 32) {
+        const int q = q0 + lane;
+        int key = -1;
+        if (q < npairs) {
+            const int t = t0 + q / p.k;
+            if (p.action[t] == 0) key = p.exp_sel[t * p.k + (q - (q / p.k) * p.k)];
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, key);
+        if (key >= 0 && (peers & lt_mask) == 0) run[warp][key] += __popc(peers);
+    }
+    if (p.has_shared) {
+        const bool take = lane < tn && (p.action[t0 + lane] == 0 || p.action[t0 + lane] == 1);
+        const unsigned ball = __ballot_sync(0xffffffffu, take);
+        if (lane == 0) run[warp][p.E] = __popc(ball);
+    }
+    __syncthreads();
+    // Per-warp starting positions: exclusive prefix over the warps, per bucket.
+    for (int e = threadIdx.x; e < nb; e += blockDim.x) {
+        int acc = p.goff[e] + p.blk_base[blockIdx.x * nb + e];
+        for (int w = 0; w < kScatWarps; ++w) {
+            const int c = run[w][e];
+            run[w][e] = acc;
+            acc += c;
+        }
+    }
+    __syncthreads();
+    // Pass 2: routed pairs.
     for (int q0 = 0; q0 < npairs; q0 += 32) {
         const int q = q0 + lane;
         int key = -1, code = -1;
@@ -91,94 +145,81 @@ __global__ void __launch_bounds__(32) scatter_kernel(const CompactParams p) {
         }
         const unsigned peers = __match_any_sync(0xffffffffu, key);
         if (key >= 0) {
-            const int rank = __popc(peers & lt_mask);
-            const int pos = run[key] + rank;
+            const int pos = run[warp][key] + __popc(peers & lt_mask);
             p.perm[pos] = code;
             p.pos_pair[code] = pos;
         }
         __syncwarp();
-        if (key >= 0 && (peers & lt_mask) == 0) run[key] += __popc(peers);
+        if (key >= 0 && (peers & lt_mask) == 0) run[warp][key] += __popc(peers);
         __syncwarp();
     }
     // Shared-expert rows: executed or skipped tokens, by t.
-    if (p.has_shared) {
-        for (int q0 = 0; q0 < tn; q0 += 32) {
-            const int q = q0 + lane;
-            bool take = false;
-            int t = t0 + q;
-            if (q < tn) {
-                const int a = p.action[t];
-                take = (a == 0 || a == 1);
-                if (!take) p.pos_sh[t] = -1;
-            }
-            const unsigned ball = __ballot_sync(0xffffffffu, take);
-            if (take) {
-                const int pos = run[p.E] + __popc(ball & lt_mask);
-                p.perm[pos] = t;
-                p.pos_sh[t] = pos - p.goff[p.E];
-            }
-            __syncwarp();
-            if (lane == 0) run[p.E] += __popc(ball);
-            __syncwarp();
+    if (p.has_shared && tn > 0) {
+        const int t = t0 + lane;
+        bool take = false;
+        if (lane < tn) {
+            const int a = p.action[t];
+            take = (a == 0 || a == 1);
+            if (!take) p.pos_sh[t] = -1;
+        }
+        const unsigned ball = __ballot_sync(0xffffffffu, take);
+        if (take) {
+            const int pos = run[warp][p.E] + __popc(ball & lt_mask);
+            p.perm[pos] = t;
+            p.pos_sh[t] = pos - p.goff[p.E];
         }
     }
 }
 
 // Xp[row] = expert input of the row's token: bf16(h * r * gamma) with the
-// pre-FFN RMSNorm, or h itself without it; one warp per row.
+// pre-FFN RMSNorm, or h itself without it; one warp per row, gamma staged in
+// shared memory once per block, kGU chunks of 16 bytes per lane in flight.
+constexpr int kGU = 8;
+constexpr int kMaxGatherD = 16384;   // gamma staged in shared memory (32 KB)
+
 __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ goff, int E, int k,
                                                      int d, const __nv_bfloat16* __restrict__ h,
                                                      const float* __restrict__ rnorm,
                                                      const __nv_bfloat16* __restrict__ gamma,
                                                      __nv_bfloat16* __restrict__ Xp) {
+    extern __shared__ uint4 sg[];      // gamma, d / 8 chunks
     const int nrows = goff[E + 1];
     const int routed = goff[E];
     const int lane = threadIdx.x & 31;
     const int nchunk = d >> 3;
+    if (gamma) {
+        const uint4* gv4 = reinterpret_cast<const uint4*>(gamma);
+        for (int c = threadIdx.x; c < nchunk; c += blockDim.x) sg[c] = __ldg(gv4 + c);
+        __syncthreads();
+    }
     for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < nrows;
          r += (gridDim.x * blockDim.x) >> 5) {
         const int code = perm[r];
         const int t = r < routed ? code / k : code;
         const uint4* __restrict__ src = reinterpret_cast<const uint4*>(h + (size_t)t * d);
         uint4* __restrict__ dst = reinterpret_cast<uint4*>(Xp + (size_t)r * d);
-        // kU chunks of 16 bytes per lane in flight at a time.
-        constexpr int kU = 4;
-        if (!gamma) {
-            for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
-                uint4 v[kU];
+        const float rn = gamma ? rnorm[t] : 1.f;
+        for (int c0 = lane; c0 < nchunk; c0 += 32 * kGU) {
+            uint4 hv[kGU];
 #pragma unroll
-                for (int u = 0; u < kU; ++u)
-                    if (c0 + 32 * u < nchunk) v[u] = src[c0 + 32 * u];
+            for (int u = 0; u < kGU; ++u)
+                if (c0 + 32 * u < nchunk) hv[u] = src[c0 + 32 * u];
 #pragma unroll
-                for (int u = 0; u < kU; ++u)
-                    if (c0 + 32 * u < nchunk) dst[c0 + 32 * u] = v[u];
-            }
-            continue;
-        }
-        const float rn = rnorm[t];
-        const uint4* gv4 = reinterpret_cast<const uint4*>(gamma);
-        for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
-            uint4 hv[kU], gv[kU];
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
+            for (int u = 0; u < kGU; ++u) {
                 const int c = c0 + 32 * u;
-                if (c < nchunk) {
-                    hv[u] = src[c];
-                    gv[u] = __ldg(gv4 + c);
+                if (c >= nchunk) continue;
+                if (!gamma) {
+                    dst[c] = hv[u];
+                    continue;
                 }
-            }
-#pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                const int c = c0 + 32 * u;
-                if (c < nchunk) {
-                    uint4 o;
-                    o.x = pack_bf16x2(bf16_lo(hv[u].x) * rn * bf16_lo(gv[u].x), bf16_hi(hv[u].x) * rn * bf16_hi(gv[u].x));
-                    o.y = pack_bf16x2(bf16_lo(hv[u].y) * rn * bf16_lo(gv[u].y), bf16_hi(hv[u].y) * rn * bf16_hi(gv[u].y));
-                    o.z = pack_bf16x2(bf16_lo(hv[u].z) * rn * bf16_lo(gv[u].z), bf16_hi(hv[u].z) * rn * bf16_hi(gv[u].z));
-                    o.w = pack_bf16x2(bf16_lo(hv[u].w) * rn * bf16_lo(gv[u].w), bf16_hi(hv[u].w) * rn * bf16_hi(gv[u].w));
-                    dst[c] = o;
-                }
+                const uint4 gv = sg[c];
+                uint4 o;
+                o.x = pack_bf16x2(bf16_lo(hv[u].x) * rn * bf16_lo(gv.x), bf16_hi(hv[u].x) * rn * bf16_hi(gv.x));
+                o.y = pack_bf16x2(bf16_lo(hv[u].y) * rn * bf16_lo(gv.y), bf16_hi(hv[u].y) * rn * bf16_hi(gv.y));
+                o.z = pack_bf16x2(bf16_lo(hv[u].z) * rn * bf16_lo(gv.z), bf16_hi(hv[u].z) * rn * bf16_hi(gv.z));
+                o.w = pack_bf16x2(bf16_lo(hv[u].w) * rn * bf16_lo(gv.w), bf16_hi(hv[u].w) * rn * bf16_hi(gv.w));
+                dst[c] = o;
             }
         }
     }
@@ -189,8 +230,8 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
     count_kernel<<<p.nblk, kChunk, 0, st>>>(p);
-    scan_kernel<<<1, 256, 0, st>>>(p);
-    scatter_kernel<<<p.nblk, 32, 0, st>>>(p);
+    scan_kernel<<<1, 1024, 0, st>>>(p);
+    scatter_kernel<<<p.nblk, kChunk, 0, st>>>(p);
     return cudaGetLastError();
 }
 
@@ -198,9 +239,19 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
                           const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,
                           __nv_bfloat16* Xp, int max_rows, int num_sms, cudaStream_t st) {
     if (max_rows <= 0) return cudaSuccess;
+    if (d > kMaxGatherD) return cudaErrorInvalidValue;
+    const size_t smem = gamma ? (size_t)d * 2 : 0;
+    static int per_sm = 0;
+    if (per_sm == 0) {
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gather_kernel, 256, (size_t)kMaxGatherD * 2) !=
+                cudaSuccess || n < 1)
+            n = 1;
+        per_sm = n;
+    }
     int blocks = (max_rows + 7) / 8;
-    blocks = blocks < num_sms * 8 ? blocks : num_sms * 8;
-    gather_kernel<<<blocks, 256, 0, st>>>(perm, goff, E, k, d, h, rnorm, gamma, Xp);
+    blocks = blocks < num_sms * per_sm ? blocks : num_sms * per_sm;
+    gather_kernel<<<blocks, 256, smem, st>>>(perm, goff, E, k, d, h, rnorm, gamma, Xp);
     return cudaGetLastError();
 }
 

@@ -330,6 +330,7 @@ trimmoe_status validate_config(const trimmoe_config* c, std::string& why) {
     if (!(c->d_ref_ms > 0.f) || !std::isfinite(c->d_ref_ms)) { why = "config: d_ref_ms must be > 0"; return TRIMMOE_ERR_ARG; }
     if (!(c->norm_eps >= 0.f) || !std::isfinite(c->norm_eps)) { why = "config: norm_eps must be >= 0"; return TRIMMOE_ERR_ARG; }
     if (c->d % 256) { why = "config: d must be a multiple of 256"; return TRIMMOE_ERR_UNSUPPORTED; }
+    if (c->d > 16384) { why = "config: d > 16384"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->act == 1 && c->F % 128) { why = "config: SwiGLU F must be a multiple of 128"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->act == 0 && c->F % 256) { why = "config: ReLU F must be a multiple of 256"; return TRIMMOE_ERR_UNSUPPORTED; }
     if (c->F_sh % 128) { why = "config: F_sh must be a multiple of 128"; return TRIMMOE_ERR_UNSUPPORTED; }
