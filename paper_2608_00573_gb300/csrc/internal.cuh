@@ -26,7 +26,7 @@ constexpr size_t kMaxTabFloats = (size_t)16 << 20; // 64 MB of shared look-ahead
 constexpr int kGateUp = 128;        // W13 gate/up row interleave
 
 // Device error codes (first one wins).
-enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3 };
+enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3, ERR_TIMEOUT_ROUTER = 4 };
 
 // Device-side counters (trimmoe_stats_t is assembled from these).
 struct DevCounters {
@@ -56,7 +56,9 @@ struct DevTables {
 };
 
 // Router and exit-head partial logits of one layer (kernel a0), split over d:
-// block (x, y) covers tokens [64x, 64x+64) and columns [y*d/ksplit, (y+1)*d/ksplit).
+// unit (tile, y) covers tokens [128 tile, 128 tile + 128) and columns
+// [y*d/ksplit, (y+1)*d/ksplit); the hidden rows come through a tensor map
+// passed beside these parameters.
 struct RouterParams {
     int T, d;
     int n_out;                  // E + C logits per token
@@ -71,6 +73,7 @@ struct RouterParams {
     const __nv_bfloat16* Blo;   // [E][d] lo(gamma * W_r)
     float* zpart;               // [ksplit][T][zs] partial dot products
     float* sqpart;              // [ksplit][T] partial sums of h^2
+    int* err;                   // device error word (bounded waits)
 };
 
 struct DecideParams {
@@ -205,8 +208,10 @@ struct FeedbackParams {
 };
 
 // Launchers (one translation unit each).
-cudaError_t launch_router(const RouterParams& p, cudaStream_t st);
-size_t router_smem_bytes(int ng, int nl);
+// Tensor maps (64-column boxes, 128-byte swizzle): tmA the hidden rows [T][d]
+// in 128-row boxes, tmBhi / tmBlo the pass's weight rows in ng / nl-row boxes.
+cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, const CUtensorMap* tmBlo,
+                          const RouterParams& p, int num_sms, cudaStream_t st);
 int router_lo_rows(int n_lo, int ng);
 int router_pass_rows(int n_out);
 int router_ksplit(int T, int d, int num_sms);

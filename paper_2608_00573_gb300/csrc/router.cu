@@ -3,10 +3,10 @@
 //   z[t][e]     = r_t * sum_i h[t][i] * gamma_i * W_r[e][i] + b_r[e]     e < E   (Eq. 4 input)
 //   z[t][E + c] = r_t * sum_i h[t][i] * W_x[c][i]            + b_x[c]     c < C   (Eq. 7 input)
 // with r_t = 1/sqrt(mean_i h[t][i]^2 + eps) (1 without the pre-FFN RMSNorm).
-// The columns i are split into ksplit ranges, one per blockIdx.y, so that the
-// grid covers every SM several times even for small token counts; each block
-// writes its partial sums (and partial sums of h^2), and the decision kernel
-// adds the ranges in a fixed order before applying r and the bias.
+// The columns i are split into ksplit ranges; each (128-token tile, column
+// range) unit writes its partial sums (and partial sums of h^2), and the
+// decision kernel adds the ranges in a fixed order before applying r and the
+// bias.
 //
 // The router's gamma * W_r products are exact in fp32 and split exactly into
 // two bf16 matrices (hi + lo), so two bf16 MMAs give the logits without
@@ -14,155 +14,235 @@
 // and its partial is added to IEEE fp32 registers (__fadd_rn): the tensor
 // core's own accumulation then only touches sums of 16-32 exact products, which
 // keeps the logits at fp32 accuracy (the decisions compare them to 1e-5).
-// mma.sync m16n8k16 (bf16 in, fp32 accumulate): the contraction is tiny (E + C
-// outputs per token) and the kernel is bound by streaming h from HBM, so the
-// tensor cores only remove the per-element unpack/FMA instruction cost.
-// One block = 64 tokens (4 warps x 16), d streamed in 64-column slabs through
-// a 4-stage cp.async ring in padded shared memory, ldmatrix fragments; up to
-// 128 output rows per pass over h.
-// Dead tokens are zero-filled without reading HBM.
+// The sum of squares comes from the same fragments: two more MMAs per k step
+// multiply the 16-token A fragment by itself (its rows reused as the B
+// operand), and the diagonal of that 16 x 16 Gram block is each token's
+// partial sum of h^2.
+//
+// Design (persistent, 288 threads per CTA):
+//   warp 8      producer (one lane): per 64-column slab, 2-D TMA boxes of the
+//               128-token hidden tile and of the pass's weight rows (hi and
+//               lo), 128-byte swizzle, rows past the tensor zero-filled, into a
+//               ring of 2-8 stages guarded by full/empty mbarriers
+//   warps 0-7   16 tokens each: ldmatrix + mma.sync m16n8k16 (bf16 in, fp32
+//               accumulate), up to 128 output rows per pass over h
+// Hidden rows of dead tokens are loaded with their tile but never stored.
+// Every wait is bounded (2 s); on expiry the kernel records an error word and
+// returns.
+#include <algorithm>
+
 #include "internal.cuh"
 
 namespace tmoe {
 
 namespace {
 
-constexpr int kTok = 64;
-constexpr int kKS = 64;
-constexpr int kPad = 72;          // padded smem row (bf16): conflict-free ldmatrix
-constexpr int kStages = 4;
+constexpr int kTok = 128;         // tokens per tile (8 consumer warps x 16)
+constexpr int kKS = 64;           // columns per slab (one 128-byte row per token / weight)
 constexpr int kNG = 128;          // largest number of outputs per pass (16 n-tiles of 8)
+constexpr int kConsumers = kTok / 16;
+constexpr int kThreads = 32 * (kConsumers + 1);
+constexpr int kA = kTok * kKS * 2;     // 16 KB hidden slab, 128-byte swizzled
+constexpr int kMaxStages = 8;
 
-// NT: n-tiles of 8 outputs held in registers per pass (8 or 16).
+struct __align__(8) RouterBars {
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
+    int abort_flag;
+};
+
+// Stage: hidden slab, then ng weight rows (hi), then nl (lo), all dense
+// 128-byte rows with 128-byte swizzle (1024-byte aligned, ng and nl % 8 == 0).
+__host__ __device__ __forceinline__ size_t stage_bytes(int ng, int nl) {
+    return (size_t)kA + (size_t)(ng + nl) * kKS * 2;
+}
+
+// Shared memory per CTA: two CTAs per SM with up to 4 n-tiles per pass, one
+// with 8 or more (the accumulators need the registers of the whole SM).
+size_t smem_budget(int nt) { return nt <= 4 ? 100 * 1024 : 200 * 1024; }
+
+int stages_for(int ng, int nl, int nt) {
+    const size_t sb = stage_bytes(ng, nl);
+    const int s = (int)((smem_budget(nt) - 1024 - sizeof(RouterBars)) / sb);
+    return std::max(2, std::min(kMaxStages, s));
+}
+
+size_t smem_for(int ng, int nl, int stages) {
+    return 1024 + (size_t)stages * stage_bytes(ng, nl) + sizeof(RouterBars);
+}
+
+// Address of 16-byte chunk c of row r in a 128-byte-swizzled tile.
+__device__ __forceinline__ uint32_t sw128(uint32_t base, int r, int c) {
+    return base + (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// NT: n-tiles of 8 outputs per pass (ng = 8 NT rows, the last ones past n_out
+// zero-filled by TMA and never stored).
 template <int NT>
-__global__ void __launch_bounds__(128) router_kernel(const RouterParams p) {
-    extern __shared__ __align__(16) uint8_t sm[];
-    const int NG = p.ng;                       // padded rows per pass (<= kNG, multiple of 8)
-    const int NL = p.nl;                       // padded rows with a lo part (<= NG)
-    __nv_bfloat16* sA = reinterpret_cast<__nv_bfloat16*>(sm);
-    __nv_bfloat16* sBh = sA + kStages * kTok * kPad;
-    __nv_bfloat16* sBl = sBh + kStages * NG * kPad;
-    __shared__ float ssq[kTok];
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int t0 = blockIdx.x * kTok;
-    const int nslab_all = p.d / kKS;
-    const int nslab = nslab_all / p.ksplit;
-    const int slab0 = blockIdx.y * nslab;
-    float* zpart = p.zpart + (size_t)blockIdx.y * p.T * p.zs;
-    float* sqpart = p.sqpart + (size_t)blockIdx.y * p.T;
-    const int g = lane >> 2, tig = lane & 3;
+__global__ void __launch_bounds__(kThreads, NT <= 4 ? 2 : 1)
+router_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmBhi,
+              const __grid_constant__ CUtensorMap tmBlo, const RouterParams p, int stages) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+    const int NG = p.ng, NL = p.nl;
+    const size_t sbytes = stage_bytes(NG, NL);
+    RouterBars* bars = reinterpret_cast<RouterBars*>(smem + (size_t)stages * sbytes);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    for (int ng0 = 0; ng0 < p.n_out; ng0 += NG) {
-        const int nrows = min(NG, p.n_out - ng0);
-        const int ntile = (nrows + 7) >> 3;
-        const bool any_lo = ng0 < p.n_lo;
-        float sq = 0.f;
-        float acc[NT][4];
-#pragma unroll
-        for (int j = 0; j < NT; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+    const int nslab = p.d / kKS / p.ksplit;
+    const int ntile = (p.T + kTok - 1) / kTok;
+    const int npass = (p.n_out + NG - 1) / NG;
+    const int nunits = ntile * p.ksplit * npass;   // unit u: pass u / (ntile*ksplit), then tile, then range
 
-        auto load_slab = [&](int s) {
-            const int buf = s % kStages;
-            const int sg = slab0 + s;                 // global slab index
-            for (int i = tid; i < kTok * (kKS / 8); i += 128) {
-                const int r = i >> 3, c = i & 7;
-                const int t = t0 + r;
-                const bool ok = t < p.T && p.alive[t];
-                const __nv_bfloat16* src = p.h + (size_t)(ok ? t : 0) * p.d + sg * kKS + c * 8;
-                cp_async16(smem_u32(sA + (buf * kTok + r) * kPad + c * 8), src, ok ? 16 : 0);
-            }
-            for (int i = tid; i < NG * (kKS / 8); i += 128) {
-                const int r = i >> 3, c = i & 7;
-                const bool ok = r < nrows;
-                const size_t off = (size_t)(ng0 + (ok ? r : 0)) * p.d + sg * kKS + c * 8;
-                cp_async16(smem_u32(sBh + (buf * NG + r) * kPad + c * 8), p.Bhi + off, ok ? 16 : 0);
-                if (any_lo && r < NL) {
-                    const bool okl = ok && (ng0 + r) < p.n_lo;
-                    cp_async16(smem_u32(sBl + (buf * NL + r) * kPad + c * 8), p.Blo + off, okl ? 16 : 0);
-                }
-            }
-        };
-
-        for (int s = 0; s < kStages - 1; ++s) {
-            if (s < nslab) load_slab(s);
-            cp_async_commit();
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < stages; ++s) {
+            mbar_init(smem_u32(&bars->full[s]), 1);
+            mbar_init(smem_u32(&bars->empty[s]), kConsumers);
         }
-        for (int s = 0; s < nslab; ++s) {
-            cp_async_wait<kStages - 2>();
-            __syncthreads();
-            if (s + kStages - 1 < nslab) load_slab(s + kStages - 1);
-            cp_async_commit();
-            const int buf = s % kStages;
-            const __nv_bfloat16* A = sA + buf * kTok * kPad;
-            if (ng0 == 0) {                     // sum of squares for the RMS factor
-                const __nv_bfloat16* row = A + (tid >> 1) * kPad + (tid & 1) * 32;
-#pragma unroll
-                for (int q = 0; q < 32; q += 8) {
-                    const uint4 v = *reinterpret_cast<const uint4*>(row + q);
-                    const float f[8] = {bf16_lo(v.x), bf16_hi(v.x), bf16_lo(v.y), bf16_hi(v.y),
-                                        bf16_lo(v.z), bf16_hi(v.z), bf16_lo(v.w), bf16_hi(v.w)};
-#pragma unroll
-                    for (int u = 0; u < 8; ++u) sq = fmaf(f[u], f[u], sq);
+        bars->abort_flag = 0;
+        fence_barrier_init();
+        prefetch_tmap(&tmA);
+        prefetch_tmap(&tmBhi);
+        if (NL > 0) prefetch_tmap(&tmBlo);
+    }
+    __syncthreads();
+    volatile int* abort_flag = &bars->abort_flag;
+
+    if (warp == kConsumers) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            int it = 0;
+            for (int u = blockIdx.x; u < nunits && !*abort_flag; u += gridDim.x) {
+                const int pass = u / (ntile * p.ksplit);
+                const int rem = u - pass * ntile * p.ksplit;
+                const int tile = rem / p.ksplit;
+                const int kr = rem - tile * p.ksplit;
+                const int ng0 = pass * NG;
+                const bool lo = ng0 < p.n_lo && NL > 0;
+                const uint32_t tx = (uint32_t)kA + (uint32_t)(NG + (lo ? NL : 0)) * (kKS * 2);
+                bool ok = true;
+                for (int sl = 0; sl < nslab; ++sl, ++it) {
+                    const int s = it % stages;
+                    const uint32_t ph = (it / stages) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&bars->empty[s]), ph ^ 1, abort_flag, p.err, ERR_TIMEOUT_ROUTER)) {
+                        ok = false;
+                        break;
+                    }
+                    const int col = (kr * nslab + sl) * kKS;
+                    const uint32_t fb = smem_u32(&bars->full[s]);
+                    const uint32_t st0 = smem_u32(smem + (size_t)s * sbytes);
+                    mbar_arrive_expect_tx(fb, tx);
+                    tma_load_2d(st0, &tmA, col, tile * kTok, fb);
+                    tma_load_2d(st0 + kA, &tmBhi, col, ng0, fb);
+                    if (lo) tma_load_2d(st0 + kA + NG * kKS * 2, &tmBlo, col, ng0, fb);
                 }
+                if (!ok) break;
             }
+        }
+    } else {
+        // ------------------------------------------------------------ consumers
+        const int g = lane >> 2, tig = lane & 3;
+        // Lane (g, g / 2) holds tokens g and 8 + g of the Gram diagonal.
+        const bool diag = (tig == (g >> 1));
+        const int dq = g & 1;
+        // Per-lane ldmatrix offsets in the 128-byte-swizzled tiles, one per k step.
+        const int ar = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+        const int br = lane & 7;
+        uint32_t a_off[kKS / 16], b_off[kKS / 16];
 #pragma unroll
-            for (int kk = 0; kk < kKS / 16; ++kk) {
-                uint32_t a[4];
-                const int ar = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-                const int ac = kk * 16 + (lane >> 4) * 8;
-                ldmatrix_x4(a, smem_u32(A + ar * kPad + ac));
-                const int br = (lane & 7);
-                const int bc = kk * 16 + ((lane >> 3) & 1) * 8;
+        for (int kk = 0; kk < kKS / 16; ++kk) {
+            a_off[kk] = (uint32_t)(ar * 128 + (((kk * 2 + (lane >> 4)) ^ (ar & 7)) << 4));
+            b_off[kk] = (uint32_t)(br * 128 + (((kk * 2 + ((lane >> 3) & 1)) ^ br) << 4));
+        }
+        const int nlt = NL / 8;                 // n-tiles with a lo part (pass 0)
+        int it = 0;
+        for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+            const int pass = u / (ntile * p.ksplit);
+            const int rem = u - pass * ntile * p.ksplit;
+            const int tile = rem / p.ksplit;
+            const int kr = rem - tile * p.ksplit;
+            const int ng0 = pass * NG;
+            const int nrows = min(NG, p.n_out - ng0);
+            const int lo_t = (pass == 0 && ng0 < p.n_lo) ? nlt : 0;
+            float acc[NT][4];
+#pragma unroll
+            for (int j = 0; j < NT; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+            float sq0 = 0.f, sq1 = 0.f;
+            // Liveness of this lane's two output rows, loaded now so that the
+            // stores after the last slab do not wait on it.
+            const int t_lo = tile * kTok + warp * 16 + g, t_hi = t_lo + 8;
+            const bool st_lo = t_lo < p.T && p.alive[t_lo];
+            const bool st_hi = t_hi < p.T && p.alive[t_hi];
+            bool ok = true;
+            for (int sl = 0; sl < nslab; ++sl, ++it) {
+                const int s = it % stages;
+                const uint32_t ph = (it / stages) & 1;
+                int w = 1;
+                if (lane == 0) w = mbar_wait_bounded(smem_u32(&bars->full[s]), ph, abort_flag, p.err, ERR_TIMEOUT_ROUTER);
+                w = __shfl_sync(0xffffffffu, w, 0);
+                if (!w) { ok = false; break; }
+                const uint32_t sA = smem_u32(smem + (size_t)s * sbytes);
+                const uint32_t sBh = sA + kA;
+                const uint32_t sBl = sBh + NG * kKS * 2;
+                // One slab: the tensor core sums its 64 (hi) + 64 (lo) exact
+                // products per output; the slab sums are then added in IEEE fp32.
+                float part[NT][4];
+#pragma unroll
+                for (int j = 0; j < NT; ++j) part[j][0] = part[j][1] = part[j][2] = part[j][3] = 0.f;
+                float g0[4] = {0.f, 0.f, 0.f, 0.f}, g1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int kk = 0; kk < kKS / 16; ++kk) {
+                    uint32_t a[4];
+                    ldmatrix_x4(a, sA + a_off[kk]);
+#pragma unroll
+                    for (int j = 0; j < NT; ++j) {
+                        uint32_t b[2];
+                        ldmatrix_x2(b, sBh + j * 1024 + b_off[kk]);
+                        mma_bf16_16816(part[j], a, b);
+                        if (j < lo_t) {
+                            ldmatrix_x2(b, sBl + j * 1024 + b_off[kk]);
+                            mma_bf16_16816(part[j], a, b);
+                        }
+                    }
+                    if (pass == 0) {
+                        // Gram blocks: tokens 0-7 and 8-15 of the fragment as B.
+                        const uint32_t b0[2] = {a[0], a[2]}, b1[2] = {a[1], a[3]};
+                        mma_bf16_16816(g0, a, b0);
+                        mma_bf16_16816(g1, a, b1);
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&bars->empty[s]));
+#pragma unroll
+                for (int j = 0; j < NT; ++j)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) acc[j][q] = __fadd_rn(acc[j][q], part[j][q]);
+                sq0 = __fadd_rn(sq0, dq ? g0[1] : g0[0]);
+                sq1 = __fadd_rn(sq1, dq ? g1[3] : g1[2]);
+            }
+            if (!ok) break;
+            float* zpart = p.zpart + (size_t)kr * p.T * p.zs;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const int t = half ? t_hi : t_lo;
+                if (!(half ? st_hi : st_lo)) continue;
+                if (pass == 0 && diag) p.sqpart[(size_t)kr * p.T + t] = half ? sq1 : sq0;
+                float* zrow = zpart + (size_t)t * p.zs;
 #pragma unroll
                 for (int j = 0; j < NT; ++j) {
-                    if (j < ntile) {
-                        uint32_t b[2];
-                        float part[4] = {0.f, 0.f, 0.f, 0.f};
-                        ldmatrix_x2(b, smem_u32(sBh + (buf * NG + j * 8 + br) * kPad + bc));
-                        mma_bf16_16816(part, a, b);
-                        if (ng0 + j * 8 < p.n_lo) {
-                            ldmatrix_x2(b, smem_u32(sBl + (buf * NL + j * 8 + br) * kPad + bc));
-                            mma_bf16_16816(part, a, b);
-                        }
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) acc[j][q] = __fadd_rn(acc[j][q], part[q]);
-                    }
-                }
-            }
-        }
-        cp_async_wait<0>();
-        if (ng0 == 0) {
-            sq += __shfl_xor_sync(0xffffffffu, sq, 1);
-            if ((tid & 1) == 0) ssq[tid >> 1] = sq;
-        }
-        __syncthreads();
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            const int r = warp * 16 + g + half * 8;
-            const int t = t0 + r;
-            if (t >= p.T || !p.alive[t]) continue;
-            if (ng0 == 0 && tig == 0) sqpart[t] = ssq[r];
-            float* zrow = zpart + (size_t)t * p.zs;
-#pragma unroll
-            for (int j = 0; j < NT; ++j) {
-                if (j < ntile) {
 #pragma unroll
                     for (int q = 0; q < 2; ++q) {
-                        const int col = ng0 + j * 8 + tig * 2 + q;
-                        if (col < p.n_out) zrow[col] = acc[j][half * 2 + q];
+                        const int col = j * 8 + tig * 2 + q;
+                        if (col < nrows) zrow[ng0 + col] = acc[j][half * 2 + q];
                     }
                 }
             }
         }
-        __syncthreads();
     }
 }
 
 }  // namespace
-
-size_t router_smem_bytes(int ng, int nl) {
-    return (size_t)kStages * (kTok + ng + nl) * kPad * sizeof(__nv_bfloat16);
-}
 
 int router_lo_rows(int n_lo, int ng) {
     const int r = ((n_lo + 7) / 8) * 8;
@@ -170,37 +250,63 @@ int router_lo_rows(int n_lo, int ng) {
 }
 
 // Column ranges per launch: a power of two dividing d/64, chosen so that the
-// grid has at least about four blocks per SM.
+// persistent grid has at least about eight units per SM.
 int router_ksplit(int T, int d, int num_sms) {
     const int nslab = d / kKS;
     const int tiles = (T + kTok - 1) / kTok;
     int ks = 1;
-    while (ks < nslab && (long long)tiles * ks < 4ll * num_sms && nslab % (ks * 2) == 0) ks *= 2;
+    while (ks < nslab && (long long)tiles * ks < 8ll * num_sms && nslab % (ks * 2) == 0) ks *= 2;
     return ks;
 }
 
+// Rows per pass: n-tiles of 8 rounded up to 1, 2, 4, 8, 12 or 16 (the kernel's
+// register tile), at most 128.
 int router_pass_rows(int n_out) {
-    const int r = ((n_out + 7) / 8) * 8;
-    return r < kNG ? r : kNG;
+    const int t = (n_out + 7) / 8;
+    const int nt = t <= 1 ? 1 : t <= 2 ? 2 : t <= 4 ? 4 : t <= 8 ? 8 : t <= 12 ? 12 : 16;
+    return nt * 8;
 }
 
-cudaError_t launch_router(const RouterParams& p, cudaStream_t st) {
+cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, const CUtensorMap* tmBlo,
+                          const RouterParams& p, int num_sms, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    if (p.d % kKS || p.ksplit < 1 || (p.d / kKS) % p.ksplit) return cudaErrorInvalidValue;
-    const size_t smem = router_smem_bytes(p.ng, p.nl);
+    if (p.d % kKS || p.ksplit < 1 || (p.d / kKS) % p.ksplit || p.ng < 8 || p.ng > kNG || p.ng % 8 ||
+        p.nl < 0 || p.nl > p.ng || p.nl % 8 || !tmA || !tmBhi || (p.nl > 0 && !tmBlo))
+        return cudaErrorInvalidValue;
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(router_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)router_smem_bytes(kNG, kNG));
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(router_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)router_smem_bytes(kNG, kNG));
+        cudaError_t e = cudaSuccess;
+        auto set = [&](const void* f, int nt) {
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_budget(nt));
+        };
+        set((const void*)router_kernel<1>, 1);
+        set((const void*)router_kernel<2>, 2);
+        set((const void*)router_kernel<4>, 4);
+        set((const void*)router_kernel<8>, 8);
+        set((const void*)router_kernel<12>, 12);
+        set((const void*)router_kernel<16>, 16);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    const dim3 grid((p.T + kTok - 1) / kTok, p.ksplit);
-    if (p.ng <= 64) router_kernel<8><<<grid, 128, smem, st>>>(p);
-    else router_kernel<16><<<grid, 128, smem, st>>>(p);
+    const int nt = p.ng / 8;
+    if (nt != 1 && nt != 2 && nt != 4 && nt != 8 && nt != 12 && nt != 16) return cudaErrorInvalidValue;
+    const int stages = stages_for(p.ng, p.nl, nt);
+    const size_t smem = smem_for(p.ng, p.nl, stages);
+    const int ntile = (p.T + kTok - 1) / kTok;
+    const int npass = (p.n_out + p.ng - 1) / p.ng;
+    const long long units = (long long)ntile * p.ksplit * npass;
+    const int per_sm = nt <= 4 ? 2 : 1;
+    const int grid = (int)std::min<long long>(units, (long long)per_sm * num_sms);
+    const CUtensorMap* lo = p.nl > 0 ? tmBlo : tmBhi;
+    switch (nt) {
+        case 1: router_kernel<1><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+        case 2: router_kernel<2><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+        case 4: router_kernel<4><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+        case 8: router_kernel<8><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+        case 12: router_kernel<12><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+        default: router_kernel<16><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+    }
     return cudaGetLastError();
 }
 

@@ -183,6 +183,9 @@ struct trimmoe {
     float* sqbuf_x = nullptr;         // [rows_part] partial sums of squares of the layer input
     CUtensorMap tmAttn;
     std::vector<CUtensorMap> tmWqkv, tmWo, tmWqkvp, tmWop;
+    // router weight rows per layer (64-column boxes): hi and lo of the router
+    // pass, and the exit-head / centroid rows read from the layer input (full block)
+    std::vector<CUtensorMap> tmRhi, tmRlo, tmRxhi;
     double flops_attn = 0.0, flops_attn_gemm = 0.0;
 
     // host-buffer forward
@@ -687,6 +690,24 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
                  make_tmap(&h->tmWqkvp[l], Wqkv + (size_t)l * h->nqkv * d, d, (uint64_t)h->nqkv, 128) &&
                  make_tmap(&h->tmWop[l], Wo + (size_t)l * d * hd, hd, (uint64_t)d, 128);
     }
+    if (tm) {
+        // Router weights: with the attention sublayer the router rows and the
+        // exit-head / centroid rows are read in separate passes over different
+        // inputs, so they get separate maps (boxes of one pass's rows).
+        h->tmRhi.resize(N);
+        h->tmRlo.resize(N);
+        if (has_attn) h->tmRxhi.resize(N);
+        const int n_main = has_attn ? E : n_out;
+        const int ng = router_pass_rows(n_main);
+        const int nl = router_lo_rows(E, ng);
+        for (int l = 0; l < N && tm; ++l) {
+            tm = make_tmap(&h->tmRhi[l], h->rt_hi + (size_t)l * n_out * d, d, (uint64_t)n_main, (uint32_t)ng) &&
+                 make_tmap(&h->tmRlo[l], h->rt_lo + (size_t)l * E * d, d, (uint64_t)E, (uint32_t)nl);
+            if (tm && has_attn)
+                tm = make_tmap(&h->tmRxhi[l], h->rt_hi + ((size_t)l * n_out + E) * d, d, (uint64_t)(n_out - E),
+                               (uint32_t)router_pass_rows(n_out - E));
+        }
+    }
     if (!tm) return bail(TRIMMOE_ERR_CUDA, "create: cuTensorMapEncodeTiled failed");
     *out = h;
     return TRIMMOE_OK;
@@ -819,6 +840,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     rp.Blo = h->rt_lo + (size_t)layer * E * d;
     rp.zpart = h->zbuf;
     rp.sqpart = h->sqbuf;
+    rp.err = h->dev_err;
     // With the attention sublayer the router rows read h_mid while the exit-head
     // and centroid rows read the state entering the layer: two passes.
     RouterParams rx = rp;
@@ -835,9 +857,15 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         rx.zpart = h->zbuf + E;
         rx.sqpart = h->sqbuf_x;
     }
+    // Hidden rows for the router's TMA loads (128-token x 64-column boxes).
+    CUtensorMap tm_h, tm_hx;
+    if (T > 0 && (!make_tmap(&tm_h, rp.h, d, T, 128) || (has_attn && !make_tmap(&tm_hx, rx.h, d, T, 128))))
+        return h->fail(TRIMMOE_ERR_CUDA, "router: cuTensorMapEncodeTiled failed");
     e = h->timed(K_ROUTER, st, [&] {
-        cudaError_t e2 = launch_router(rp, st);
-        return (e2 == cudaSuccess && has_attn) ? launch_router(rx, st) : e2;
+        cudaError_t e2 = launch_router(&tm_h, &h->tmRhi[layer], &h->tmRlo[layer], rp, h->num_sms, st);
+        return (e2 == cudaSuccess && has_attn)
+                   ? launch_router(&tm_hx, &h->tmRxhi[layer], nullptr, rx, h->num_sms, st)
+                   : e2;
     });
     if (has_attn) h->launches += 1;
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("router: ") + cudaGetErrorString(e));
