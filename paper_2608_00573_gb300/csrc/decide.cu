@@ -139,12 +139,12 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
         float rn = 1.f;
         if (p.use_norm) {
             float sq = 0.f;
-            for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart[(size_t)ks * p.T + t]);
+            for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart[(size_t)t * p.ksplit + ks]);
             rn = rsqrtf(sq / (float)p.d + p.norm_eps);
             if (lane == 0) p.rnorm[t] = rn;
         }
-        const size_t kstride = (size_t)p.T * p.zs;
-        const float* zrow = p.zpart + (size_t)t * p.zs;
+        const size_t kstride = (size_t)p.zs;      // the column ranges of a token are contiguous
+        const float* zrow = p.zpart + (size_t)t * p.ksplit * p.zs;
         for (int e = lane; e < E; e += 32) {
             float acc = 0.f;
             for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + e]);
@@ -189,7 +189,7 @@ __global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams 
             float rx = rn;
             if (p.use_norm && p.sqpart_x) {
                 float sq = 0.f;
-                for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart_x[(size_t)ks * p.T + t]);
+                for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart_x[(size_t)t * p.ksplit + ks]);
                 rx = rsqrtf(sq / (float)p.d + p.norm_eps);
             }
             for (int c = lane; c < C; c += 32) {

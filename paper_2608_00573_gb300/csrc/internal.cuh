@@ -71,17 +71,17 @@ struct RouterParams {
     const uint8_t* alive;
     const __nv_bfloat16* Bhi;   // [n_out][d] hi(gamma * W_r) then W_x of the previous layer
     const __nv_bfloat16* Blo;   // [E][d] lo(gamma * W_r)
-    float* zpart;               // [ksplit][T][zs] partial dot products
-    float* sqpart;              // [ksplit][T] partial sums of h^2
+    float* zpart;               // [T][ksplit][zs] partial dot products
+    float* sqpart;              // [T][ksplit] partial sums of h^2
     int* err;                   // device error word (bounded waits)
 };
 
 struct DecideParams {
     int layer, T, N, d, E, k, C, M, H;
     float omega_T, omega_D, d_ref;
-    const float* zpart;         // [ksplit][T][zs] partial router then exit-head dot products
-    const float* sqpart;        // [ksplit][T] partial sums of h^2
-    const float* sqpart_x;      // [ksplit][T] partial sums of the exit head's input^2 (NULL: sqpart)
+    const float* zpart;         // [T][ksplit][zs] partial router then exit-head dot products
+    const float* sqpart;        // [T][ksplit] partial sums of h^2
+    const float* sqpart_x;      // [T][ksplit] partial sums of the exit head's input^2 (NULL: sqpart)
     const float* bias;          // [E + C] router then exit-head biases of this layer
     int zs, ksplit;
     int use_norm;

@@ -4,7 +4,8 @@
 //   z[t][E + c] = r_t * sum_i h[t][i] * W_x[c][i]            + b_x[c]     c < C   (Eq. 7 input)
 // with r_t = 1/sqrt(mean_i h[t][i]^2 + eps) (1 without the pre-FFN RMSNorm).
 // The columns i are split into ksplit ranges; each (128-token tile, column
-// range) unit writes its partial sums (and partial sums of h^2), and the
+// range) unit writes its partial sums (and partial sums of h^2; a token's
+// ranges are contiguous: [T][ksplit][zs]), and the
 // decision kernel adds the ranges in a fixed order before applying r and the
 // bias.
 //
@@ -222,13 +223,12 @@ router_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
                 sq1 = __fadd_rn(sq1, dq ? g1[3] : g1[2]);
             }
             if (!ok) break;
-            float* zpart = p.zpart + (size_t)kr * p.T * p.zs;
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
                 const int t = half ? t_hi : t_lo;
                 if (!(half ? st_hi : st_lo)) continue;
-                if (pass == 0 && diag) p.sqpart[(size_t)kr * p.T + t] = half ? sq1 : sq0;
-                float* zrow = zpart + (size_t)t * p.zs;
+                if (pass == 0 && diag) p.sqpart[(size_t)t * p.ksplit + kr] = half ? sq1 : sq0;
+                float* zrow = p.zpart + ((size_t)t * p.ksplit + kr) * p.zs;
 #pragma unroll
                 for (int j = 0; j < NT; ++j) {
 #pragma unroll
