@@ -79,7 +79,7 @@ struct WarpCounters {
     float max_ratio;
 };
 
-__global__ void __launch_bounds__(kWarps * 32) decide_kernel(const DecideParams p) {
+__global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecideParams p) {
     extern __shared__ float smem[];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
