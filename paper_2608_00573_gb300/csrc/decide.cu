@@ -1,5 +1,6 @@
 // Kernel (a): exit gate + skip test + substitute-or-fetch with server argmin and
-// look-ahead + state update, one warp per live token.
+// look-ahead + state update, one group of 8, 16 or 32 lanes per live token (the
+// smallest group with a lane per expert).
 //
 // Paper: Sec. V, the per-token body of Algorithm 2.  Router and importance: Eq. (4);
 // exit confidence: Eq. (7)-(9); skip admission: Eq. (5), (34), (35); per-step
@@ -29,37 +30,41 @@ namespace {
 constexpr int kWarps = 4;
 #define kInf __int_as_float(0x7f800000)
 
-__device__ __forceinline__ float warp_sum(float v) {
+// Reductions over the G lanes of one token's group (mask gmask); arg-reductions
+// break ties to the lower index.
+template <int G>
+__device__ __forceinline__ float grp_sum(unsigned gmask, float v) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(gmask, v, o);
     return v;
 }
-__device__ __forceinline__ float warp_max(float v) {
+template <int G>
+__device__ __forceinline__ float grp_max(unsigned gmask, float v) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    for (int o = G / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(gmask, v, o));
     return v;
 }
-__device__ __forceinline__ float warp_min(float v) {
+template <int G>
+__device__ __forceinline__ float grp_min(unsigned gmask, float v) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    for (int o = G / 2; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(gmask, v, o));
     return v;
 }
-
-// (value, index) argmin over the warp; ties go to the lower index.
-__device__ __forceinline__ void warp_argmin(float& v, int& i) {
+template <int G>
+__device__ __forceinline__ void grp_argmin(unsigned gmask, float& v, int& i) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        float ov = __shfl_xor_sync(0xffffffffu, v, o);
-        int oi = __shfl_xor_sync(0xffffffffu, i, o);
+    for (int o = G / 2; o > 0; o >>= 1) {
+        float ov = __shfl_xor_sync(gmask, v, o);
+        int oi = __shfl_xor_sync(gmask, i, o);
         if (ov < v || (ov == v && oi < i)) { v = ov; i = oi; }
     }
 }
-// (value, index) argmax; ties go to the lower index.
-__device__ __forceinline__ void warp_argmax(float& v, int& i) {
+template <int G>
+__device__ __forceinline__ void grp_argmax(unsigned gmask, float& v, int& i) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        float ov = __shfl_xor_sync(0xffffffffu, v, o);
-        int oi = __shfl_xor_sync(0xffffffffu, i, o);
+    for (int o = G / 2; o > 0; o >>= 1) {
+        float ov = __shfl_xor_sync(gmask, v, o);
+        int oi = __shfl_xor_sync(gmask, i, o);
         if (ov > v || (ov == v && oi < i)) { v = ov; i = oi; }
     }
 }
@@ -79,17 +84,25 @@ struct WarpCounters {
     float max_ratio;
 };
 
+// G lanes per token (8, 16 or 32): a warp decides 32 / G tokens at once.  With
+// E <= G every per-expert value sits in its own lane, so the reduction trees
+// over experts are those of a full warp with the unused lanes at zero.
+template <int G>
 __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecideParams p) {
     extern __shared__ float smem[];
-    const int lane = threadIdx.x & 31;
+    const int lane = threadIdx.x & (G - 1);          // lane within the token's group
     const int warp = threadIdx.x >> 5;
+    const int grp = (threadIdx.x & 31) / G;
+    const unsigned gmask = G == 32 ? 0xffffffffu : (((1u << G) - 1u) << (grp * G));
+    constexpr int kGroups = kWarps * (32 / G);      // tokens in flight per block
+    const int slot = warp * (32 / G) + grp;
     const int E = p.E, M = p.M, C = p.C, K = p.k, l = p.layer;
     const int ME = M * E;
     const int MC = p.tab.max_layer_cand;
-    // Per-warp scratch: logits z[E], probabilities pr[E], head logits x[C],
+    // Per-group scratch: logits z[E], probabilities pr[E], head logits x[C],
     // look-ahead tables V[M*E] and Phi[M*E], staged candidate terms.
     const size_t per_warp = (size_t)(2 * E + C + 2 * ME + 2 * MC) + (size_t)((MC + 3) / 4) * 2;
-    float* zs = smem + (size_t)warp * per_warp;
+    float* zs = smem + (size_t)slot * per_warp;
     float* ps = zs + E;
     float* xs = ps + E;
     float* bufV = xs + C;
@@ -110,8 +123,8 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
     const float* ct_l = p.tab.ctab + (size_t)l * M * M;
 
     WarpCounters wc = {};
-    const int nwarps = gridDim.x * kWarps;
-    for (int t = blockIdx.x * kWarps + warp; t < p.T; t += nwarps) {
+    const int ngroups = gridDim.x * kGroups;
+    for (int t = blockIdx.x * kGroups + slot; t < p.T; t += ngroups) {
         if (!p.alive[t]) {
             if (lane == 0) {
                 p.action[t] = 3;
@@ -145,37 +158,37 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
         }
         const size_t kstride = (size_t)p.zs;      // the column ranges of a token are contiguous
         const float* zrow = p.zpart + (size_t)t * p.ksplit * p.zs;
-        for (int e = lane; e < E; e += 32) {
+        for (int e = lane; e < E; e += G) {
             float acc = 0.f;
             for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + e]);
             const float v = __fadd_rn(__fmul_rn(acc, rn), p.bias[e]);
             zs[e] = (v != v) ? -kInf : v;
         }
-        __syncwarp();
+        __syncwarp(gmask);
         float zmax = -FLT_MAX;
-        for (int e = lane; e < E; e += 32) zmax = fmaxf(zmax, zs[e]);
-        zmax = warp_max(zmax);
+        for (int e = lane; e < E; e += G) zmax = fmaxf(zmax, zs[e]);
+        zmax = grp_max<G>(gmask, zmax);
         float S = 0.f;
-        for (int e = lane; e < E; e += 32) {
+        for (int e = lane; e < E; e += G) {
             const float ex = expf(zs[e] - zmax);
             ps[e] = ex;
             S += ex;
         }
-        S = warp_sum(S);
-        __syncwarp();
-        for (int e = lane; e < E; e += 32) ps[e] = __fdiv_rn(ps[e], S);
-        __syncwarp();
+        S = grp_sum<G>(gmask, S);
+        __syncwarp(gmask);
+        for (int e = lane; e < E; e += G) ps[e] = __fdiv_rn(ps[e], S);
+        __syncwarp(gmask);
         int topk[kMaxK];
         float g[kMaxK];
-        unsigned used = 0u;   // bit i: expert lane + 32 i taken
+        unsigned used = 0u;   // bit i: expert lane + G i taken
         for (int j = 0; j < K; ++j) {
             float bz = -kInf;
             int be = 0x7fffffff;
-            for (int i = 0, e = lane; e < E; ++i, e += 32)
+            for (int i = 0, e = lane; e < E; ++i, e += G)
                 if (!((used >> i) & 1u) && (zs[e] > bz || (zs[e] == bz && e < be))) { bz = zs[e]; be = e; }
-            warp_argmax(bz, be);
+            grp_argmax<G>(gmask, bz, be);
             topk[j] = be;
-            if ((be & 31) == lane) used |= 1u << (be >> 5);
+            if ((be % G) == lane) used |= 1u << (be / G);
         }
         float I = 0.f;
         for (int j = 0; j < K; ++j) { g[j] = ps[topk[j]]; I = __fadd_rn(I, g[j]); }
@@ -192,21 +205,21 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
                 for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart_x[(size_t)t * p.ksplit + ks]);
                 rx = rsqrtf(sq / (float)p.d + p.norm_eps);
             }
-            for (int c = lane; c < C; c += 32) {
+            for (int c = lane; c < C; c += G) {
                 float acc = 0.f;
                 for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + c]);
                 xs[c] = __fadd_rn(__fmul_rn(acc, rx), p.bias[E + c]);
             }
-            __syncwarp();
+            __syncwarp(gmask);
             if (C == 1) {
                 xi = __fdiv_rn(1.f, __fadd_rn(1.f, expf(-xs[0])));
             } else {
                 float xm = -FLT_MAX;
-                for (int c = lane; c < C; c += 32) xm = fmaxf(xm, xs[c]);
-                xm = warp_max(xm);
+                for (int c = lane; c < C; c += G) xm = fmaxf(xm, xs[c]);
+                xm = grp_max<G>(gmask, xm);
                 float Sx = 0.f;
-                for (int c = lane; c < C; c += 32) Sx += expf(xs[c] - xm);
-                Sx = warp_sum(Sx);
+                for (int c = lane; c < C; c += G) Sx += expf(xs[c] - xm);
+                Sx = grp_sum<G>(gmask, Sx);
                 xi = __fdiv_rn(1.f, Sx);
             }
         }
@@ -219,14 +232,14 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
         if (p.n_cent > 0) {
             float bsc = -kInf;
             int bj = 0x7fffffff;
-            for (int j = lane; j < p.n_cent; j += 32) {
+            for (int j = lane; j < p.n_cent; j += G) {
                 float acc = 0.f;
                 for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + C + j]);
                 const float cn = p.cnorm[j];
                 const float sc = cn > 0.f ? __fdiv_rn(acc, cn) : -kInf;
                 if (sc > bsc || (sc == bsc && j < bj)) { bsc = sc; bj = j; }
             }
-            warp_argmax(bsc, bj);
+            grp_argmax<G>(gmask, bsc, bj);
             Lhat = p.lhat_tab[bj];
         }
         if (lane == 0 && p.lhat_out) p.lhat_out[t] = (int16_t)Lhat;
@@ -236,14 +249,14 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
         for (int j = 0; j < K; ++j) {
             const int c0 = coff_l[topk[j]], c1 = coff_l[topk[j] + 1];
             float gmin = kInf;
-            for (int c = c0 + lane; c < c1; c += 32) {
+            for (int c = c0 + lane; c < c1; c += G) {
                 const float Q = p.tab.cand_Q[c];
                 if (__fadd_rn(Dhat, Q) <= Dbar) {
                     const int m = p.tab.cand_m[c];
                     gmin = fminf(gmin, (m != s) ? p.tab.trans[s * M + m] : 0.f);
                 }
             }
-            Gamma = __fadd_rn(Gamma, warp_min(gmin));
+            Gamma = __fadd_rn(Gamma, grp_min<G>(gmask, gmin));
         }
         const float Lambda = __fmul_rn(p.tab.lambda[l], I);
         const bool skip_ok = (Gamma > 0.f) && (I <= p.tab.theta[l]) && (__fadd_rn(Dhat, Lambda) <= Dbar);
@@ -274,7 +287,7 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
             const int cb = coff[0];
             const int nc = coff[E] - cb;
             // (1) per-candidate terms
-            for (int c = lane; c < nc; c += 32) {
+            for (int c = lane; c < nc; c += G) {
                 const float Q = p.tab.cand_Q[cb + c];
                 const int mm = p.tab.cand_m[cb + c];
                 cok[c] = (Q <= R) ? 1 : 0;
@@ -282,12 +295,12 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
                 cph[c] = have_phi ? bufPhi[mm * E + p.tab.cand_k[cb + c]] : 0.f;
                 cmv[c] = (uint8_t)mm;
             }
-            __syncwarp();
+            __syncwarp(gmask);
             // (2) V(m, k') = best next action from m for target k'
             const float* ct = p.tab.ctab + (size_t)lp * M * M;
             const float skip_cost = __fmul_rn(p.omega_D, __fdiv_rn(eps, Dbar));
             const bool skip_budget = eps <= R;
-            for (int idx = lane; idx < ME; idx += 32) {
+            for (int idx = lane; idx < ME; idx += G) {
                 const int m = idx / E, kp = idx - (idx / E) * E;
                 const int s0 = coff[kp] - cb, s1 = coff[kp + 1] - cb;
                 const float* ctm = ct + m * M;
@@ -310,10 +323,10 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
                 }
                 bufV[idx] = best;
             }
-            __syncwarp();
+            __syncwarp(gmask);
             // (3) Phi_{l'-1}(m, k)
             const float* Pl = p.tab.P + (size_t)(lp - 1) * E * E;
-            for (int idx = lane; idx < ME; idx += 32) {
+            for (int idx = lane; idx < ME; idx += G) {
                 const int m = idx / E, k = idx - (idx / E) * E;
                 const float* Prow = Pl + k * E;
                 const float* Vrow = bufV + m * E;
@@ -321,7 +334,7 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
                 for (int kp = 0; kp < E; ++kp) acc = __fadd_rn(acc, __fmul_rn(__ldg(Prow + kp), Vrow[kp]));
                 bufPhi[idx] = acc;
             }
-            __syncwarp();
+            __syncwarp(gmask);
             have_phi = true;
         }
 
@@ -333,7 +346,7 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
             const int c0 = coff_l[topk[j]], c1 = coff_l[topk[j] + 1];
             float bv = kInf;
             int bi = 0x7fffffff;
-            for (int c = c0 + lane; c < c1; c += 32) {
+            for (int c = c0 + lane; c < c1; c += G) {
                 const float Q = p.tab.cand_Q[c];
                 if (!(__fadd_rn(Dhat, Q) <= Dbar)) continue;
                 if (!(__fadd_rn(Drun, Q) <= Dbar)) continue;
@@ -343,7 +356,7 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
                 if (j == 0) v = __fadd_rn(f, have_phi ? phiP[m * E + p.tab.cand_k[c]] : 0.f);
                 if (v < bv) { bv = v; bi = c; }
             }
-            warp_argmin(bv, bi);
+            grp_argmin<G>(gmask, bv, bi);
             esel[j] = p.tab.cand_k[bi];
             msel[j] = p.tab.cand_m[bi];
             Drun = __fadd_rn(Drun, p.tab.cand_Q[bi]);
@@ -412,7 +425,7 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
             if (use_shared) ++wc.shared_phi;
             if (Dbar > 0.f && Dbar < FLT_MAX) wc.max_ratio = fmaxf(wc.max_ratio, Dnew / Dbar);
         }
-        __syncwarp();
+        __syncwarp(gmask);
     }
     if (lane == 0) {
         atomicAdd(&blk_cnt[0], wc.layer_tokens);
@@ -430,7 +443,7 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
     }
     __syncthreads();
     if (threadIdx.x == 0 && blk_cnt[0]) {
-        DevCounters* c = p.ctr;
+        DevCounters* c = p.ctr + (blockIdx.x % kCtrCopies);
         atomicAdd(&c->layer_tokens, blk_cnt[0]);
         atomicAdd(&c->exec_tokens, blk_cnt[1]);
         atomicAdd(&c->skipped, blk_cnt[2]);
@@ -536,10 +549,13 @@ cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStre
     return cudaGetLastError();
 }
 
+// Lanes per token: the smallest group that holds one expert per lane.
+int decide_group(int E) { return E <= 8 ? 8 : E <= 16 ? 16 : 32; }
+
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand) {
     const size_t MC = (size_t)max_layer_cand;
-    const size_t per_warp = (size_t)(2 * E + C + 2 * M * E) + 2 * MC + ((MC + 3) / 4) * 2;
-    return per_warp * sizeof(float) * kWarps;
+    const size_t per_group = (size_t)(2 * E + C + 2 * M * E) + 2 * MC + ((MC + 3) / 4) * 2;
+    return per_group * sizeof(float) * kWarps * (32 / decide_group(E));
 }
 
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
@@ -547,15 +563,22 @@ cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
     const size_t smem = decide_smem_bytes(p.E, p.C, p.M, p.tab.max_layer_cand);
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(decide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             200 * 1024);
+        cudaError_t e = cudaFuncSetAttribute(decide_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(decide_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(decide_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     if (smem > 200 * 1024) return cudaErrorInvalidValue;
-    int blocks = (p.T + kWarps - 1) / kWarps;
+    const int G = decide_group(p.E);
+    const int per_block = kWarps * (32 / G);
+    int blocks = (p.T + per_block - 1) / per_block;
     blocks = blocks < num_sms * 16 ? blocks : num_sms * 16;
-    decide_kernel<<<blocks, kWarps * 32, smem, st>>>(p);
+    if (G == 8) decide_kernel<8><<<blocks, kWarps * 32, smem, st>>>(p);
+    else if (G == 16) decide_kernel<16><<<blocks, kWarps * 32, smem, st>>>(p);
+    else decide_kernel<32><<<blocks, kWarps * 32, smem, st>>>(p);
     return cudaGetLastError();
 }
 

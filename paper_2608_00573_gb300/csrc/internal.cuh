@@ -28,8 +28,12 @@ constexpr int kGateUp = 128;        // W13 gate/up row interleave
 // Device error codes (first one wins).
 enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3, ERR_TIMEOUT_ROUTER = 4 };
 
-// Device-side counters (trimmoe_stats_t is assembled from these).
-struct DevCounters {
+// Device-side counters (trimmoe_stats_t is assembled from these).  The handle
+// keeps kCtrCopies copies, each on its own cache lines; a block of the
+// decision kernel adds to copy blockIdx.x % kCtrCopies so that the atomics of
+// different blocks do not queue on one line, and the host sums the copies.
+constexpr int kCtrCopies = 32;
+struct __align__(256) DevCounters {
     unsigned long long layer_tokens, exec_tokens, skipped, exited;
     unsigned long long pairs_local_exact, pairs_local_sub, pairs_remote_exact, pairs_remote_sub;
     unsigned long long shared_rows, remote_hops, pairs_total;
@@ -38,6 +42,7 @@ struct DevCounters {
     double delay_ms;
     unsigned int max_budget_ratio_bits;   // non-negative float bits, atomicMax-able
 };
+static_assert(sizeof(DevCounters) == 256, "counter copies on separate cache lines");
 
 // Per-layer decision tables on the device (built at create).
 struct DevTables {

@@ -595,7 +595,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->goff, (size_t)E + 2) && h->dalloc(&h->blk_counts, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->blk_base, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
-              h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, 1) && h->dalloc(&h->dev_err, 1) &&
+              h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, kCtrCopies) && h->dalloc(&h->dev_err, 1) &&
               h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2) &&
               h->dalloc(&h->prev_target, T) && h->dalloc(&h->phi_tabs, std::max<size_t>(tab_floats, 1)) &&
               h->dalloc(&h->thr, std::max<size_t>(h->h_thr.size(), 1)) && h->dalloc(&h->dbar_shared, 1);
@@ -643,7 +643,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
             }
         up(h->rope, rt.data(), rt.size() * sizeof(float2));
     }
-    if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters));
+    if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies);
     if (ce == cudaSuccess) ce = cudaMemset(h->dev_err, 0, sizeof(int));
     if (ce == cudaSuccess) ce = cudaMemset(h->Xp, 0, (size_t)h->rows_xp * d * 2);
     if (ce != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, std::string("create: ") + cudaGetErrorString(ce));
@@ -1241,6 +1241,33 @@ extern "C" trimmoe_status trimmoe_forward_host(trimmoe_handle h, int T, trimmoe_
     return TRIMMOE_OK;
 }
 
+// Sum of the device counter copies (copy order; the ratio is a maximum).
+cudaError_t read_counters(const DevCounters* dev, DevCounters* out) {
+    DevCounters c[kCtrCopies];
+    const cudaError_t e = cudaMemcpy(c, dev, sizeof c, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return e;
+    std::memset(out, 0, sizeof *out);
+    for (int i = 0; i < kCtrCopies; ++i) {
+        out->layer_tokens += c[i].layer_tokens;
+        out->exec_tokens += c[i].exec_tokens;
+        out->skipped += c[i].skipped;
+        out->exited += c[i].exited;
+        out->pairs_local_exact += c[i].pairs_local_exact;
+        out->pairs_local_sub += c[i].pairs_local_sub;
+        out->pairs_remote_exact += c[i].pairs_remote_exact;
+        out->pairs_remote_sub += c[i].pairs_remote_sub;
+        out->shared_rows += c[i].shared_rows;
+        out->remote_hops += c[i].remote_hops;
+        out->pairs_total += c[i].pairs_total;
+        out->experts_touched += c[i].experts_touched;
+        out->shared_touched += c[i].shared_touched;
+        out->lookahead_shared += c[i].lookahead_shared;
+        out->delay_ms += c[i].delay_ms;
+        out->max_budget_ratio_bits = std::max(out->max_budget_ratio_bits, c[i].max_budget_ratio_bits);
+    }
+    return cudaSuccess;
+}
+
 extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) {
     if (!h || !out) return TRIMMOE_ERR_ARG;
     DeviceGuard g(h->dev);
@@ -1248,7 +1275,7 @@ extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) 
         return h->fail(TRIMMOE_ERR_CUDA, std::string("stats: ") + cudaGetErrorString(cudaGetLastError()));
     DevCounters dc;
     int derr = 0;
-    if (cudaMemcpy(&dc, h->ctr, sizeof dc, cudaMemcpyDeviceToHost) != cudaSuccess ||
+    if (read_counters(h->ctr, &dc) != cudaSuccess ||
         cudaMemcpy(&derr, h->dev_err, sizeof derr, cudaMemcpyDeviceToHost) != cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "stats: copy failed");
     h->drain_events();
@@ -1303,7 +1330,7 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
     DeviceGuard g(h->dev);
     if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, "reset: sync failed");
     h->drain_events();
-    if (cudaMemset(h->ctr, 0, sizeof(DevCounters)) != cudaSuccess ||
+    if (cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies) != cudaSuccess ||
         cudaMemset(h->dev_err, 0, sizeof(int)) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "reset: memset failed");
@@ -1461,7 +1488,7 @@ extern "C" trimmoe_status trimmoe_feedback(trimmoe_handle h, const trimmoe_feedb
     double res[2] = {0.0, 0.0};
     DevCounters dc;
     if (e == cudaSuccess) e = cudaMemcpy(res, h->fb_result, sizeof res, cudaMemcpyDeviceToHost);
-    if (e == cudaSuccess) e = cudaMemcpy(&dc, h->ctr, sizeof dc, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = read_counters(h->ctr, &dc);
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("feedback: ") + cudaGetErrorString(e));
     const double window_delay = dc.delay_ms - h->win_delay0;
     const double ref = h->win_ref_slots;
