@@ -552,15 +552,23 @@ cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStre
 // Lanes per token: the smallest group that holds one expert per lane.
 int decide_group(int E) { return E <= 8 ? 8 : E <= 16 ? 16 : 32; }
 
-size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand) {
+size_t decide_smem_for(int E, int C, int M, int max_layer_cand, int G) {
     const size_t MC = (size_t)max_layer_cand;
     const size_t per_group = (size_t)(2 * E + C + 2 * M * E) + 2 * MC + ((MC + 3) / 4) * 2;
-    return per_group * sizeof(float) * kWarps * (32 / decide_group(E));
+    return per_group * sizeof(float) * kWarps * (32 / G);
+}
+
+size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand) {
+    return decide_smem_for(E, C, M, max_layer_cand, decide_group(E));
 }
 
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    const size_t smem = decide_smem_bytes(p.E, p.C, p.M, p.tab.max_layer_cand);
+    // Groups smaller than a warp pay off when the tokens outnumber the resident
+    // warps; a small batch keeps a full warp per token for the shortest
+    // per-token latency (its look-ahead loops run over M*E entries).
+    const int G = p.T >= num_sms * 16 ? decide_group(p.E) : 32;
+    const size_t smem = decide_smem_for(p.E, p.C, p.M, p.tab.max_layer_cand, G);
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(decide_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
@@ -572,7 +580,6 @@ cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
         attr_set = true;
     }
     if (smem > 200 * 1024) return cudaErrorInvalidValue;
-    const int G = decide_group(p.E);
     const int per_block = kWarps * (32 / G);
     int blocks = (p.T + per_block - 1) / per_block;
     blocks = blocks < num_sms * 16 ? blocks : num_sms * 16;
