@@ -363,7 +363,7 @@ trimmoe_status trimmoe_replicate(int N, int E, int M, const float* lambda, const
  * int32 [T*k] (position of pair t*k+j in perm, -1 if not executed) and pos_sh
  * int32 [T] (row of token t among the shared-expert rows, -1 if none; may be
  * NULL when has_shared == 0).  Per-chunk scratch lives in one static device
- * array of about 264 KB held by every GPU that loads the library until exit;
+ * array of about 132 KB held by every GPU that loads the library until exit;
  * hence T <= 65536 and E <= 128 (ERR_ARG beyond, with a message in
  * trimmoe_last_error(NULL)).  It calls no cudaMalloc/cudaFree.  The first call on
  * each device looks up the array's device address once; make that first call

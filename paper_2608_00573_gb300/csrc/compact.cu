@@ -7,10 +7,10 @@
 // (Sec. V-E) removes exited tokens from the active set; only the survivors'
 // pairs reach the expert FFN.
 //
-// Three passes over chunks of kChunk tokens: per-chunk bucket counts, one
-// scan over chunks and buckets, and a scatter in which each warp of a chunk's
-// block walks its 32 tokens in order and ranks equal buckets with
-// __match_any_sync.
+// Two passes over chunks of kChunk tokens: per-chunk bucket counts, then a
+// scatter in which each chunk's block derives its base and the group offsets
+// from all chunks' counts and each of its warps walks its 32 tokens in order,
+// ranking equal buckets with __match_any_sync.
 #include <mutex>
 #include <string>
 
@@ -38,31 +38,45 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const CompactParams p) {
     for (int i = threadIdx.x; i < nb; i += blockDim.x) p.blk_counts[blockIdx.x * nb + i] = cnt[i];
 }
 
-// One block of 1024 threads: each warp takes buckets e = warp, warp + 32, ...
-// and scans the chunks' counts of that bucket (32 chunks per step); then one
-// warp turns the bucket totals into group offsets.
-__global__ void __launch_bounds__(1024) scan_kernel(const CompactParams p) {
-    __shared__ int total[kMaxE + 1];
-    const int nb = p.E + 1;
+// One block per chunk, one warp per 32 consecutive tokens of it.  The block
+// first reads every chunk's counts: per bucket, the sum over the earlier chunks
+// (this chunk's base) and over all chunks (the bucket total), and scans the
+// totals into the group offsets (block 0 publishes them).  Each warp counts its
+// pairs per bucket, the block turns the counts into per-warp starting
+// positions (group offset + chunk base + the earlier warps' counts), and each
+// warp then walks its pairs in (t, j) order, 32 at a time, ranking equal
+// buckets with __match_any_sync.  Integer sums: the result does not depend on
+// the order of the additions.
+constexpr int kScatWarps = kChunk / 32;
+
+__global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) {
+    __shared__ int run[kScatWarps][kMaxE + 1];
+    __shared__ int cbase[kMaxE + 1], total[kMaxE + 1], goff_s[kMaxE + 2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int e = warp; e < nb; e += 32) {
-        int run = 0;
+    const int nb = p.E + 1;
+    for (int i = threadIdx.x; i < kScatWarps * nb; i += blockDim.x) run[i / nb][i % nb] = 0;
+    // Chunk base and total per bucket: a warp per bucket, lanes over chunks.
+    for (int e = warp; e < nb; e += kScatWarps) {
+        int pre = 0, all = 0;
         for (int b0 = 0; b0 < p.nblk; b0 += 32) {
             const int b = b0 + lane;
             const int c = b < p.nblk ? p.blk_counts[b * nb + e] : 0;
-            int incl = c;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int v = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += v;
-            }
-            if (b < p.nblk) p.blk_base[b * nb + e] = run + incl - c;
-            run += __shfl_sync(0xffffffffu, incl, 31);
+            all += c;
+            pre += b < (int)blockIdx.x ? c : 0;
         }
-        if (lane == 0) total[e] = run;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            all += __shfl_xor_sync(0xffffffffu, all, o);
+            pre += __shfl_xor_sync(0xffffffffu, pre, o);
+        }
+        if (lane == 0) {
+            cbase[e] = pre;
+            total[e] = all;
+        }
     }
     __syncthreads();
     if (warp == 0) {
+        // Group offsets: exclusive prefix of the bucket totals.
         int base = 0;
         unsigned long long touched = 0;
         for (int e0 = 0; e0 < nb; e0 += 32) {
@@ -74,32 +88,22 @@ __global__ void __launch_bounds__(1024) scan_kernel(const CompactParams p) {
                 const int v = __shfl_up_sync(0xffffffffu, incl, o);
                 if (lane >= o) incl += v;
             }
-            if (e < nb) p.goff[e] = base + incl - c;
+            if (e < nb) goff_s[e] = base + incl - c;
             touched += __popc(__ballot_sync(0xffffffffu, e < p.E && c > 0));
             base += __shfl_sync(0xffffffffu, incl, 31);
         }
-        if (lane == 0) {
-            p.goff[nb] = base;
-            atomicAdd(&p.ctr->pairs_total, (unsigned long long)(base - total[p.E]));
-            atomicAdd(&p.ctr->shared_rows, (unsigned long long)total[p.E]);
-            atomicAdd(&p.ctr->experts_touched, touched);
-            if (total[p.E] > 0) atomicAdd(&p.ctr->shared_touched, 1ull);
+        if (lane == 0) goff_s[nb] = base;
+        if (blockIdx.x == 0) {
+            __syncwarp();
+            for (int e = lane; e <= nb; e += 32) p.goff[e] = goff_s[e];
+            if (lane == 0) {
+                atomicAdd(&p.ctr->pairs_total, (unsigned long long)(base - total[p.E]));
+                atomicAdd(&p.ctr->shared_rows, (unsigned long long)total[p.E]);
+                atomicAdd(&p.ctr->experts_touched, touched);
+                if (total[p.E] > 0) atomicAdd(&p.ctr->shared_touched, 1ull);
+            }
         }
     }
-}
-
-// One block per chunk, one warp per 32 consecutive tokens of it.  Each warp
-// counts its pairs per bucket, the block turns the counts into per-warp
-// starting positions (the chunk's base plus the earlier warps' counts), and
-// each warp then walks its pairs in (t, j) order, 32 at a time, ranking equal
-// buckets with __match_any_sync.
-constexpr int kScatWarps = kChunk / 32;
-
-__global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) {
-    __shared__ int run[kScatWarps][kMaxE + 1];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nb = p.E + 1;
-    for (int i = threadIdx.x; i < kScatWarps * nb; i += blockDim.x) run[i / nb][i % nb] = 0;
     __syncthreads();
     const int t0 = blockIdx.x * kChunk + warp * 32;
     const int tn = max(0, min(32, p.T - t0));
@@ -124,7 +128,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) 
     __syncthreads();
     // Per-warp starting positions: exclusive prefix over the warps, per bucket.
     for (int e = threadIdx.x; e < nb; e += blockDim.x) {
-        int acc = p.goff[e] + p.blk_base[blockIdx.x * nb + e];
+        int acc = goff_s[e] + cbase[e];
         for (int w = 0; w < kScatWarps; ++w) {
             const int c = run[w][e];
             run[w][e] = acc;
@@ -166,7 +170,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) 
         if (take) {
             const int pos = run[warp][p.E] + __popc(ball & lt_mask);
             p.perm[pos] = t;
-            p.pos_sh[t] = pos - p.goff[p.E];
+            p.pos_sh[t] = pos - goff_s[p.E];
         }
     }
 }
@@ -230,7 +234,6 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
     count_kernel<<<p.nblk, kChunk, 0, st>>>(p);
-    scan_kernel<<<1, 1024, 0, st>>>(p);
     scatter_kernel<<<p.nblk, kChunk, 0, st>>>(p);
     return cudaGetLastError();
 }
@@ -265,7 +268,7 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
 // another pool, or hosts that must not allocate during a captured or
 // latency-critical section.  For them the per-chunk counts and bases of the
 // compaction live in this file-scope device array instead of a handle's
-// workspace.  Its size is fixed (about 264 KB); every GPU that loads the
+// workspace.  Its size is fixed (about 132 KB); every GPU that loads the
 // library holds it until the process exits.
 namespace tmoe {
 namespace {
@@ -275,7 +278,6 @@ constexpr int kNoAllocMaxBlk = kNoAllocMaxT / kChunk;
 
 struct NoAllocScratch {
     int32_t blk_counts[kNoAllocMaxBlk * (kMaxE + 1)];
-    int32_t blk_base[kNoAllocMaxBlk * (kMaxE + 1)];
     DevCounters ctr;
 };
 
@@ -336,7 +338,7 @@ extern "C" trimmoe_status trimmoe_compact_noalloc(const uint8_t* action, const u
     trimmoe_status rc = noalloc_scratch(&s);
     if (rc != TRIMMOE_OK) return rc;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    // Only the counters must start at zero; counts and bases are fully rewritten.
+    // Only the counters must start at zero; the counts are fully rewritten.
     if (cudaMemsetAsync(&s->ctr, 0, sizeof(DevCounters), st) != cudaSuccess) {
         set_global_error("compact_noalloc: cudaMemsetAsync failed");
         return TRIMMOE_ERR_CUDA;
@@ -357,7 +359,6 @@ extern "C" trimmoe_status trimmoe_compact_noalloc(const uint8_t* action, const u
     cp.action = action;
     cp.exp_sel = exp_sel;
     cp.blk_counts = s->blk_counts;
-    cp.blk_base = s->blk_base;
     cp.goff = group_off;
     cp.perm = perm;
     cp.pos_pair = pos_pair;

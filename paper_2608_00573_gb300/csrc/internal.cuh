@@ -139,7 +139,6 @@ struct CompactParams {
     const uint8_t* action;
     const uint8_t* exp_sel;
     int32_t* blk_counts;   // [nblk][E+1]
-    int32_t* blk_base;     // [nblk][E+1]
     int32_t* goff;         // [E+2]
     int32_t* perm;         // [T*k + T]
     int32_t* pos_pair;     // [T*k]

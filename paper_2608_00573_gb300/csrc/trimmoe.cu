@@ -163,7 +163,7 @@ struct trimmoe {
     uint8_t* srv_sel = nullptr;
     int32_t *perm = nullptr, *pos_pair = nullptr, *pos_sh = nullptr, *goff = nullptr;
     float* rnorm = nullptr;
-    int32_t *blk_counts = nullptr, *blk_base = nullptr;
+    int32_t* blk_counts = nullptr;
     __nv_bfloat16 *Xp = nullptr, *act = nullptr, *act_sh = nullptr, *Y = nullptr, *Ysh = nullptr;
     DevCounters* ctr = nullptr;
     int* dev_err = nullptr;
@@ -593,7 +593,6 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->perm, TK + T) && h->dalloc(&h->pos_pair, TK) && h->dalloc(&h->pos_sh, T) &&
               h->dalloc(&h->rnorm, T) &&
               h->dalloc(&h->goff, (size_t)E + 2) && h->dalloc(&h->blk_counts, (size_t)nblk * (E + 1)) &&
-              h->dalloc(&h->blk_base, (size_t)nblk * (E + 1)) &&
               h->dalloc(&h->Xp, (size_t)h->rows_xp * d) && h->dalloc(&h->act, TK * c.F) &&
               h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, kCtrCopies) && h->dalloc(&h->dev_err, 1) &&
               h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2) &&
@@ -947,7 +946,6 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     cp.action = dp.action;
     cp.exp_sel = dp.exp_sel;
     cp.blk_counts = h->blk_counts;
-    cp.blk_base = h->blk_base;
     cp.goff = h->goff;
     cp.perm = h->perm;
     cp.pos_pair = h->pos_pair;
@@ -1013,7 +1011,8 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm down: ") + cudaGetErrorString(e));
     h->n_gemm_up++;
     h->n_gemm_down++;
-    h->launches += 8 + (shared_tabs ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
+    // router, decide, count, scatter, gather, gate/up GEMM, down GEMM (+ look-ahead tables, split-K finishes)
+    h->launches += 7 + (shared_tabs ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
     if (has_sh) {
         GemmLaunch s1 = g1;
         s1.ksplit = 1;
