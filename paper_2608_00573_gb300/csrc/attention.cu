@@ -62,6 +62,8 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
 
 // One warp per token row: RMS factor in fp32, then a = bf16(h * r * gamma).
 __global__ void __launch_bounds__(256) attn_norm_kernel(const AttnParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     if (blockIdx.x == 0 && threadIdx.x == 0) {
         p.goff[0] = 0;
         p.goff[1] = p.T;
@@ -94,6 +96,7 @@ __global__ void __launch_bounds__(256) attn_norm_kernel(const AttnParams p) {
 
 template <int DH>
 __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
     constexpr int LD = DH + 8;                 // padded row (bf16): conflict-free ldmatrix
     constexpr int NTO = DH / 8;                // output n-tiles
     extern __shared__ __align__(16) uint8_t sm[];
@@ -232,6 +235,7 @@ __global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
         }
         __syncwarp();
     }
+    pdl_trigger();   // the next kernel may be scheduled once every block got here or exited
 }
 
 template <int DH>
@@ -245,7 +249,8 @@ cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st) 
     if (p.T <= 0) return cudaSuccess;
     int blocks = (p.T + 7) / 8;
     blocks = blocks < num_sms * 8 ? blocks : num_sms * 8;
-    attn_norm_kernel<<<blocks, 256, 0, st>>>(p);
+    const cudaError_t e = launch_pdl(attn_norm_kernel, dim3(blocks), dim3(256), 0, st, p);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
@@ -263,9 +268,11 @@ cudaError_t launch_attention(const AttnParams& p, int head_dim, cudaStream_t st)
         attr_set = true;
     }
     const dim3 grid(p.Hq, (p.T + p.S - 1) / p.S);
-    if (head_dim == 64) attention_kernel<64><<<grid, 128, attn_smem<64>(), st>>>(p);
-    else if (head_dim == 128) attention_kernel<128><<<grid, 128, attn_smem<128>(), st>>>(p);
+    cudaError_t e;
+    if (head_dim == 64) e = launch_pdl(attention_kernel<64>, grid, dim3(128), attn_smem<64>(), st, p);
+    else if (head_dim == 128) e = launch_pdl(attention_kernel<128>, grid, dim3(128), attn_smem<128>(), st, p);
     else return cudaErrorInvalidValue;
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -24,6 +24,8 @@ namespace {
 // per lane each) are issued before the first one is used.
 template <int KT>
 __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     constexpr int kU = KT <= 2 ? 4 : 2;
     const int lane = threadIdx.x & 31;
     const int nchunk = p.d >> 3;
@@ -117,10 +119,12 @@ int combine_grid(int T, int num_sms) {
 
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    if (p.k <= 1) combine_kernel<1><<<combine_grid<1>(p.T, num_sms), 256, 0, st>>>(p);
-    else if (p.k <= 2) combine_kernel<2><<<combine_grid<2>(p.T, num_sms), 256, 0, st>>>(p);
-    else if (p.k <= 4) combine_kernel<4><<<combine_grid<4>(p.T, num_sms), 256, 0, st>>>(p);
-    else combine_kernel<kMaxK><<<combine_grid<kMaxK>(p.T, num_sms), 256, 0, st>>>(p);
+    cudaError_t e;
+    if (p.k <= 1) e = launch_pdl(combine_kernel<1>, dim3(combine_grid<1>(p.T, num_sms)), dim3(256), 0, st, p);
+    else if (p.k <= 2) e = launch_pdl(combine_kernel<2>, dim3(combine_grid<2>(p.T, num_sms)), dim3(256), 0, st, p);
+    else if (p.k <= 4) e = launch_pdl(combine_kernel<4>, dim3(combine_grid<4>(p.T, num_sms)), dim3(256), 0, st, p);
+    else e = launch_pdl(combine_kernel<kMaxK>, dim3(combine_grid<kMaxK>(p.T, num_sms)), dim3(256), 0, st, p);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

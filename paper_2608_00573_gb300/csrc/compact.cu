@@ -23,6 +23,8 @@ namespace {
 constexpr int kChunk = 256;
 
 __global__ void __launch_bounds__(kChunk) count_kernel(const CompactParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     __shared__ int cnt[kMaxE + 1];
     const int nb = p.E + 1;
     for (int i = threadIdx.x; i < nb; i += blockDim.x) cnt[i] = 0;
@@ -50,6 +52,8 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const CompactParams p) {
 constexpr int kScatWarps = kChunk / 32;
 
 __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     __shared__ int run[kScatWarps][kMaxE + 1];
     __shared__ int cbase[kMaxE + 1], total[kMaxE + 1], goff_s[kMaxE + 2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -187,6 +191,8 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
                                                      const float* __restrict__ rnorm,
                                                      const __nv_bfloat16* __restrict__ gamma,
                                                      __nv_bfloat16* __restrict__ Xp) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint4 sg[];      // gamma, d / 8 chunks
     const int nrows = goff[E + 1];
     const int routed = goff[E];
@@ -233,8 +239,9 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
 
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    count_kernel<<<p.nblk, kChunk, 0, st>>>(p);
-    scatter_kernel<<<p.nblk, kChunk, 0, st>>>(p);
+    cudaError_t e = launch_pdl(count_kernel, dim3(p.nblk), dim3(kChunk), 0, st, p);
+    if (e == cudaSuccess) e = launch_pdl(scatter_kernel, dim3(p.nblk), dim3(kChunk), 0, st, p);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
@@ -254,7 +261,9 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
     }
     int blocks = (max_rows + 7) / 8;
     blocks = blocks < num_sms * per_sm ? blocks : num_sms * per_sm;
-    gather_kernel<<<blocks, 256, smem, st>>>(perm, goff, E, k, d, h, rnorm, gamma, Xp);
+    const cudaError_t e = launch_pdl(gather_kernel, dim3(blocks), dim3(256), smem, st, perm, goff, E, k, d, h, rnorm,
+                                     gamma, Xp);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -13,6 +13,8 @@ namespace tmoe {
 namespace {
 
 __global__ void __launch_bounds__(128) feedback_users_kernel(const FeedbackParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     const int u = blockIdx.x * blockDim.x + threadIdx.x;
     if (u >= p.users) return;
     const int t0 = u * p.user_size;
@@ -41,6 +43,8 @@ __global__ void __launch_bounds__(128) feedback_users_kernel(const FeedbackParam
 }
 
 __global__ void feedback_reduce_kernel(const FeedbackParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     if (threadIdx.x != 0 || blockIdx.x != 0) return;
     double s = 0.0;
     int n = 0;
@@ -55,8 +59,10 @@ __global__ void feedback_reduce_kernel(const FeedbackParams p) {
 }  // namespace
 
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st) {
-    if (p.users > 0) feedback_users_kernel<<<(p.users + 127) / 128, 128, 0, st>>>(p);
-    feedback_reduce_kernel<<<1, 32, 0, st>>>(p);
+    cudaError_t e = cudaSuccess;
+    if (p.users > 0) e = launch_pdl(feedback_users_kernel, dim3((p.users + 127) / 128), dim3(128), 0, st, p);
+    if (e == cudaSuccess) e = launch_pdl(feedback_reduce_kernel, dim3(1), dim3(32), 0, st, p);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

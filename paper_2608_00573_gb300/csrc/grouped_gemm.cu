@@ -287,6 +287,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
                     int rope_S, int rope_dh, int n_rot, int mblk, int ksplit, float* __restrict__ partial,
                     int ldp, size_t pstride) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -434,6 +436,8 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
                          __nv_bfloat16* __restrict__ out, int ldo, int* err,
                          const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
                          int rope_S, int rope_dh, int n_rot, int mblk) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -618,17 +622,21 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     const long long a_tile_bytes = (long long)BM * g.K * 2;
     if (g.tmB_pair && (g.ksplit <= 1) && pair_clusters(num_sms) > 0) {
         const int mblk2 = (int)std::max(1LL, (48LL << 20) / (2 * a_tile_bytes));
-        grouped_gemm_pair_kernel<<<2 * pair_clusters(num_sms), kThreads, kPairSmemBytes, st>>>(
-            *g.tmA, *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh,
-            g.n_rot, mblk2);
+        const cudaError_t e = launch_pdl(
+            grouped_gemm_pair_kernel, dim3(2 * pair_clusters(num_sms)), dim3(kThreads), kPairSmemBytes, st, *g.tmA,
+            *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
+            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot,
+            mblk2);
+        if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }
     const int mblk = (int)std::max(1LL, (48LL << 20) / a_tile_bytes);
-    grouped_gemm_kernel<<<num_sms, kThreads, kSmemBytes, st>>>(
-        *g.tmA, *g.tmB, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-        g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot,
-        mblk, g.ksplit > 1 ? g.ksplit : 1, g.partial, g.ldp, g.pstride);
+    const cudaError_t e = launch_pdl(
+        grouped_gemm_kernel, dim3(num_sms), dim3(kThreads), kSmemBytes, st, *g.tmA, *g.tmB, g.goff, g.first_group,
+        g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n, g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err,
+        g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot, mblk, g.ksplit > 1 ? g.ksplit : 1, g.partial, g.ldp,
+        g.pstride);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
@@ -657,6 +665,8 @@ __global__ void __launch_bounds__(256) splitk_finish_kernel(const int* __restric
                                                             const float* __restrict__ partial, int ldp,
                                                             size_t pstride, int epi_mode,
                                                             __nv_bfloat16* __restrict__ out, int ldo) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     const int r0 = out_rebase ? 0 : goff[first_group];
     const int r1 = goff[first_group + ngroups] - (out_rebase ? goff[first_group] : 0);
     const int ncol = epi_mode == EPI_SWIGLU ? ldp / 2 : ldp;
@@ -687,8 +697,10 @@ __global__ void __launch_bounds__(256) splitk_finish_kernel(const int* __restric
 
 cudaError_t launch_splitk_finish(const GemmLaunch& g, int num_sms, cudaStream_t st) {
     if (g.epi_mode != EPI_STORE && g.epi_mode != EPI_SWIGLU && g.epi_mode != EPI_RELU) return cudaErrorInvalidValue;
-    splitk_finish_kernel<<<num_sms * 2, 256, 0, st>>>(g.goff, g.first_group, g.ngroups, g.out_rebase, g.ksplit,
-                                                       g.partial, g.ldp, g.pstride, g.epi_mode, g.out, g.ldo);
+    const cudaError_t e = launch_pdl(splitk_finish_kernel, dim3(num_sms * 2), dim3(256), 0, st, g.goff, g.first_group,
+                                     g.ngroups, g.out_rebase, g.ksplit, g.partial, g.ldp, g.pstride, g.epi_mode, g.out,
+                                     g.ldo);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -8,7 +8,10 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <cstdlib>
+#include <cstring>
 #include <string>
+#include <utility>
 
 #include "../../include/trimmoe.h"
 
@@ -235,6 +238,34 @@ cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st)
 cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);
 cudaError_t launch_attention(const AttnParams& p, int head_dim, cudaStream_t st);
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
+
+// Programmatic dependent launch.  The library's kernels are launched with
+// programmatic stream serialisation: a kernel may be scheduled while the
+// preceding grid in its stream is still finishing, runs its independent
+// prologue, then waits (pdl_wait) for that grid to complete and its memory to be
+// visible before touching anything written upstream.  Single-wave and
+// persistent kernels let the next grid be scheduled right after their wait
+// (pdl_trigger), multi-wave kernels only when each block is done, so that
+// waiting blocks never take the room of their later waves.  After a launch
+// without the attribute pdl_wait returns at once.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // Error text for calls made without a handle (read by trimmoe_last_error(NULL)).
 void set_global_error(const std::string& msg);

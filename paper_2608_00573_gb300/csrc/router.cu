@@ -108,6 +108,8 @@ router_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
         if (NL > 0) prefetch_tmap(&tmBlo);
     }
     __syncthreads();
+    pdl_wait();      // hidden states and liveness written by the preceding kernels
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     volatile int* abort_flag = &bars->abort_flag;
 
     if (warp == kConsumers) {
@@ -299,14 +301,16 @@ cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, cons
     const int per_sm = nt <= 4 ? 2 : 1;
     const int grid = (int)std::min<long long>(units, (long long)per_sm * num_sms);
     const CUtensorMap* lo = p.nl > 0 ? tmBlo : tmBhi;
+    cudaError_t e;
     switch (nt) {
-        case 1: router_kernel<1><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
-        case 2: router_kernel<2><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
-        case 4: router_kernel<4><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
-        case 8: router_kernel<8><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
-        case 12: router_kernel<12><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
-        default: router_kernel<16><<<grid, kThreads, smem, st>>>(*tmA, *tmBhi, *lo, p, stages); break;
+        case 1: e = launch_pdl(router_kernel<1>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
+        case 2: e = launch_pdl(router_kernel<2>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
+        case 4: e = launch_pdl(router_kernel<4>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
+        case 8: e = launch_pdl(router_kernel<8>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
+        case 12: e = launch_pdl(router_kernel<12>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
+        default: e = launch_pdl(router_kernel<16>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
     }
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
