@@ -8,8 +8,6 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include <cstdlib>
-#include <cstring>
 #include <string>
 #include <utility>
 
