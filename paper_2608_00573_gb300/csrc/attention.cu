@@ -21,17 +21,23 @@
 // host-made cos/sin table) is applied by the projection GEMM's epilogue to the
 // fp32 accumulators before their bf16 rounding.
 //
-// attention_kernel: one block per (query head, sequence), 4 warps.  Q, K and V
-// of the sequence (S <= 128 rows) are staged in padded shared memory by
-// cp.async with every load in flight at once.  Each warp owns two 16-row query blocks
-// (mb and 7 - mb, which balances the causal work), computes the full causal
-// score rows with mma.sync m16n8k16 (bf16 in, fp32 accumulate), takes the
-// softmax in fp32 registers (quad shuffles), rounds the probabilities to bf16
-// as the A operand of the P.V product (V fragments by ldmatrix.trans), divides
-// by the fp32 row sums and writes bf16 rows through shared memory with 16-byte
-// stores.  The contraction is small (S x S x Dh per head) next to the
-// projections, so the legacy mma.sync path is used; the projections are the
-// tcgen05 grouped GEMM.
+// attention_kernel: one CTA per (key/value head, sequence), 192 threads, on
+// the 5th-generation tensor cores.  S <= 128 keys fit one tile, so there is no
+// running maximum: per query head of the group
+//   S = Q K^T          tcgen05.mma M = 128 (queries), N = 128 (keys), K = Dh -> TMEM
+//   P = exp(scale (S - max))   causal mask, fp32 (exp as one ex2.approx per
+//                      key), rounded to bf16 into shared memory by the 128
+//                      softmax threads (one query row each; a warp skips the
+//                      32-key chunks above its rows' diagonal)
+//   O = P V            tcgen05.mma M = 128, N = Dh, K = 128 keys -> TMEM
+//   out = bf16(O / l)  l = the fp32 row sum of the unrounded probabilities
+// warp 0 loads K and V of the group once and the query heads one after another
+// (TMA, 128-byte swizzle); warp 1 issues the MMAs; warps 2-5 transpose V once
+// into a K-major tile (keys contiguous, so that every operand is K-major), then
+// run the softmax and the epilogue of each head while the tensor core computes
+// the next head's scores.  Rows past the sequence are loaded (the next
+// sequence's rows, or zero fill) but masked as keys and never stored as
+// queries.  Every wait is bounded (2 s) and records an error word on expiry.
 #include "internal.cuh"
 
 namespace tmoe {
@@ -94,153 +100,261 @@ __global__ void __launch_bounds__(256) attn_norm_kernel(const AttnParams p) {
     }
 }
 
+constexpr int kAttnThreads = 192;
+
+// Shared-memory layout (byte offsets from a 1024-aligned base).  A box is 128
+// rows x 64 bf16 columns (16 KB, 128-byte rows, 128-byte swizzle).
 template <int DH>
-__global__ void __launch_bounds__(128) attention_kernel(const AttnParams p) {
-    pdl_wait();      // results of the preceding kernel in the stream
-    constexpr int LD = DH + 8;                 // padded row (bf16): conflict-free ldmatrix
-    constexpr int NTO = DH / 8;                // output n-tiles
-    extern __shared__ __align__(16) uint8_t sm[];
-    __nv_bfloat16* sQ = reinterpret_cast<__nv_bfloat16*>(sm);
-    __nv_bfloat16* sK = sQ + kSeqMax * LD;
-    __nv_bfloat16* sV = sK + kSeqMax * LD;
+struct AttnLayout {
+    static constexpr int KB = DH / 64;                    // 64-column blocks of a head
+    static constexpr int BOX = 128 * 128;
+    static constexpr int Q = 0;                           // [KB][128 query rows][128 B]
+    static constexpr int K = Q + KB * BOX;                // [KB][128 key rows][128 B]
+    static constexpr int V = K + KB * BOX;                // as loaded: [KB][128 key rows][64 dims]
+    static constexpr int VT = V + KB * BOX;               // [2 key blocks][DH dim rows][64 keys]
+    static constexpr int P = VT + 2 * DH * 128;           // [2 key blocks][128 query rows][64 keys]
+    static constexpr int BYTES = P + 2 * BOX;
+};
 
-    const int hq = blockIdx.x, b = blockIdx.y;
-    const int g = hq / (p.Hq / p.Hkv);
-    const int t0 = b * p.S;
-    const int n = min(p.S, p.T - t0);
-    const int n16 = (n + 15) & ~15;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const size_t qoff = (size_t)hq * DH;
-    const size_t koff = (size_t)(p.Hq + g) * DH;
-    const size_t voff = (size_t)(p.Hq + p.Hkv + g) * DH;
-
-    // Stage Q, K and V of the sequence (the projection's epilogue has already
-    // rotated Q and K) with every load in flight at once; rows >= n are zero.
-    constexpr int RC = DH / 8;                 // 16-byte chunks per row
-    for (int i = tid; i < 3 * n16 * RC; i += 128) {
-        const int which = i / (n16 * RC);      // 0: query head, 1: key head, 2: value head
-        const int rem = i - which * n16 * RC;
-        const int r = rem / RC, c = (rem - r * RC) * 8;
-        __nv_bfloat16* dst = (which == 0 ? sQ : which == 1 ? sK : sV) + r * LD + c;
-        const size_t off = which == 0 ? qoff : which == 1 ? koff : voff;
-        const bool ok = r < n;
-        const __nv_bfloat16* src = p.qkv + (size_t)(t0 + (ok ? r : 0)) * p.nqkv + off + c;
-        cp_async16(smem_u32(dst), src, ok ? 16 : 0);
-    }
-    cp_async_commit();
-    cp_async_wait<0>();
-    __syncthreads();
-
-    const int gq = lane >> 2, tig = lane & 3;
-    const int nmb = n16 >> 4;
-    const size_t ostride = (size_t)p.Hq * DH;
-#pragma unroll 1
-    for (int pass = 0; pass < 2; ++pass) {
-        const int mb = pass == 0 ? warp : 7 - warp;
-        if (mb >= nmb) continue;
-        const int nt = 2 * (mb + 1);            // key tiles of 8 up to the block's last row
-        float s[16][4];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-            uint32_t a[4];
-            ldmatrix_x4(a, smem_u32(sQ + (mb * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LD + kk * 16 +
-                                    (lane >> 4) * 8));
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                if (j < nt) {
-                    uint32_t bb[2];
-                    ldmatrix_x2(bb, smem_u32(sK + (j * 8 + (lane & 7)) * LD + kk * 16 + ((lane >> 3) & 1) * 8));
-                    mma_bf16_16816(s[j], a, bb);
-                }
-            }
-        }
-        // Causal mask, softmax in fp32 (rows r0 and r1 of this thread).
-        const int r0 = mb * 16 + gq, r1 = r0 + 8;
-        float m0 = -INFINITY, m1 = -INFINITY;
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            if (j < nt) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int key = j * 8 + tig * 2 + (q & 1);
-                    const int row = q < 2 ? r0 : r1;
-                    if (key > row || key >= n) s[j][q] = -INFINITY;
-                }
-                m0 = fmaxf(m0, fmaxf(s[j][0], s[j][1]));
-                m1 = fmaxf(m1, fmaxf(s[j][2], s[j][3]));
-            }
-        }
-#pragma unroll
-        for (int o = 1; o <= 2; o <<= 1) {
-            m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, o));
-            m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, o));
-        }
-        float l0 = 0.f, l1 = 0.f;
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            if (j < nt) {
-                s[j][0] = expf((s[j][0] - m0) * p.scale);
-                s[j][1] = expf((s[j][1] - m0) * p.scale);
-                s[j][2] = expf((s[j][2] - m1) * p.scale);
-                s[j][3] = expf((s[j][3] - m1) * p.scale);
-                l0 += s[j][0] + s[j][1];
-                l1 += s[j][2] + s[j][3];
-            }
-        }
-#pragma unroll
-        for (int o = 1; o <= 2; o <<= 1) {
-            l0 += __shfl_xor_sync(0xffffffffu, l0, o);
-            l1 += __shfl_xor_sync(0xffffffffu, l1, o);
-        }
-        // O = P V over the key steps of 16 up to the block's last row.
-        float acc[NTO][4];
-#pragma unroll
-        for (int j = 0; j < NTO; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-            if (kk <= mb) {
-                uint32_t a[4];
-                a[0] = pack_bf16x2(s[2 * kk][0], s[2 * kk][1]);
-                a[1] = pack_bf16x2(s[2 * kk][2], s[2 * kk][3]);
-                a[2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-                a[3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-                for (int jn = 0; jn < NTO; jn += 2) {
-                    uint32_t bb[4];
-                    ldmatrix_x4_trans(bb, smem_u32(sV + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LD +
-                                                   jn * 8 + (lane >> 4) * 8));
-                    const uint32_t b0[2] = {bb[0], bb[1]}, b1[2] = {bb[2], bb[3]};
-                    mma_bf16_16816(acc[jn], a, b0);
-                    mma_bf16_16816(acc[jn + 1], a, b1);
-                }
-            }
-        }
-        // Normalise, stage the 16 rows in this warp's own Q rows, store 16-byte rows.
-        const float i0 = 1.f / l0, i1 = 1.f / l1;
-#pragma unroll
-        for (int jn = 0; jn < NTO; ++jn) {
-            const int col = jn * 8 + tig * 2;
-            *reinterpret_cast<uint32_t*>(sQ + r0 * LD + col) = pack_bf16x2(acc[jn][0] * i0, acc[jn][1] * i0);
-            *reinterpret_cast<uint32_t*>(sQ + r1 * LD + col) = pack_bf16x2(acc[jn][2] * i1, acc[jn][3] * i1);
-        }
-        __syncwarp();
-        for (int i = lane; i < 16 * (DH / 8); i += 32) {
-            const int rr = i / (DH / 8), c = (i - rr * (DH / 8)) * 8;
-            const int row = mb * 16 + rr;
-            if (row < n)
-                *reinterpret_cast<uint4*>(p.out + (size_t)(t0 + row) * ostride + qoff + c) =
-                    *reinterpret_cast<const uint4*>(sQ + row * LD + c);
-        }
-        __syncwarp();
-    }
-    pdl_trigger();   // the next kernel may be scheduled once every block got here or exited
-}
+struct __align__(8) AttnBars {
+    uint64_t kv, q, vt, s, sfree, pfull, pfree, o, ofree, qfree;
+    uint32_t tmem_base;
+    int abort_flag;
+};
 
 template <int DH>
 constexpr size_t attn_smem() {
-    return (size_t)3 * kSeqMax * (DH + 8) * sizeof(__nv_bfloat16);
+    return 1024 + (size_t)AttnLayout<DH>::BYTES + sizeof(AttnBars);
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    using L = AttnLayout<DH>;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+    const uint32_t sb = smem_u32(smem);
+    AttnBars* bars = reinterpret_cast<AttnBars*>(smem + L::BYTES);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = blockIdx.x, b = blockIdx.y;
+    const int G = p.Hq / p.Hkv;                          // query heads per key/value head
+    const int t0 = b * p.S;
+    const int n = min(p.S, p.T - t0);
+    const int kcol = (p.Hq + g) * DH, vcol = (p.Hq + p.Hkv + g) * DH;
+
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bars->kv), 1);
+        mbar_init(smem_u32(&bars->q), 1);
+        mbar_init(smem_u32(&bars->vt), 4);
+        mbar_init(smem_u32(&bars->s), 1);
+        mbar_init(smem_u32(&bars->sfree), 4);
+        mbar_init(smem_u32(&bars->pfull), 4);
+        mbar_init(smem_u32(&bars->pfree), 1);
+        mbar_init(smem_u32(&bars->o), 1);
+        mbar_init(smem_u32(&bars->ofree), 4);
+        mbar_init(smem_u32(&bars->qfree), 1);
+        bars->abort_flag = 0;
+        fence_barrier_init();
+        prefetch_tmap(&tm);
+    }
+    if (warp == 0) tmem_alloc(smem_u32(&bars->tmem_base), 256);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tS = bars->tmem_base, tO = bars->tmem_base + 128;
+    volatile int* abort_flag = &bars->abort_flag;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ------------------------------------------------------- loads
+            const uint32_t kvb = smem_u32(&bars->kv);
+            mbar_arrive_expect_tx(kvb, 2 * L::KB * L::BOX);
+            for (int kb = 0; kb < L::KB; ++kb) {
+                tma_load_2d(sb + L::K + kb * L::BOX, &tm, kcol + kb * 64, t0, kvb);
+                tma_load_2d(sb + L::V + kb * L::BOX, &tm, vcol + kb * 64, t0, kvb);
+            }
+            for (int i = 0; i < G; ++i) {
+                if (i > 0 && !mbar_wait_bounded(smem_u32(&bars->qfree), (i - 1) & 1, abort_flag, p.err,
+                                                ERR_TIMEOUT_ATTN))
+                    break;
+                const uint32_t qb = smem_u32(&bars->q);
+                mbar_arrive_expect_tx(qb, L::KB * L::BOX);
+                const int qcol = (g * G + i) * DH;
+                for (int kb = 0; kb < L::KB; ++kb) tma_load_2d(sb + L::Q + kb * L::BOX, &tm, qcol + kb * 64, t0, qb);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ------------------------------------------------------- MMAs
+            constexpr uint32_t idS = idesc_bf16_f32(128, 128);
+            constexpr uint32_t idO = idesc_bf16_f32(128, DH);
+            bool ok = mbar_wait_bounded(smem_u32(&bars->kv), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
+                      mbar_wait_bounded(smem_u32(&bars->vt), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+            for (int i = 0; i < G && ok; ++i) {
+                const uint32_t ph = i & 1, pph = (i - 1) & 1;
+                ok = mbar_wait_bounded(smem_u32(&bars->q), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
+                     (i == 0 || mbar_wait_bounded(smem_u32(&bars->sfree), pph, abort_flag, p.err, ERR_TIMEOUT_ATTN));
+                if (!ok) break;
+                tc_fence_after();
+#pragma unroll
+                for (int kb = 0; kb < L::KB; ++kb)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        tc_mma_bf16(tS, smem_desc_sw128(sb + L::Q + kb * L::BOX + kk * 32),
+                                    smem_desc_sw128(sb + L::K + kb * L::BOX + kk * 32), idS, (kb | kk) ? 1u : 0u);
+                tc_commit(smem_u32(&bars->s));
+                tc_commit(smem_u32(&bars->qfree));
+                ok = mbar_wait_bounded(smem_u32(&bars->pfull), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
+                     (i == 0 || mbar_wait_bounded(smem_u32(&bars->ofree), pph, abort_flag, p.err, ERR_TIMEOUT_ATTN));
+                if (!ok) break;
+                tc_fence_after();
+#pragma unroll
+                for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        tc_mma_bf16(tO, smem_desc_sw128(sb + L::P + kb * L::BOX + kk * 32),
+                                    smem_desc_sw128(sb + L::VT + kb * DH * 128 + kk * 32), idO, (kb | kk) ? 1u : 0u);
+                tc_commit(smem_u32(&bars->o));
+                tc_commit(smem_u32(&bars->pfree));
+            }
+        }
+    } else {
+        // ----------------------------------------------- softmax and epilogue
+        const int qw = warp & 3;                       // TMEM lane quarter
+        const int r = qw * 32 + lane;                  // query row of the tile
+        const uint32_t loff = (uint32_t)(qw * 32) << 16;
+        const int tid = threadIdx.x - 64;              // 0..127
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->kv), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (ok) {
+            // V^T: chunk (8 keys) kc of dimension row dim, from V[key][dim].
+            for (int idx = tid; idx < DH * 16; idx += 128) {
+                const int kc = idx / DH, dim = idx - (idx / DH) * DH;
+                const int db = dim >> 6, dc = (dim & 63) >> 3, de = (dim & 7) * 2;
+                uint32_t w[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int k0 = kc * 8 + 2 * e;
+                    const uint16_t v0 = *reinterpret_cast<const uint16_t*>(
+                        smem + L::V + db * L::BOX + k0 * 128 + ((dc ^ (k0 & 7)) << 4) + de);
+                    const uint16_t v1 = *reinterpret_cast<const uint16_t*>(
+                        smem + L::V + db * L::BOX + (k0 + 1) * 128 + ((dc ^ ((k0 + 1) & 7)) << 4) + de);
+                    w[e] = (uint32_t)v0 | ((uint32_t)v1 << 16);
+                }
+                *reinterpret_cast<uint4*>(smem + L::VT + (kc >> 3) * DH * 128 + dim * 128 +
+                                          (((kc & 7) ^ (dim & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars->vt));
+        }
+        for (int i = 0; i < G && ok; ++i) {
+            const uint32_t ph = i & 1, pph = (i - 1) & 1;
+            if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->s), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            tc_fence_after();
+            // Keys of this warp's rows: 32-key chunks up to the last row's
+            // diagonal (the rest of the row is masked).
+            const int nch = min((qw * 32 + 31) / 32 + 1, (n + 31) / 32);
+            float sv[128];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (c < nch) {
+                    uint32_t u[32];
+                    tmem_ld_32x32(tS + loff + c * 32, u);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) sv[c * 32 + j] = __uint_as_float(u[j]);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars->sfree));
+            // Causal softmax over keys 0..min(r, n - 1); exp(x) as 2^(x log2 e),
+            // one ex2.approx per key (P is rounded to bf16 next).
+            const int kmax = min(r, n - 1);
+            float m = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < nch)
+#pragma unroll
+                    for (int j = c * 32; j < c * 32 + 32; ++j)
+                        if (j <= kmax) m = fmaxf(m, sv[j]);
+            const float sl2 = p.scale * 1.4426950408889634f;
+            const float ms = m * sl2;
+            float l = 0.f;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (c < nch) {
+#pragma unroll
+                    for (int j = c * 32; j < c * 32 + 32; ++j) {
+                        float e;
+                        asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(fmaf(sv[j], sl2, -ms)));
+                        sv[j] = j <= kmax ? e : 0.f;
+                        l += sv[j];
+                    }
+                }
+            }
+            if (i > 0) {
+                if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->pfree), pph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) break;
+            }
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                uint4 w = make_uint4(0u, 0u, 0u, 0u);
+                if (c < nch * 4) {
+                    w.x = pack_bf16x2(sv[c * 8 + 0], sv[c * 8 + 1]);
+                    w.y = pack_bf16x2(sv[c * 8 + 2], sv[c * 8 + 3]);
+                    w.z = pack_bf16x2(sv[c * 8 + 4], sv[c * 8 + 5]);
+                    w.w = pack_bf16x2(sv[c * 8 + 6], sv[c * 8 + 7]);
+                }
+                *reinterpret_cast<uint4*>(smem + L::P + (c >> 3) * L::BOX + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = w;
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars->pfull));
+            // Epilogue: O / l as bf16, rows of the sequence only.
+            if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->o), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) break;
+            tc_fence_after();
+            const float il = 1.f / l;
+            __nv_bfloat16* orow = p.out + (size_t)(t0 + min(r, n - 1)) * p.Hq * DH + (size_t)(g * G + i) * DH;
+#pragma unroll
+            for (int c = 0; c < DH; c += 32) {
+                uint32_t u[32];
+                tmem_ld_32x32(tO + loff + c, u);
+                tmem_ld_wait();
+                if (r < n) {
+                    uint4* d4 = reinterpret_cast<uint4*>(orow + c);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        uint4 w;
+                        w.x = pack_bf16x2(__uint_as_float(u[8 * q4 + 0]) * il, __uint_as_float(u[8 * q4 + 1]) * il);
+                        w.y = pack_bf16x2(__uint_as_float(u[8 * q4 + 2]) * il, __uint_as_float(u[8 * q4 + 3]) * il);
+                        w.z = pack_bf16x2(__uint_as_float(u[8 * q4 + 4]) * il, __uint_as_float(u[8 * q4 + 5]) * il);
+                        w.w = pack_bf16x2(__uint_as_float(u[8 * q4 + 6]) * il, __uint_as_float(u[8 * q4 + 7]) * il);
+                        d4[q4] = w;
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&bars->ofree));
+        }
+    }
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(bars->tmem_base, 256);
+    }
+    pdl_trigger();   // the next kernel may be scheduled once every block got here or exited
 }
 
 }  // namespace
@@ -254,9 +368,9 @@ cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st) 
     return cudaGetLastError();
 }
 
-cudaError_t launch_attention(const AttnParams& p, int head_dim, cudaStream_t st) {
+cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int head_dim, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    if (p.S < 1 || p.S > kSeqMax || p.Hkv < 1 || p.Hq % p.Hkv) return cudaErrorInvalidValue;
+    if (p.S < 1 || p.S > kSeqMax || p.Hkv < 1 || p.Hq % p.Hkv || !tm_qkv) return cudaErrorInvalidValue;
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(attention_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -267,10 +381,11 @@ cudaError_t launch_attention(const AttnParams& p, int head_dim, cudaStream_t st)
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    const dim3 grid(p.Hq, (p.T + p.S - 1) / p.S);
+    const dim3 grid(p.Hkv, (p.T + p.S - 1) / p.S);
     cudaError_t e;
-    if (head_dim == 64) e = launch_pdl(attention_kernel<64>, grid, dim3(128), attn_smem<64>(), st, p);
-    else if (head_dim == 128) e = launch_pdl(attention_kernel<128>, grid, dim3(128), attn_smem<128>(), st, p);
+    if (head_dim == 64) e = launch_pdl(attention_kernel<64>, grid, dim3(kAttnThreads), attn_smem<64>(), st, *tm_qkv, p);
+    else if (head_dim == 128)
+        e = launch_pdl(attention_kernel<128>, grid, dim3(kAttnThreads), attn_smem<128>(), st, *tm_qkv, p);
     else return cudaErrorInvalidValue;
     if (e != cudaSuccess) return e;
     return cudaGetLastError();

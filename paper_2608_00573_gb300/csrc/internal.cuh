@@ -27,7 +27,8 @@ constexpr size_t kMaxTabFloats = (size_t)16 << 20; // 64 MB of shared look-ahead
 constexpr int kGateUp = 128;        // W13 gate/up row interleave
 
 // Device error codes (first one wins).
-enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3, ERR_TIMEOUT_ROUTER = 4 };
+enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3, ERR_TIMEOUT_ROUTER = 4,
+             ERR_TIMEOUT_ATTN = 5 };
 
 // Device-side counters (trimmoe_stats_t is assembled from these).  The handle
 // keeps kCtrCopies copies, each on its own cache lines; a block of the
@@ -184,6 +185,7 @@ struct AttnParams {
     int* goff;                    // [2] {0, T}: the projections' single GEMM group
     const __nv_bfloat16* qkv;     // [T][nqkv] query heads, key heads (rotated), value heads
     __nv_bfloat16* out;           // [T][Hq*Dh] attention output
+    int* err;                     // device error word (bounded waits)
 };
 
 struct CombineParams {
@@ -234,7 +236,8 @@ int grouped_gemm_pair_clusters(int num_sms);
 size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
 cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);
-cudaError_t launch_attention(const AttnParams& p, int head_dim, cudaStream_t st);
+// tm_qkv: the q/k/v rows [T][nqkv] in 128-row x 64-column boxes, 128-byte swizzle.
+cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int head_dim, cudaStream_t st);
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
 
 // Programmatic dependent launch.  The library's kernels are launched with

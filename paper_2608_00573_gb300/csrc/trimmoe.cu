@@ -769,6 +769,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         ap.a = h->Xp;
         ap.goff = h->goff_attn;
         ap.qkv = h->qkv;
+        ap.err = h->dev_err;
         ap.out = h->attn_out;
         e = h->timed(K_ATTN, st, [&] { return launch_attn_norm(ap, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention norm: ") + cudaGetErrorString(e));
@@ -792,7 +793,13 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         qg.tmB_pair = pair_gemm(T) ? &h->tmWqkvp[layer] : nullptr;
         e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(qg, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("qkv gemm: ") + cudaGetErrorString(e));
-        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, c.head_dim, st); });
+        // q/k/v rows of this call only: a sequence's 128-row box reads zeros past T
+        // (never stale or uninitialised rows, which the masked products would
+        // still multiply by zero).
+        CUtensorMap tm_qkv;
+        if (!make_tmap(&tm_qkv, h->qkv, h->nqkv, T, 128))
+            return h->fail(TRIMMOE_ERR_CUDA, "attention: cuTensorMapEncodeTiled failed");
+        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, &tm_qkv, c.head_dim, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(e));
         GemmLaunch og = qg;
         og.rope = nullptr;
