@@ -100,13 +100,15 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
     const int E = p.E, M = p.M, C = p.C, K = p.k, l = p.layer;
     const int ME = M * E;
     const int MC = p.tab.max_layer_cand;
-    // Per-group scratch: logits z[E], probabilities pr[E], head logits x[C],
-    // look-ahead tables V[M*E] and Phi[M*E], staged candidate terms.
-    const size_t per_warp = (size_t)(2 * E + C + 2 * ME + 2 * MC) + (size_t)((MC + 3) / 4) * 2;
-    float* zs = smem + (size_t)slot * per_warp;
+    // Per-group scratch: logits z[E], probabilities pr[E], head logits x[C]
+    // in shared memory; look-ahead tables V[M*E] and Phi[M*E] and the staged
+    // candidate terms after them, or in the group's global slot.
+    const size_t per_head = (size_t)(2 * E + C);
+    const size_t per_la = (size_t)(2 * ME + 2 * MC) + (size_t)((MC + 3) / 4) * 2;
+    float* zs = smem + (size_t)slot * (p.la_scratch ? per_head : per_head + per_la);
     float* ps = zs + E;
     float* xs = ps + E;
-    float* bufV = xs + C;
+    float* bufV = p.la_scratch ? p.la_scratch + ((size_t)blockIdx.x * kGroups + slot) * per_la : xs + C;
     float* bufPhi = bufV + ME;
     float* cqt = bufPhi + ME;                  // omega_D * Q / Dbar, or -1: no quality term
     float* cph = cqt + MC;                     // deeper cost-to-go of the candidate
@@ -559,10 +561,23 @@ cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStre
 // Lanes per token: the smallest group that holds one expert per lane.
 int decide_group(int E) { return E <= 8 ? 8 : E <= 16 ? 16 : 32; }
 
-size_t decide_smem_for(int E, int C, int M, int max_layer_cand, int G) {
+size_t decide_la_floats(int E, int M, int max_layer_cand) {
     const size_t MC = (size_t)max_layer_cand;
-    const size_t per_group = (size_t)(2 * E + C + 2 * M * E) + 2 * MC + ((MC + 3) / 4) * 2;
+    return (size_t)2 * M * E + 2 * MC + ((MC + 3) / 4) * 2;
+}
+
+size_t decide_smem_for(int E, int C, int M, int max_layer_cand, int G, bool la_global = false) {
+    const size_t per_group = (size_t)(2 * E + C) + (la_global ? 0 : decide_la_floats(E, M, max_layer_cand));
     return per_group * sizeof(float) * kWarps * (32 / G);
+}
+
+// Blocks of the decision kernel when the look-ahead scratch is global: at most
+// this many per SM (the register-limited occupancy is six).
+constexpr int kDecideLaBlocksPerSm = 8;
+
+size_t decide_la_scratch_floats(int E, int M, int max_layer_cand, int num_sms) {
+    return (size_t)num_sms * kDecideLaBlocksPerSm * kWarps * (32 / decide_group(E)) *
+           decide_la_floats(E, M, max_layer_cand);
 }
 
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand) {
@@ -575,7 +590,8 @@ cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
     // warps; a small batch keeps a full warp per token for the shortest
     // per-token latency (its look-ahead loops run over M*E entries).
     const int G = p.T >= num_sms * 16 ? decide_group(p.E) : 32;
-    const size_t smem = decide_smem_for(p.E, p.C, p.M, p.tab.max_layer_cand, G);
+    const bool la_global = p.la_scratch != nullptr;
+    const size_t smem = decide_smem_for(p.E, p.C, p.M, p.tab.max_layer_cand, G, la_global);
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(decide_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
@@ -589,7 +605,8 @@ cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
     if (smem > 200 * 1024) return cudaErrorInvalidValue;
     const int per_block = kWarps * (32 / G);
     int blocks = (p.T + per_block - 1) / per_block;
-    blocks = blocks < num_sms * 16 ? blocks : num_sms * 16;
+    const int cap = la_global ? num_sms * kDecideLaBlocksPerSm : num_sms * 16;   // global slots exist for cap blocks
+    blocks = blocks < cap ? blocks : cap;
     cudaError_t e;
     if (G == 8) e = launch_pdl(decide_kernel<8>, dim3(blocks), dim3(kWarps * 32), smem, st, p);
     else if (G == 16) e = launch_pdl(decide_kernel<16>, dim3(blocks), dim3(kWarps * 32), smem, st, p);

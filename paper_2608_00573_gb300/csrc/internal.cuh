@@ -109,6 +109,10 @@ struct DecideParams {
     int dmin;
     float* phi_tabs_out;        // written by the shared-table kernel
     float* dbar_shared_out;
+    // Per-token look-ahead scratch in global memory (one slot per resident
+    // token group), used when the layer has shared tables (most tokens then
+    // read a table and the scratch is rarely touched); NULL: in shared memory.
+    float* la_scratch;
     // Offline-stage calibration counts (Algorithm 1), accumulated when calib != 0.
     int calib;
     int16_t* prev_target;       // [T] slot-0 target at the previous layer, -1 none
@@ -224,6 +228,7 @@ int router_pass_rows(int n_out);
 int router_ksplit(int T, int d, int num_sms);
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand);
+size_t decide_la_scratch_floats(int E, int M, int max_layer_cand, int num_sms);
 cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStream_t st);
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);
 cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,

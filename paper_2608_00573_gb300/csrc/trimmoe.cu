@@ -168,6 +168,7 @@ struct trimmoe {
     DevCounters* ctr = nullptr;
     int* dev_err = nullptr;
     float* splitk = nullptr;          // [8][64][max(n13 F, d)] partial sums of split-K GEMMs
+    float* la_scratch = nullptr;      // per-token look-ahead scratch of the decision kernel (shared-table layers)
     int rows_xp = 0;
 
     CUtensorMap tmXp, tmAct, tmActSh;
@@ -602,6 +603,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     ok = ok && h->dalloc(&h->c_counts, h->n_counts) &&
          h->dalloc(&h->splitk, (size_t)kSplitKMax * kSplitKRows * std::max<size_t>((size_t)h->n13 * c.F, (size_t)d));
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
+    if (ok && tab_floats > 0)
+        ok = h->dalloc(&h->la_scratch, decide_la_scratch_floats(E, M, h->max_layer_cand, h->num_sms));
     const int has_attn = c.attn_heads > 0;
     if (has_attn) {
         h->nqkv = (c.attn_heads + 2 * c.attn_kv_heads) * c.head_dim;
@@ -901,6 +904,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.dmin = top_full - n_depth + 1;
     dp.phi_tabs_out = h->phi_tabs;
     dp.dbar_shared_out = h->dbar_shared;
+    dp.la_scratch = shared_tabs ? h->la_scratch : nullptr;
     dp.calib = h->calib;
     dp.prev_target = h->prev_target;
     dp.c_trans = h->c_counts;
