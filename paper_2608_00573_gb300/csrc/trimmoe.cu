@@ -169,6 +169,10 @@ struct trimmoe {
     int* dev_err = nullptr;
     float* splitk = nullptr;          // [8][64][max(n13 F, d)] partial sums of split-K GEMMs
     float* la_scratch = nullptr;      // per-token look-ahead scratch of the decision kernel (shared-table layers)
+    // Side stream for the shared look-ahead tables: they depend only on the
+    // tables and the budget, so they are computed while the router runs.
+    cudaStream_t aux = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     int rows_xp = 0;
 
     CUtensorMap tmXp, tmAct, tmActSh;
@@ -645,6 +649,9 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
             }
         up(h->rope, rt.data(), rt.size() * sizeof(float2));
     }
+    if (ce == cudaSuccess) ce = cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking);
+    if (ce == cudaSuccess) ce = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
+    if (ce == cudaSuccess) ce = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
     if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies);
     if (ce == cudaSuccess) ce = cudaMemset(h->dev_err, 0, sizeof(int));
     if (ce == cudaSuccess) ce = cudaMemset(h->Xp, 0, (size_t)h->rows_xp * d * 2);
@@ -866,18 +873,6 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         rx.zpart = h->zbuf + E;
         rx.sqpart = h->sqbuf_x;
     }
-    // Hidden rows for the router's TMA loads (128-token x 64-column boxes).
-    CUtensorMap tm_h, tm_hx;
-    if (T > 0 && (!make_tmap(&tm_h, rp.h, d, T, 128) || (has_attn && !make_tmap(&tm_hx, rx.h, d, T, 128))))
-        return h->fail(TRIMMOE_ERR_CUDA, "router: cuTensorMapEncodeTiled failed");
-    e = h->timed(K_ROUTER, st, [&] {
-        cudaError_t e2 = launch_router(&tm_h, &h->tmRhi[layer], &h->tmRlo[layer], rp, h->num_sms, st);
-        return (e2 == cudaSuccess && has_attn)
-                   ? launch_router(&tm_hx, &h->tmRxhi[layer], nullptr, rx, h->num_sms, st)
-                   : e2;
-    });
-    if (has_attn) h->launches += 1;
-    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("router: ") + cudaGetErrorString(e));
     dp.zpart = h->zbuf;
     dp.sqpart = h->sqbuf;
     dp.sqpart_x = has_attn ? h->sqbuf_x : nullptr;
@@ -941,9 +936,36 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.tab.eps = h->eps;
     dp.ctr = h->ctr;
 
+    // Shared look-ahead tables: light ones (M*E <= 256) on the side stream,
+    // overlapping the router; heavy ones in line after it (run beside the
+    // issue-bound router they slowed it more than they saved: Qwen-shaped,
+    // M*E = 600, 23.5 -> 24.7 ms per forward; Switch-shaped 1.47 -> 1.40 ms).
+    const bool tabs_aside = shared_tabs && c.M * E <= 256;
+    if (tabs_aside) {
+        e = cudaEventRecord(h->ev_fork, st);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(h->aux, h->ev_fork, 0);
+        if (e == cudaSuccess) e = launch_lookahead_shared(dp, n_depth, h->aux);
+        if (e == cudaSuccess) e = cudaEventRecord(h->ev_join, h->aux);
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("look-ahead tables: ") + cudaGetErrorString(e));
+    }
+    // Hidden rows for the router's TMA loads (128-token x 64-column boxes).
+    CUtensorMap tm_h, tm_hx;
+    if (T > 0 && (!make_tmap(&tm_h, rp.h, d, T, 128) || (has_attn && !make_tmap(&tm_hx, rx.h, d, T, 128))))
+        return h->fail(TRIMMOE_ERR_CUDA, "router: cuTensorMapEncodeTiled failed");
+    e = h->timed(K_ROUTER, st, [&] {
+        cudaError_t e2 = launch_router(&tm_h, &h->tmRhi[layer], &h->tmRlo[layer], rp, h->num_sms, st);
+        return (e2 == cudaSuccess && has_attn)
+                   ? launch_router(&tm_hx, &h->tmRxhi[layer], nullptr, rx, h->num_sms, st)
+                   : e2;
+    });
+    if (has_attn) h->launches += 1;
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("router: ") + cudaGetErrorString(e));
+    if (tabs_aside) {
+        e = cudaStreamWaitEvent(st, h->ev_join, 0);
+        if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("look-ahead join: ") + cudaGetErrorString(e));
+    }
     e = h->timed(K_DECIDE, st, [&] {
-        cudaError_t e2 = cudaSuccess;
-        if (shared_tabs) e2 = launch_lookahead_shared(dp, n_depth, st);
+        cudaError_t e2 = (shared_tabs && !tabs_aside) ? launch_lookahead_shared(dp, n_depth, st) : cudaSuccess;
         return e2 == cudaSuccess ? launch_decide(dp, h->num_sms, st) : e2;
     });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("decide: ") + cudaGetErrorString(e));
@@ -1541,6 +1563,9 @@ extern "C" void trimmoe_destroy(trimmoe_handle h) {
     h->drain_events();
     h->drop_graph();
     for (cudaEvent_t e : h->ev_free) cudaEventDestroy(e);
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    if (h->ev_join) cudaEventDestroy(h->ev_join);
+    if (h->aux) cudaStreamDestroy(h->aux);
     for (void* p : h->allocs) cudaFree(p);
     delete h;
 }
