@@ -20,13 +20,13 @@
 // operand), and the diagonal of that 16 x 16 Gram block is each token's
 // partial sum of h^2.
 //
-// Design (persistent, 288 threads per CTA):
+// Design (persistent, 288 threads per CTA, two CTAs per SM):
 //   warp 8      producer (one lane): per 64-column slab, 2-D TMA boxes of the
 //               128-token hidden tile and of the pass's weight rows (hi and
 //               lo), 128-byte swizzle, rows past the tensor zero-filled, into a
 //               ring of 2-8 stages guarded by full/empty mbarriers
 //   warps 0-7   16 tokens each: ldmatrix + mma.sync m16n8k16 (bf16 in, fp32
-//               accumulate), up to 128 output rows per pass over h
+//               accumulate), up to 32 output rows per pass over h
 // Hidden rows of dead tokens are loaded with their tile but never stored.
 // Every wait is bounded (2 s); on expiry the kernel records an error word and
 // returns.
@@ -40,7 +40,7 @@ namespace {
 
 constexpr int kTok = 128;         // tokens per tile (8 consumer warps x 16)
 constexpr int kKS = 64;           // columns per slab (one 128-byte row per token / weight)
-constexpr int kNG = 128;          // largest number of outputs per pass (16 n-tiles of 8)
+constexpr int kNG = 32;           // largest number of outputs per pass (4 n-tiles of 8)
 constexpr int kConsumers = kTok / 16;
 constexpr int kThreads = 32 * (kConsumers + 1);
 constexpr int kA = kTok * kKS * 2;     // 16 KB hidden slab, 128-byte swizzled
@@ -58,13 +58,12 @@ __host__ __device__ __forceinline__ size_t stage_bytes(int ng, int nl) {
     return (size_t)kA + (size_t)(ng + nl) * kKS * 2;
 }
 
-// Shared memory per CTA: two CTAs per SM with up to 4 n-tiles per pass, one
-// with 8 or more (the accumulators need the registers of the whole SM).
-size_t smem_budget(int nt) { return nt <= 4 ? 100 * 1024 : 200 * 1024; }
+// Shared memory per CTA: two CTAs per SM.
+constexpr size_t kSmemBudget = 100 * 1024;
 
-int stages_for(int ng, int nl, int nt) {
+int stages_for(int ng, int nl) {
     const size_t sb = stage_bytes(ng, nl);
-    const int s = (int)((smem_budget(nt) - 1024 - sizeof(RouterBars)) / sb);
+    const int s = (int)((kSmemBudget - 1024 - sizeof(RouterBars)) / sb);
     return std::max(2, std::min(kMaxStages, s));
 }
 
@@ -78,9 +77,9 @@ __device__ __forceinline__ uint32_t sw128(uint32_t base, int r, int c) {
 }
 
 // NT: n-tiles of 8 outputs per pass (ng = 8 NT rows, the last ones past n_out
-// zero-filled by TMA and never stored).
+// zero-filled by TMA and never stored): 1, 2 or 4.
 template <int NT>
-__global__ void __launch_bounds__(kThreads, NT <= 4 ? 2 : 1)
+__global__ void __launch_bounds__(kThreads, 2)
 router_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmBhi,
               const __grid_constant__ CUtensorMap tmBlo, const RouterParams p, int stages) {
     extern __shared__ uint8_t smem_raw[];
@@ -158,7 +157,7 @@ router_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             a_off[kk] = (uint32_t)(ar * 128 + (((kk * 2 + (lane >> 4)) ^ (ar & 7)) << 4));
             b_off[kk] = (uint32_t)(br * 128 + (((kk * 2 + ((lane >> 3) & 1)) ^ br) << 4));
         }
-        const int nlt = NL / 8;                 // n-tiles with a lo part (pass 0)
+        const int nlt = NL / 8;                 // n-tiles with a lo part in a pass
         int it = 0;
         for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
             const int pass = u / (ntile * p.ksplit);
@@ -167,7 +166,7 @@ router_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             const int kr = rem - tile * p.ksplit;
             const int ng0 = pass * NG;
             const int nrows = min(NG, p.n_out - ng0);
-            const int lo_t = (pass == 0 && ng0 < p.n_lo) ? nlt : 0;
+            const int lo_t = ng0 < p.n_lo ? min(nlt, (p.n_lo - ng0 + 7) / 8) : 0;
             float acc[NT][4];
 #pragma unroll
             for (int j = 0; j < NT; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
@@ -261,11 +260,12 @@ int router_ksplit(int T, int d, int num_sms) {
     return ks;
 }
 
-// Rows per pass: n-tiles of 8 rounded up to 1, 2, 4, 8, 12 or 16 (the kernel's
-// register tile), at most 128.
+// Rows per pass: n-tiles of 8 rounded up to 1, 2 or 4 (the kernel's register
+// tile), at most 32: wider passes need the registers of a whole SM per CTA,
+// and a second CTA per SM (plus a re-read of h per extra pass) was faster.
 int router_pass_rows(int n_out) {
     const int t = (n_out + 7) / 8;
-    const int nt = t <= 1 ? 1 : t <= 2 ? 2 : t <= 4 ? 4 : t <= 8 ? 8 : t <= 12 ? 12 : 16;
+    const int nt = t <= 1 ? 1 : t <= 2 ? 2 : 4;
     return nt * 8;
 }
 
@@ -278,38 +278,24 @@ cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, cons
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaSuccess;
-        auto set = [&](const void* f, int nt) {
-            if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_budget(nt));
-        };
-        set((const void*)router_kernel<1>, 1);
-        set((const void*)router_kernel<2>, 2);
-        set((const void*)router_kernel<4>, 4);
-        set((const void*)router_kernel<8>, 8);
-        set((const void*)router_kernel<12>, 12);
-        set((const void*)router_kernel<16>, 16);
+        for (const void* f : {(const void*)router_kernel<1>, (const void*)router_kernel<2>, (const void*)router_kernel<4>})
+            if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBudget);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
     const int nt = p.ng / 8;
-    if (nt != 1 && nt != 2 && nt != 4 && nt != 8 && nt != 12 && nt != 16) return cudaErrorInvalidValue;
-    const int stages = stages_for(p.ng, p.nl, nt);
+    if (nt != 1 && nt != 2 && nt != 4) return cudaErrorInvalidValue;
+    const int stages = stages_for(p.ng, p.nl);
     const size_t smem = smem_for(p.ng, p.nl, stages);
     const int ntile = (p.T + kTok - 1) / kTok;
     const int npass = (p.n_out + p.ng - 1) / p.ng;
     const long long units = (long long)ntile * p.ksplit * npass;
-    const int per_sm = nt <= 4 ? 2 : 1;
-    const int grid = (int)std::min<long long>(units, (long long)per_sm * num_sms);
+    const int grid = (int)std::min<long long>(units, 2LL * num_sms);
     const CUtensorMap* lo = p.nl > 0 ? tmBlo : tmBhi;
     cudaError_t e;
-    switch (nt) {
-        case 1: e = launch_pdl(router_kernel<1>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
-        case 2: e = launch_pdl(router_kernel<2>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
-        case 4: e = launch_pdl(router_kernel<4>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
-        case 8: e = launch_pdl(router_kernel<8>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
-        case 12: e = launch_pdl(router_kernel<12>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
-        default: e = launch_pdl(router_kernel<16>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages); break;
-    }
+    if (nt == 1) e = launch_pdl(router_kernel<1>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages);
+    else if (nt == 2) e = launch_pdl(router_kernel<2>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages);
+    else e = launch_pdl(router_kernel<4>, dim3(grid), dim3(kThreads), smem, st, *tmA, *tmBhi, *lo, p, stages);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
