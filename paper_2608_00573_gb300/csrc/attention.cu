@@ -21,21 +21,22 @@
 // host-made cos/sin table) is applied by the projection GEMM's epilogue to the
 // fp32 accumulators before their bf16 rounding.
 //
-// attention_kernel: one CTA per (key/value head, sequence), 192 threads, on
+// attention_kernel: one CTA per (key/value head, sequence), 320 threads, on
 // the 5th-generation tensor cores.  S <= 128 keys fit one tile, so there is no
 // running maximum: per query head of the group
 //   S = Q K^T          tcgen05.mma M = 128 (queries), N = 128 (keys), K = Dh -> TMEM
 //   P = exp(scale (S - max))   causal mask, fp32 (exp as one ex2.approx per
-//                      key), rounded to bf16 into shared memory by the 128
-//                      softmax threads (one query row each; a warp skips the
-//                      32-key chunks above its rows' diagonal)
+//                      key), rounded to bf16 into shared memory by the 256
+//                      softmax threads (two per query row, one per key half;
+//                      a warp skips the 32-key chunks above its rows' diagonal)
 //   O = P V            tcgen05.mma M = 128, N = Dh, K = 128 keys -> TMEM
 //   out = bf16(O / l)  l = the fp32 row sum of the unrounded probabilities
 // warp 0 loads K and V of the group once and the query heads one after another
-// (TMA, 128-byte swizzle); warp 1 issues the MMAs; warps 2-5 transpose V once
+// (TMA, 128-byte swizzle); warp 1 issues the MMAs; warps 2-9 transpose V once
 // into a K-major tile (keys contiguous, so that every operand is K-major), then
-// run the softmax and the epilogue of each head while the tensor core computes
-// the next head's scores.  Rows past the sequence are loaded (the next
+// run the softmax and the epilogue of each head (two warps per 32 query rows,
+// one per half of the keys) while the tensor core computes the next head's
+// scores.  Rows past the sequence are loaded (the next
 // sequence's rows, or zero fill) but masked as keys and never stored as
 // queries.  Every wait is bounded (2 s) and records an error word on expiry.
 #include "internal.cuh"
@@ -100,7 +101,7 @@ __global__ void __launch_bounds__(256) attn_norm_kernel(const AttnParams p) {
     }
 }
 
-constexpr int kAttnThreads = 192;
+constexpr int kAttnThreads = 320;            // load warp, MMA warp, 8 softmax / epilogue warps
 
 // Shared-memory layout (byte offsets from a 1024-aligned base).  A box is 128
 // rows x 64 bf16 columns (16 KB, 128-byte rows, 128-byte swizzle).
@@ -113,11 +114,13 @@ struct AttnLayout {
     static constexpr int V = K + KB * BOX;                // as loaded: [KB][128 key rows][64 dims]
     static constexpr int VT = V + KB * BOX;               // [2 key blocks][DH dim rows][64 keys]
     static constexpr int P = VT + 2 * DH * 128;           // [2 key blocks][128 query rows][64 keys]
-    static constexpr int BYTES = P + 2 * BOX;
+    static constexpr int X = P + 2 * BOX;                 // row maxima and sums of the two key halves
+    static constexpr int BYTES = X + 4 * 128 * 4;
 };
 
 struct __align__(8) AttnBars {
     uint64_t kv, q, vt, s, sfree, pfull, pfree, o, ofree, qfree;
+    uint64_t pair[4];          // the two softmax warps of a TMEM lane quarter
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -147,13 +150,14 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
     if (threadIdx.x == 0) {
         mbar_init(smem_u32(&bars->kv), 1);
         mbar_init(smem_u32(&bars->q), 1);
-        mbar_init(smem_u32(&bars->vt), 4);
+        mbar_init(smem_u32(&bars->vt), 8);
         mbar_init(smem_u32(&bars->s), 1);
-        mbar_init(smem_u32(&bars->sfree), 4);
-        mbar_init(smem_u32(&bars->pfull), 4);
+        mbar_init(smem_u32(&bars->sfree), 8);
+        mbar_init(smem_u32(&bars->pfull), 8);
         mbar_init(smem_u32(&bars->pfree), 1);
         mbar_init(smem_u32(&bars->o), 1);
-        mbar_init(smem_u32(&bars->ofree), 4);
+        mbar_init(smem_u32(&bars->ofree), 8);
+        for (int j = 0; j < 4; ++j) mbar_init(smem_u32(&bars->pair[j]), 2);
         mbar_init(smem_u32(&bars->qfree), 1);
         bars->abort_flag = 0;
         fence_barrier_init();
@@ -222,16 +226,35 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
         }
     } else {
         // ----------------------------------------------- softmax and epilogue
-        const int qw = warp & 3;                       // TMEM lane quarter
-        const int r = qw * 32 + lane;                  // query row of the tile
+        // Eight warps: warps w and w + 4 share TMEM lane quarter qw = w & 3 (32
+        // query rows) and take the key halves hk = 0 and 1; a row's maximum
+        // and sum combine the halves through shared memory (a two-arrival
+        // mbarrier per quarter, bounded waits), and the epilogue splits O's
+        // columns the same way.
+        const int qw = warp & 3;
+        const int hk = (warp - 2) >> 2;
+        const int r = qw * 32 + lane;
         const uint32_t loff = (uint32_t)(qw * 32) << 16;
-        const int tid = threadIdx.x - 64;              // 0..127
+        const int tid = threadIdx.x - 64;              // 0..255
+        float* xmax = reinterpret_cast<float*>(smem + L::X);     // [2][128]
+        float* xsum = xmax + 256;                                // [2][128]
+        const uint32_t pbar = smem_u32(&bars->pair[qw]);
         int ok = 1;
+        // Both warps of the pair write, then wait for the pair (phase u of use k).
+        auto pair_sync = [&](uint32_t parity) -> int {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(pbar);
+            int w = 1;
+            if (lane == 0) w = mbar_wait_bounded(pbar, parity, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+            w = __shfl_sync(0xffffffffu, w, 0);
+            __syncwarp();
+            return w;
+        };
         if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->kv), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (ok) {
             // V^T: chunk (8 keys) kc of dimension row dim, from V[key][dim].
-            for (int idx = tid; idx < DH * 16; idx += 128) {
+            for (int idx = tid; idx < DH * 16; idx += 256) {
                 const int kc = idx / DH, dim = idx - (idx / DH) * DH;
                 const int db = dim >> 6, dc = (dim & 63) >> 3, de = (dim & 7) * 2;
                 uint32_t w[4];
@@ -251,51 +274,54 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bars->vt));
         }
+        const float sl2 = p.scale * 1.4426950408889634f;
+        const int kmax = min(r, n - 1);
+        // 32-key chunks of this warp's half that some row of the quarter needs.
+        const int kq = min(qw * 32 + 31, n - 1);
         for (int i = 0; i < G && ok; ++i) {
             const uint32_t ph = i & 1, pph = (i - 1) & 1;
             if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->s), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (!ok) break;
             tc_fence_after();
-            // Keys of this warp's rows: 32-key chunks up to the last row's
-            // diagonal (the rest of the row is masked).
-            const int nch = min((qw * 32 + 31) / 32 + 1, (n + 31) / 32);
-            float sv[128];
+            float sv[64];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c < nch) {
+            for (int cc = 0; cc < 2; ++cc) {
+                if ((2 * hk + cc) * 32 <= kq) {
                     uint32_t u[32];
-                    tmem_ld_32x32(tS + loff + c * 32, u);
+                    tmem_ld_32x32(tS + loff + (2 * hk + cc) * 32, u);
                     tmem_ld_wait();
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) sv[c * 32 + j] = __uint_as_float(u[j]);
+                    for (int j = 0; j < 32; ++j) sv[cc * 32 + j] = __uint_as_float(u[j]);
                 }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bars->sfree));
-            // Causal softmax over keys 0..min(r, n - 1); exp(x) as 2^(x log2 e),
-            // one ex2.approx per key (P is rounded to bf16 next).
-            const int kmax = min(r, n - 1);
+            // Causal softmax over keys 0..kmax; exp(x) as 2^(x log2 e), one
+            // ex2.approx per key (P is rounded to bf16 next).
             float m = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < nch)
+            for (int cc = 0; cc < 2; ++cc)
+                if ((2 * hk + cc) * 32 <= kq)
 #pragma unroll
-                    for (int j = c * 32; j < c * 32 + 32; ++j)
-                        if (j <= kmax) m = fmaxf(m, sv[j]);
-            const float sl2 = p.scale * 1.4426950408889634f;
+                    for (int j = 0; j < 32; ++j)
+                        if (64 * hk + cc * 32 + j <= kmax) m = fmaxf(m, sv[cc * 32 + j]);
+            xmax[hk * 128 + r] = m;
+            ok = pair_sync(0);
+            if (!ok) break;
+            m = fmaxf(xmax[r], xmax[128 + r]);
             const float ms = m * sl2;
             float l = 0.f;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c < nch) {
+            for (int cc = 0; cc < 2; ++cc) {
+                if ((2 * hk + cc) * 32 <= kq) {
 #pragma unroll
-                    for (int j = c * 32; j < c * 32 + 32; ++j) {
+                    for (int j = 0; j < 32; ++j) {
                         float e;
-                        asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(fmaf(sv[j], sl2, -ms)));
-                        sv[j] = j <= kmax ? e : 0.f;
-                        l += sv[j];
+                        asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(fmaf(sv[cc * 32 + j], sl2, -ms)));
+                        sv[cc * 32 + j] = (64 * hk + cc * 32 + j <= kmax) ? e : 0.f;
+                        l += sv[cc * 32 + j];
                     }
                 }
             }
@@ -305,28 +331,31 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
                 if (!ok) break;
             }
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
+            for (int c = 0; c < 8; ++c) {
                 uint4 w = make_uint4(0u, 0u, 0u, 0u);
-                if (c < nch * 4) {
+                if ((2 * hk + (c >> 2)) * 32 <= kq) {
                     w.x = pack_bf16x2(sv[c * 8 + 0], sv[c * 8 + 1]);
                     w.y = pack_bf16x2(sv[c * 8 + 2], sv[c * 8 + 3]);
                     w.z = pack_bf16x2(sv[c * 8 + 4], sv[c * 8 + 5]);
                     w.w = pack_bf16x2(sv[c * 8 + 6], sv[c * 8 + 7]);
                 }
-                *reinterpret_cast<uint4*>(smem + L::P + (c >> 3) * L::BOX + r * 128 + (((c & 7) ^ (r & 7)) << 4)) = w;
+                *reinterpret_cast<uint4*>(smem + L::P + hk * L::BOX + r * 128 + ((c ^ (r & 7)) << 4)) = w;
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&bars->pfull));
-            // Epilogue: O / l as bf16, rows of the sequence only.
+            xsum[hk * 128 + r] = l;
+            // Epilogue: O / l as bf16, this half's columns, rows of the sequence only.
             if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->o), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (!ok) break;
+            ok = pair_sync(1);
+            if (!ok) break;
             tc_fence_after();
-            const float il = 1.f / l;
+            const float il = 1.f / (xsum[r] + xsum[128 + r]);
             __nv_bfloat16* orow = p.out + (size_t)(t0 + min(r, n - 1)) * p.Hq * DH + (size_t)(g * G + i) * DH;
 #pragma unroll
-            for (int c = 0; c < DH; c += 32) {
+            for (int c = hk * (DH / 2); c < (hk + 1) * (DH / 2); c += 32) {
                 uint32_t u[32];
                 tmem_ld_32x32(tO + loff + c, u);
                 tmem_ld_wait();
