@@ -251,6 +251,16 @@ def test_layer_parity_pair_gemm(name, kw):
     assert tot["exec"] > 0
 
 
+def test_layer_parity_decision_lane_groups_of_16():
+    """8 < E <= 16 with more tokens than the resident warps (T >= 16 x SMs):
+    the decision kernel runs two tokens per warp on 16-lane groups."""
+    cfg = small_cfg(name="g16", N=2, d=256, E=16, k=2, F=128, T=2600, M=10, H=3, seed=99)
+    reports = _run_all_layers(cfg, theta=0.9, exit_bias=1.0, row_sample=np.arange(0, 2600, 5))
+    tot = {k: sum(r[k] for r in reports) for k in ("exec", "skip", "exit")}
+    print("g16", tot)
+    assert tot["exec"] > 0 and tot["skip"] > 0 and tot["exit"] > 0, tot
+
+
 @pytest.mark.parametrize("budget", [0.0, float("inf")])
 def test_budget_edge_cases(budget):
     """Dbar = 0: only exact execution fits (Q = 0), no skip; Dbar = inf: every
