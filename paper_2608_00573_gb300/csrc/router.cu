@@ -11,20 +11,20 @@
 //
 // The router's gamma * W_r products are exact in fp32 and split exactly into
 // two bf16 matrices (hi + lo), so two bf16 MMAs give the logits without
-// rounding the normalised input.  Each 16-wide k step starts its MMA from zero
-// and its partial is added to IEEE fp32 registers (__fadd_rn): the tensor
-// core's own accumulation then only touches sums of 16-32 exact products, which
-// keeps the logits at fp32 accuracy (the decisions compare them to 1e-5).
-// The sum of squares comes from the same fragments: two more MMAs per k step
-// multiply the 16-token A fragment by itself (its rows reused as the B
-// operand), and the diagonal of that 16 x 16 Gram block is each token's
-// partial sum of h^2.
+// rounding the normalised input.  Each 64-column slab starts its MMAs from
+// zero and the slab's sums are added to IEEE fp32 registers (__fadd_rn): the
+// tensor core's own accumulation then only touches sums of 64 (hi) + 64 (lo)
+// exact products, which keeps the logits at fp32 accuracy (the decisions
+// compare them to 1e-5).  The sum of squares comes from the same fragments:
+// two more MMAs per 16-column step multiply the 16-token A fragment by itself
+// (its rows reused as the B operand), and the diagonal of the resulting 16 x 16
+// Gram block is each token's partial sum of h^2.
 //
 // Design (persistent, 288 threads per CTA, two CTAs per SM):
 //   warp 8      producer (one lane): per 64-column slab, 2-D TMA boxes of the
 //               128-token hidden tile and of the pass's weight rows (hi and
 //               lo), 128-byte swizzle, rows past the tensor zero-filled, into a
-//               ring of 2-8 stages guarded by full/empty mbarriers
+//               ring of up to 8 stages guarded by full/empty mbarriers
 //   warps 0-7   16 tokens each: ldmatrix + mma.sync m16n8k16 (bf16 in, fp32
 //               accumulate), up to 32 output rows per pass over h
 // Hidden rows of dead tokens are loaded with their tile but never stored.
