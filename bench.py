@@ -408,7 +408,7 @@ def run_ours(args):
 
 # Revision tag of the timed GEMM kernel; a stored ncu traffic figure is used
 # only when it was taken on this revision.
-KERNEL_REV = "gemm-v6"
+KERNEL_REV = "gemm-v7"
 
 
 def main():

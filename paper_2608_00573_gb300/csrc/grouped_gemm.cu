@@ -621,7 +621,9 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     // a block stays resident while the weight tiles stream past it.
     const long long a_tile_bytes = (long long)BM * g.K * 2;
     if (g.tmB_pair && (g.ksplit <= 1) && pair_clusters(num_sms) > 0) {
-        const int mblk2 = (int)std::max(1LL, (48LL << 20) / (2 * a_tile_bytes));
+        // Row-pair tiles per block: about 32 MB of activations (same speed as
+        // 40 or 48 MB within the run-to-run spread, fewest DRAM re-reads).
+        const int mblk2 = (int)std::max(1LL, (32LL << 20) / (2 * a_tile_bytes));
         const cudaError_t e = launch_pdl(
             grouped_gemm_pair_kernel, dim3(2 * pair_clusters(num_sms)), dim3(kThreads), kPairSmemBytes, st, *g.tmA,
             *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
