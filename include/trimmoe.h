@@ -20,8 +20,8 @@
  *    dense, row-major, with the shapes given in brackets.
  *  - Layers, experts, servers and tokens are 0-based.
  *  - Calls are asynchronous on the given stream (a cudaStream_t passed as
- *    void*, NULL = legacy default stream) except trimmoe_stats and
- *    trimmoe_forward_host, which synchronise.  A handle must not be used by
+ *    void*, NULL = legacy default stream) except trimmoe_stats,
+ *    trimmoe_forward_host and trimmoe_watchdog_selftest, which synchronise.  A handle must not be used by
  *    two streams or two host threads at the same time: its workspaces are
  *    shared by all its calls.
  */
@@ -47,6 +47,20 @@ typedef enum {
 typedef struct trimmoe* trimmoe_handle;
 
 /* Actions written to trimmoe_layer_out.action (Sec. V-A). */
+/* Which bounded device wait ran out first (trimmoe_stats_t.device_error).
+ * Every wait of a kernel on an mbarrier or a flag has a time limit; the first
+ * one to run out writes its code, makes the other roles of its CTA return, and
+ * the kernel ends normally, so the CUDA context stays usable. */
+enum {
+    TRIMMOE_DEVERR_NONE = 0,
+    TRIMMOE_DEVERR_GEMM_PRODUCER = 1,  /* grouped GEMM: TMA producer waiting for a free stage */
+    TRIMMOE_DEVERR_GEMM_MMA = 2,       /* grouped GEMM: MMA issuer waiting for operands or TMEM */
+    TRIMMOE_DEVERR_GEMM_EPILOGUE = 3,  /* grouped GEMM: epilogue waiting for an accumulator */
+    TRIMMOE_DEVERR_ROUTER = 4,         /* router logits kernel */
+    TRIMMOE_DEVERR_ATTENTION = 5,      /* attention kernel (including its softmax pair barriers) */
+    TRIMMOE_DEVERR_SELFTEST = 6        /* trimmoe_watchdog_selftest */
+};
+
 enum { TRIMMOE_EXEC = 0, TRIMMOE_SKIP = 1, TRIMMOE_EXIT = 2, TRIMMOE_DEAD = 3 };
 
 /* Model and policy hyper-parameters.
@@ -225,7 +239,7 @@ typedef struct {
     double delay_ms;              /* sum of d(m, k) of Eq. (30) over executed pairs */
     double remote_hops;           /* executed pairs on a server other than s */
     float max_budget_ratio;       /* max Dhat / Dbar seen after a decision */
-    int device_error;             /* non-zero if a kernel flagged a timeout */
+    int device_error;             /* 0, or the TRIMMOE_DEVERR_* code of the first wait that ran out */
     uint64_t launches;            /* kernels launched by the library */
     uint64_t layer_calls;         /* layers processed */
     double gemm_flops;            /* 2*M*N*K of the grouped FFN GEMMs that ran */
@@ -277,6 +291,19 @@ trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out);
 
 /* Zero the counters and the device error flag (synchronises). */
 trimmoe_status trimmoe_reset_stats(trimmoe_handle h);
+
+/* Failure-detection self-check of the bounded device waits.  Launches one
+ * kernel on stream whose mbarrier never receives an arrival: warp 0 waits on
+ * it with a limit of timeout_us microseconds (1 ... 1000000), runs out, raises
+ * the CTA's abort flag and writes TRIMMOE_DEVERR_SELFTEST to the handle's
+ * device error word; warp 1 waits on the same barrier with the kernels' normal
+ * two-second limit and returns as soon as it sees the abort.  The call then
+ * synchronises the stream and reads the word back.
+ * Returns DEVICE_TIMEOUT when the wait ran out as designed (the flag stays set,
+ * and trimmoe_stats reports it, until trimmoe_reset_stats), OK if the word was
+ * not set, ARG for a NULL handle or a limit out of range, CUDA if the launch
+ * failed.  The handle stays usable afterwards. */
+trimmoe_status trimmoe_watchdog_selftest(trimmoe_handle h, int timeout_us, void* stream);
 
 /* Last error message of the handle ("" if none); NULL handle: the last error of
  * a call made without a handle (trimmoe_create, trimmoe_compact_noalloc). */

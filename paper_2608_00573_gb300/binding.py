@@ -99,7 +99,7 @@ class trimmoe_calibration_t(C.Structure):
 EXPORTS = ("trimmoe_create", "trimmoe_layer_step", "trimmoe_forward", "trimmoe_forward_host",
            "trimmoe_stats", "trimmoe_reset_stats", "trimmoe_last_error", "trimmoe_destroy",
            "trimmoe_compact_noalloc", "trimmoe_feedback", "trimmoe_calibration_begin",
-           "trimmoe_calibration_end", "trimmoe_replicate")
+           "trimmoe_calibration_end", "trimmoe_replicate", "trimmoe_watchdog_selftest")
 
 _lib = None
 _lock = threading.Lock()
@@ -127,6 +127,8 @@ def lib():
             L.trimmoe_stats.restype = i
             L.trimmoe_reset_stats.argtypes = [vp]
             L.trimmoe_reset_stats.restype = i
+            L.trimmoe_watchdog_selftest.argtypes = [vp, i, vp]
+            L.trimmoe_watchdog_selftest.restype = i
             L.trimmoe_last_error.argtypes = [vp]
             L.trimmoe_last_error.restype = C.c_char_p
             L.trimmoe_destroy.argtypes = [vp]
@@ -183,6 +185,12 @@ def trimmoe_stats(h) -> dict:
 
 def trimmoe_reset_stats(h):
     _check(lib().trimmoe_reset_stats(h), h)
+
+
+def trimmoe_watchdog_selftest(h, timeout_us: int, stream: int = 0) -> int:
+    """Run the bounded-wait self-check; returns the status code (DEVICE_TIMEOUT when the
+    wait ran out as designed) instead of raising."""
+    return lib().trimmoe_watchdog_selftest(h, timeout_us, C.c_void_p(stream))
 
 
 def trimmoe_last_error(h=None) -> str:

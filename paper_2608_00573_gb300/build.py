@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libtrimmoe.so")
 SOURCES = ["trimmoe.cu", "router.cu", "decide.cu", "compact.cu", "grouped_gemm.cu", "combine.cu", "attention.cu",
-           "feedback.cu"]
+           "feedback.cu", "watchdog.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

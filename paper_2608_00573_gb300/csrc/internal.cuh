@@ -26,9 +26,11 @@ constexpr size_t kMaxIntervals = 4096;            // shared look-ahead tables pe
 constexpr size_t kMaxTabFloats = (size_t)16 << 20; // 64 MB of shared look-ahead tables
 constexpr int kGateUp = 128;        // W13 gate/up row interleave
 
-// Device error codes (first one wins).
-enum : int { ERR_NONE = 0, ERR_TIMEOUT_PRODUCER = 1, ERR_TIMEOUT_MMA = 2, ERR_TIMEOUT_EPI = 3, ERR_TIMEOUT_ROUTER = 4,
-             ERR_TIMEOUT_ATTN = 5 };
+// Device error codes (first one wins); the public TRIMMOE_DEVERR_* values.
+enum : int { ERR_NONE = TRIMMOE_DEVERR_NONE, ERR_TIMEOUT_PRODUCER = TRIMMOE_DEVERR_GEMM_PRODUCER,
+             ERR_TIMEOUT_MMA = TRIMMOE_DEVERR_GEMM_MMA, ERR_TIMEOUT_EPI = TRIMMOE_DEVERR_GEMM_EPILOGUE,
+             ERR_TIMEOUT_ROUTER = TRIMMOE_DEVERR_ROUTER, ERR_TIMEOUT_ATTN = TRIMMOE_DEVERR_ATTENTION,
+             ERR_TIMEOUT_SELFTEST = TRIMMOE_DEVERR_SELFTEST };
 
 // Device-side counters (trimmoe_stats_t is assembled from these).  The handle
 // keeps kCtrCopies copies, each on its own cache lines; a block of the
@@ -244,6 +246,7 @@ cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);
 // tm_qkv: the q/k/v rows [T][nqkv] in 128-row x 64-column boxes, 128-byte swizzle.
 cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int head_dim, cudaStream_t st);
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
+cudaError_t launch_watchdog_selftest(int* err, uint64_t limit_ns, cudaStream_t st);
 
 // Programmatic dependent launch.  The library's kernels are launched with
 // programmatic stream serialisation: a kernel may be scheduled while the
@@ -318,18 +321,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait: gives up after kTimeoutNs, raising the CTA abort flag and the
-// device error word; also returns early once another role has aborted.
+// Bounded wait: gives up after limit_ns (kTimeoutNs by default), raising the
+// CTA abort flag and the device error word; also returns early once another
+// role has aborted.
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
-                                                  volatile int* abort_flag, int* err, int code) {
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                                  int* err, int code, uint64_t limit_ns = kTimeoutNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > kTimeoutNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             *abort_flag = 1;
             atomicCAS(err, 0, code);
             return false;

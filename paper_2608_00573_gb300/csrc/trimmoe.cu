@@ -1374,6 +1374,24 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
     return TRIMMOE_OK;
 }
 
+extern "C" trimmoe_status trimmoe_watchdog_selftest(trimmoe_handle h, int timeout_us, void* stream) {
+    if (!h) return TRIMMOE_ERR_ARG;
+    if (timeout_us < 1 || timeout_us > 1000000) return h->fail(TRIMMOE_ERR_ARG, "watchdog_selftest: timeout_us out of range");
+    DeviceGuard g(h->dev);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    h->last_stream = st;
+    if (launch_watchdog_selftest(h->dev_err, (uint64_t)timeout_us * 1000ull, st) != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, std::string("watchdog_selftest: ") + cudaGetErrorString(cudaGetLastError()));
+    h->launches += 1;
+    int derr = 0;
+    if (cudaStreamSynchronize(st) != cudaSuccess ||
+        cudaMemcpy(&derr, h->dev_err, sizeof derr, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, std::string("watchdog_selftest: ") + cudaGetErrorString(cudaGetLastError()));
+    if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "watchdog_selftest: a device wait ran out (code " +
+                                                              std::to_string(derr) + ")");
+    return TRIMMOE_OK;
+}
+
 extern "C" trimmoe_status trimmoe_calibration_begin(trimmoe_handle h) {
     if (!h) return TRIMMOE_ERR_ARG;
     DeviceGuard g(h->dev);

@@ -194,6 +194,36 @@ def test_stats_counters_consistent():
     eng.close()
 
 
+def test_device_wait_timeout_is_reported_and_context_survives():
+    """Failure detection without a fault: a bounded mbarrier wait that nothing
+    completes runs out, the host reads DEVICE_TIMEOUT and the self-test code,
+    the second warp (two-second limit) returns on the abort flag, a reset clears
+    the flag, and the next layer step on the same context still matches the
+    oracle."""
+    import time
+    import torch
+    cfg = SMALL["swiglu_k2_renorm_h2"]
+    eng, om, tables, small, experts = make_engine(cfg)
+    dev = eng.tokens_to_device(W.make_tokens(cfg))
+    compare_layer(cfg, om, eng, 0, dev, experts)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    rc = B.trimmoe_watchdog_selftest(eng.handle, 20000, eng.stream_ptr())
+    wall = time.perf_counter() - t0
+    assert rc == -6, (rc, B.trimmoe_last_error(eng.handle))
+    assert 0.02 <= wall < 1.0, wall
+    assert "ran out (code 6)" in B.trimmoe_last_error(eng.handle)
+    st = eng.stats()
+    assert st["status"] == -6 and st["device_error"] == 6
+    eng.reset_stats()
+    st = eng.stats()
+    assert st["status"] == 0 and st["device_error"] == 0
+    compare_layer(cfg, om, eng, 1, dev, experts)
+    assert B.trimmoe_watchdog_selftest(eng.handle, 0, eng.stream_ptr()) == -1
+    assert eng.stats()["device_error"] == 0
+    eng.close()
+
+
 def test_create_rejects_bad_input():
     cfg = SMALL["swiglu_k2_renorm_h2"]
     small = W.make_small_weights(cfg)

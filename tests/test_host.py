@@ -143,6 +143,7 @@ def test_create_rejects_bad_arguments_on_host(lib):
 
 def test_null_handle_calls_fail_cleanly(lib):
     assert lib.trimmoe_layer_step(None, 0, 1, None, None, None) == -1
+    assert lib.trimmoe_watchdog_selftest(None, 1000, None) == -1
     assert lib.trimmoe_forward(None, 1, None, None) == -1
     assert lib.trimmoe_stats(None, None) == -1
     lib.trimmoe_destroy(None)
