@@ -227,7 +227,7 @@ cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, cons
                           const RouterParams& p, int num_sms, cudaStream_t st);
 int router_lo_rows(int n_lo, int ng);
 int router_pass_rows(int n_out);
-int router_ksplit(int T, int d, int num_sms);
+int router_ksplit(int T, int d, int n_out, int num_sms);
 cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand);
 size_t decide_la_scratch_floats(int E, int M, int max_layer_cand, int num_sms);

@@ -250,16 +250,6 @@ int router_lo_rows(int n_lo, int ng) {
     return r < ng ? r : ng;
 }
 
-// Column ranges per launch: a power of two dividing d/64, chosen so that the
-// persistent grid has at least about eight units per SM.
-int router_ksplit(int T, int d, int num_sms) {
-    const int nslab = d / kKS;
-    const int tiles = (T + kTok - 1) / kTok;
-    int ks = 1;
-    while (ks < nslab && (long long)tiles * ks < 8ll * num_sms && nslab % (ks * 2) == 0) ks *= 2;
-    return ks;
-}
-
 // Rows per pass: n-tiles of 8 rounded up to 1, 2 or 4 (the kernel's register
 // tile), at most 32: wider passes need the registers of a whole SM per CTA,
 // and a second CTA per SM (plus a re-read of h per extra pass) was faster.
@@ -267,6 +257,21 @@ int router_pass_rows(int n_out) {
     const int t = (n_out + 7) / 8;
     const int nt = t <= 1 ? 1 : t <= 2 ? 2 : 4;
     return nt * 8;
+}
+
+// Column ranges per launch: the smallest power of two dividing d/64 that gives
+// every SM at least one (tile, range, pass) unit.  More ranges only add
+// partial sums for the decision kernel to write and read back: on the
+// 8192-token layer with d = 2048 and 60 experts, 2 ranges took 27 us where 32
+// ranges (eight units per SM) took 50 us.
+int router_ksplit(int T, int d, int n_out, int num_sms) {
+    const int nslab = d / kKS;
+    const int tiles = (T + kTok - 1) / kTok;
+    const int ng = router_pass_rows(n_out);
+    const long long units = (long long)tiles * ((n_out + ng - 1) / ng);
+    int ks = 1;
+    while (ks < nslab && units * ks < num_sms && nslab % (ks * 2) == 0) ks *= 2;
+    return ks;
 }
 
 cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, const CUtensorMap* tmBlo,

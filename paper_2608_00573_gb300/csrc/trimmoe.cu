@@ -577,7 +577,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         }
 
     for (int tt = 1; tt <= c.T_max; ++tt)
-        h->rows_part = std::max(h->rows_part, (size_t)router_ksplit(tt, d, h->num_sms) * tt);
+        h->rows_part = std::max(h->rows_part, (size_t)router_ksplit(tt, d, n_out, h->num_sms) * tt);
 
     // Device tables and workspaces.
     const size_t T = (size_t)c.T_max, TK = T * c.k;
@@ -849,7 +849,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     rp.ng = router_pass_rows(n_out);
     rp.nl = router_lo_rows(E, rp.ng);
     rp.zs = n_out;
-    rp.ksplit = router_ksplit(T, d, h->num_sms);
+    rp.ksplit = router_ksplit(T, d, n_out, h->num_sms);
     rp.h = hid;
     rp.alive = tok->alive;
     rp.Bhi = h->rt_hi + (size_t)layer * n_out * d;
