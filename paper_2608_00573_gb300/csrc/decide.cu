@@ -466,8 +466,10 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
 // The layer's look-ahead tables for Dbar = Dbar[0]: block (i, y) computes the
 // table of interval i (R = thr[i - 1], or -inf for i = 0) at depth dmin + y,
 // each entry by one thread with the same operation order as the per-token path
-// above.
-__global__ void __launch_bounds__(256) lookahead_shared_kernel(const DecideParams p) {
+// above.  A block has a thread per entry (up to 1024): each entry is a chain of
+// dependent loads and roundings, so the table is latency-bound and the blocks
+// (one per interval and depth) are too few to fill the SMs otherwise.
+__global__ void __launch_bounds__(1024) lookahead_shared_kernel(const DecideParams p) {
     pdl_wait();      // results of the preceding kernel in the stream
     extern __shared__ float smem[];
     const int E = p.E, M = p.M, l = p.layer;
@@ -554,7 +556,9 @@ cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStre
     // A plain launch: measured with programmatic serialisation this kernel cost
     // 60 us per layer more on the Qwen-shaped layer (E = 60) and saved nothing
     // elsewhere.
-    lookahead_shared_kernel<<<dim3(p.n_thr + 1, n_depth), 256, smem, st>>>(p);
+    const int ME = p.M * p.E;
+    const int threads = std::min(1024, std::max(256, (ME + 31) / 32 * 32));
+    lookahead_shared_kernel<<<dim3(p.n_thr + 1, n_depth), threads, smem, st>>>(p);
     return cudaGetLastError();
 }
 
