@@ -326,7 +326,7 @@ def run_ours(args):
         with open(tp) as fh:
             tj = json.load(fh)
         ent = tj.get(cfg.name, {}).get(dom)
-        if ent and ent.get("kernel_rev") == KERNEL_REV:
+        if ent and ent.get("kernel_rev") == KERNEL_REV[dom]:
             traffic = ent.get("bytes_per_launch")
     # The GEMM is tensor-bound when its FLOPs take longer at peak than its bytes.
     tensor_bound = fl_k / (peaks["bf16_sus"] * 1e12) >= by_k / (peaks["hbm"] * 1e9)
@@ -406,9 +406,9 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-# Revision tag of the timed GEMM kernel; a stored ncu traffic figure is used
-# only when it was taken on this revision.
-KERNEL_REV = "gemm-v7"
+# Revision tag of each timed GEMM launch kind; a stored ncu traffic figure is
+# used only when it was taken on that revision.
+KERNEL_REV = {"grouped_gemm_gate_up": "gemm-v7", "grouped_gemm_down": "gemm-v8"}
 
 
 def main():

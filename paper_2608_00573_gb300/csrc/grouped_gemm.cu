@@ -38,6 +38,10 @@
 // (~2500 tensor cycles) of loads in flight instead of 3.  A row-pair tile
 // covers 256 rows of one group (the odd CTA's rows may lie past the group:
 // loaded, computed and masked).
+//
+// Transposed pair variant (routed down projections, ReLU up projections): the
+// weights on the MMA's M side and the tokens on its N side, N rounded up to 16
+// per tile, so a group's tail pads at most 15 tokens; described at the kernel.
 #include <algorithm>
 
 #include "internal.cuh"
@@ -106,21 +110,19 @@ __device__ __forceinline__ void build_tile_table(Tail* tl, const int* goff, int 
 // block's activation rows are read from HBM once.  A row tile has tile_rows
 // rows; this CTA takes the 128 from sub_row on and B rows from b_sub on.
 template <class Tail>
-__device__ __forceinline__ Tile map_tile(const Tail* tl, int t, int ngroups, int n_tiles_n, int base0,
-                                         int a_rebase, int out_rebase, int b_rows_per_group, int mblk,
-                                         int tile_rows, int sub_row, int b_sub) {
+__device__ __forceinline__ void locate_tile(const Tail* tl, int t, int ngroups, int n_tiles_n, int mblk,
+                                            int tile_rows, int& g, int& mt, int& nt) {
     int lo = 0, hi = ngroups - 1;
     while (lo < hi) {                      // largest g with tile_start[g] <= t
         const int mid = (lo + hi + 1) >> 1;
         if (tl->tile_start[mid] <= t) lo = mid; else hi = mid - 1;
     }
-    const int g = lo;
+    g = lo;
     const int cnt = tl->gcnt[g];
     const int mtc = (cnt + tile_rows - 1) / tile_rows;
     const int u = t - tl->tile_start[g];
     const int nfull = mtc / mblk;
     const int full_tiles = nfull * mblk * n_tiles_n;
-    int nt, mt;
     if (u < full_tiles) {
         const int b = u / (mblk * n_tiles_n);
         const int r = u - b * (mblk * n_tiles_n);
@@ -132,6 +134,15 @@ __device__ __forceinline__ Tile map_tile(const Tail* tl, int t, int ngroups, int
         nt = r / last;
         mt = nfull * mblk + (r - nt * last);
     }
+}
+
+template <class Tail>
+__device__ __forceinline__ Tile map_tile(const Tail* tl, int t, int ngroups, int n_tiles_n, int base0,
+                                         int a_rebase, int out_rebase, int b_rows_per_group, int mblk,
+                                         int tile_rows, int sub_row, int b_sub) {
+    int g, mt, nt;
+    locate_tile(tl, t, ngroups, n_tiles_n, mblk, tile_rows, g, mt, nt);
+    const int cnt = tl->gcnt[g];
     const int r0 = mt * tile_rows + sub_row;
     Tile r;
     r.rows = max(0, min(BM, cnt - r0));
@@ -576,6 +587,258 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
     }
 }
 
+// ---------------------------------------------------------------------------
+// Transposed pair variant (the routed experts' down projection, and the
+// up projection of ReLU experts): the weights take the M side and the tokens
+// the N side of tcgen05.mma.cta_group::2, D = W . X^T with M = 256 output
+// features and N = the tile's tokens rounded up to 16 (at most 256).  A
+// group's last token tile then computes at most 15 padded tokens, not up to
+// 255 padded rows, while each SM still stages only half of the shared operand
+// per FLOP.  Tiles are (group, block of token tiles, feature tile, token tile)
+// in the order of map_tile.  CTA rank r stages weight rows (features)
+// [r 128, r 128 + 128) of the feature tile and tokens [r N/2, (r+1) N/2) of
+// the tile; its TMEM lane is an output feature and its column a token.
+// Every MMA reads its operands from shared memory while TMA refills it, so
+// for long K (the main loop hides the epilogue) each warp stores its 32
+// features of a token straight from registers as one 64-byte segment; for
+// short K the epilogue is on the critical path and the results are staged in
+// shared memory and stored as 16-byte pieces of the tokens' rows.
+// SwiGLU stays on the kernels above: its gate and up accumulators would sit
+// in different warps' TMEM lanes, and every way of bringing them together
+// that was tried (through shared memory, or 16-row weight boxes that pair
+// them within a warp) was slower than the padding it saves.
+constexpr int kStageBf16 = 32 * 128;           // one 32-token x 128-feature bf16 staging buffer
+constexpr size_t kPairTailBytes = (sizeof(PairSmemTail) + 15) & ~(size_t)15;
+constexpr size_t kPairTSmemBytes = 1024 + (size_t)P_STAGES * P_STAGE_BYTES + kPairTailBytes +
+                                   2 * kStageBf16 * sizeof(__nv_bfloat16);
+constexpr int kEpiBar = 1;                    // named barrier of the four epilogue warps
+constexpr int kStagedMaxK = 4096;             // store/ReLU epilogue staged in shared memory up to this K
+
+__device__ __forceinline__ void bar_sync_named(int id, int n) {
+    asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// AND of pred over the n threads of named barrier id (a barrier as well).
+__device__ __forceinline__ int bar_and_named(int id, int n, int pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "barrier.red.and.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(pred), "r"(id), "r"(n)
+        : "memory");
+    return (int)r;
+}
+
+// Token rows of tile (g, mt); the tile's MMA takes N = this rounded up to 16.
+template <class Tail>
+__device__ __forceinline__ int tile_tokens(const Tail* tl, int g, int mt) {
+    return min(2 * BM, tl->gcnt[g] - mt * 2 * BM);
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                           const int* __restrict__ goff,
+                           int first_group, int ngroups, int x_rebase, int out_rebase, int K, int n_ft,
+                           int w_rows_per_group, int epi_mode, __nv_bfloat16* __restrict__ out, int ldo,
+                           int* err, int mblk) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
+    uint8_t* smem = smem_raw + pad;
+    const uint32_t sW = smem_u32(smem);                 // weight rows (M side), A_BYTES per stage
+    const uint32_t sX = sW + P_STAGES * A_BYTES;        // token rows (N side), PB_BYTES per stage
+    PairSmemTail* tl = reinterpret_cast<PairSmemTail*>(smem + (size_t)P_STAGES * P_STAGE_BYTES);
+    uint8_t* stage_out = smem + (size_t)P_STAGES * P_STAGE_BYTES + kPairTailBytes;   // two staging buffers
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();      // 0: issues the MMAs, 1: peer
+    const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
+
+    if (threadIdx.x == 0) build_tile_table(tl, goff, first_group, ngroups, n_ft, 2 * BM);
+    __syncthreads();
+    const int ntiles = tl->total_tiles;
+    if (cid >= ntiles) return;                    // both CTAs of the pair leave together
+    const int base0 = tl->gstart[0];
+    const int nkb = K / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < P_STAGES; ++s) {
+            mbar_init(smem_u32(&tl->full[s]), 1);
+            mbar_init(smem_u32(&tl->empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&tl->tfull[b]), 1);
+            mbar_init(smem_u32(&tl->tempty[b]), 8);
+        }
+        fence_barrier_init();
+        prefetch_tmap(&tmX);
+        prefetch_tmap(&tmW);
+    }
+    if (warp == 0) tmem_alloc_pair(smem_u32(&tl->tmem_base), TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();                               // both CTAs' barriers are initialised
+    tc_fence_after();
+    const uint32_t tmem_base = tl->tmem_base;
+    volatile int* abort_flag = &tl->abort_flag;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------------------------------------------- producer (both CTAs)
+            int it = 0;
+            for (int t = cid; t < ntiles && !*abort_flag; t += ncl) {
+                int g, mt, ft;
+                locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
+                const int half = ((tile_tokens(tl, g, mt) + 15) & ~15) >> 1;
+                const int xrow = tl->gstart[g] - (x_rebase ? base0 : 0) + mt * 2 * BM + (int)rank * half;
+                const int wrow = g * w_rows_per_group + ft * 2 * BM;
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % P_STAGES;
+                    const uint32_t ph = (it / P_STAGES) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&tl->empty[s]), ph ^ 1, abort_flag, err,
+                                           ERR_TIMEOUT_PRODUCER))
+                        break;
+                    if (rank == 0) mbar_arrive_expect_tx(smem_u32(&tl->full[s]), 2 * P_STAGE_BYTES);
+                    const uint32_t fb = mapa_shared(smem_u32(&tl->full[s]), 0);
+                    tma_load_2d_pair(sW + s * A_BYTES, &tmW, kb * BK, wrow + (int)rank * BM, fb);
+                    tma_load_2d_pair(sX + s * PB_BYTES, &tmX, kb * BK, xrow, fb);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) {
+            // ---------------------------------------------------- MMA issuer (even CTA)
+            int it = 0, tl_i = 0;
+            bool ok = true;
+            for (int t = cid; t < ntiles && ok; t += ncl, ++tl_i) {
+                int g, mt, ft;
+                locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
+                const uint32_t idesc = idesc_bf16_f32(2 * BM, (tile_tokens(tl, g, mt) + 15) & ~15);
+                const int buf = tl_i & 1;
+                const uint32_t aph = (tl_i >> 1) & 1;
+                if (!mbar_wait_bounded(smem_u32(&tl->tempty[buf]), aph ^ 1, abort_flag, err,
+                                       ERR_TIMEOUT_MMA)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int s = it % P_STAGES;
+                    const uint32_t ph = (it / P_STAGES) & 1;
+                    if (!mbar_wait_bounded(smem_u32(&tl->full[s]), ph, abort_flag, err, ERR_TIMEOUT_MMA)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t w0 = sW + s * A_BYTES;
+                    const uint32_t x0 = sX + s * PB_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        tc_mma_bf16_pair(d_tmem, smem_desc_sw128(w0 + kk * 32), smem_desc_sw128(x0 + kk * 32),
+                                         idesc, (kb != 0 || kk != 0) ? 1u : 0u);
+                    tc_commit_pair_mc(smem_u32(&tl->empty[s]), 0x3);
+                }
+                if (!ok) break;
+                tc_commit_pair_mc(smem_u32(&tl->tfull[buf]), 0x3);
+            }
+        }
+    } else {
+        // -------------------------------------------------------- epilogue (both CTAs)
+        const int q = warp & 3;                   // TMEM lane quarter of this warp
+        const int et = (warp - 2) * 32 + lane;    // epilogue thread 0..127
+        int tl_i = 0, chunk = 0;
+        for (int t = cid; t < ntiles; t += ncl, ++tl_i) {
+            int g, mt, ft;
+            locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
+            const int rows = tile_tokens(tl, g, mt);
+            const int nch = (((rows + 15) & ~15) + 31) / 32;
+            const size_t orow = (size_t)(tl->gstart[g] - (out_rebase ? base0 : 0) + mt * 2 * BM);
+            const int buf = tl_i & 1;
+            const uint32_t aph = (tl_i >> 1) & 1;
+            int ok = 1;
+            if (lane == 0)
+                ok = mbar_wait_bounded(smem_u32(&tl->tfull[buf]), aph, abort_flag, err, ERR_TIMEOUT_EPI);
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            // The four warps take the same branch (they meet at named barriers below).
+            if (!bar_and_named(kEpiBar, 128, ok)) break;
+            tc_fence_after();
+            const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
+            if (K > kStagedMaxK) {
+                // Long K: the main loop hides the epilogue, and shared-memory
+                // traffic would compete with the MMA operand reads, so each
+                // warp stores its 32 features of a token as one 64-byte segment.
+                __nv_bfloat16* ocol = out + (size_t)ft * 2 * BM + (size_t)rank * BM + q * 32 + lane;
+                const bool relu = epi_mode == EPI_RELU;
+#pragma unroll 1
+                for (int c = 0; c < nch; ++c) {
+                    uint32_t r[32];
+                    tmem_ld_32x32(tb + c * 32, r);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int tok = c * 32 + j;
+                        if (tok < rows) {
+                            const float x = __uint_as_float(r[j]);
+                            ocol[(orow + tok) * ldo] = __float2bfloat16_rn(relu ? fmaxf(x, 0.f) : x);
+                        }
+                    }
+                }
+            } else {
+                // Short K: the epilogue is on the critical path; each warp
+                // stages its 32 features of 32 tokens and the tokens' 256-byte
+                // rows are stored as 16-byte pieces.
+                __nv_bfloat16* hbase = reinterpret_cast<__nv_bfloat16*>(stage_out);
+                __nv_bfloat16* ocol = out + (size_t)ft * 2 * BM + (size_t)rank * BM;
+                const bool relu = epi_mode == EPI_RELU;
+#pragma unroll 1
+                for (int c = 0; c < nch; ++c, ++chunk) {
+                    __nv_bfloat16* hb = hbase + (chunk & 1) * 32 * 128;
+                    uint32_t r[32];
+                    tmem_ld_32x32(tb + c * 32, r);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const float x = __uint_as_float(r[j]);
+                        hb[j * 128 + q * 32 + lane] = __float2bfloat16_rn(relu ? fmaxf(x, 0.f) : x);
+                    }
+                    bar_sync_named(kEpiBar, 128);
+#pragma unroll
+                    for (int i = et; i < 32 * 16; i += 128) {
+                        const int row = i >> 4, seg = i & 15, tok = c * 32 + row;
+                        if (tok < rows)
+                            *reinterpret_cast<uint4*>(ocol + (orow + tok) * ldo + seg * 8) =
+                                *reinterpret_cast<const uint4*>(hb + row * 128 + seg * 8);
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                if (rank == 0) mbar_arrive(smem_u32(&tl->tempty[buf]));
+                else mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tempty[buf]), 0));
+            }
+        }
+    }
+
+    // A CTA that gave up tells its peer, so that the peer stops waiting on it.
+    __syncthreads();
+    if (threadIdx.x == 0 && *abort_flag)
+        st_shared_cluster_u32(mapa_shared(smem_u32(&tl->abort_flag), rank ^ 1u), 1u);
+    cluster_sync();                               // no access to the peer's memory remains in flight
+    if (warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    }
+}
+
 }  // namespace
 
 size_t grouped_gemm_smem_bytes() { return kSmemBytes; }
@@ -604,6 +867,27 @@ int pair_clusters(int num_sms) {
     return n;
 }
 
+// The same for the transposed pair kernel (a little more shared memory).
+int pair_t_clusters(int num_sms) {
+    static int n = -1;
+    if (n >= 0) return n;
+    n = 0;
+    if (cudaFuncSetAttribute(grouped_gemm_pair_t_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kPairTSmemBytes) != cudaSuccess)
+        return n;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(num_sms & ~1), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kPairTSmemBytes;
+    int ncl = 0;
+    if (cudaOccupancyMaxActiveClusters(&ncl, grouped_gemm_pair_t_kernel, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return n;
+    }
+    n = std::min(ncl, num_sms / 2);
+    return n;
+}
+
 }  // namespace
 
 int grouped_gemm_pair_clusters(int num_sms) { return pair_clusters(num_sms); }
@@ -620,6 +904,17 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     // Row tiles per block: about 48 MB of activations (a third of L2), so that
     // a block stays resident while the weight tiles stream past it.
     const long long a_tile_bytes = (long long)BM * g.K * 2;
+    if (g.transposed && g.tmB_pair && g.ksplit <= 1 && pair_t_clusters(num_sms) > 0) {
+        if (g.epi_mode != EPI_STORE && g.epi_mode != EPI_RELU) return cudaErrorInvalidValue;
+        // Token-tile blocks of about 32 MB of activations, as for the pair kernel.
+        const int mblk2 = (int)std::max(1LL, (32LL << 20) / (2 * a_tile_bytes));
+        const cudaError_t e = launch_pdl(
+            grouped_gemm_pair_t_kernel, dim3(2 * pair_t_clusters(num_sms)), dim3(kThreads), kPairTSmemBytes, st,
+            *g.tmA, *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
+            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, mblk2);
+        if (e != cudaSuccess) return e;
+        return cudaGetLastError();
+    }
     if (g.tmB_pair && (g.ksplit <= 1) && pair_clusters(num_sms) > 0) {
         // Row-pair tiles per block: about 32 MB of activations (same speed as
         // 40 or 48 MB within the run-to-run spread, fewest DRAM re-reads).

@@ -160,6 +160,10 @@ struct GemmLaunch {
     // Non-null: run the CTA-pair kernel, B loaded in 128-row boxes through this
     // map (launches whose groups are large; requires ksplit <= 1).
     const CUtensorMap* tmB_pair;
+    // Non-zero (with tmB_pair): run the transposed pair kernel instead, the
+    // weights on the M side of the MMA and the group's tokens on the N side
+    // (STORE or RELU epilogues; ksplit <= 1).
+    int transposed;
     const int* goff;
     int first_group, ngroups, a_rebase, out_rebase;
     int K, n_tiles_n, b_rows_per_group, epi_mode;

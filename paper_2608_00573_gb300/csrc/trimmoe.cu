@@ -64,6 +64,12 @@ constexpr int kPairMinRows = 2048;
 
 inline bool pair_gemm(long long rows_per_group) { return rows_per_group >= kPairMinRows; }
 
+// Routed launches whose groups average at least this many rows run their
+// store / ReLU epilogues on the transposed pair kernel; smaller groups are
+// weight-streaming bound, and its 256-feature pair tiles would leave a ragged
+// last round (Mixtral-shaped decode at 256 tokens: 15.2 -> 15.6 ms per step).
+constexpr int kTransposedMinRows = 256;
+
 enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
 
 inline float bf16_to_float(uint16_t b) {
@@ -995,8 +1001,17 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     GemmLaunch g1{};
     g1.tmA = &h->tmXp;
     g1.tmB = &h->tmW13[layer];
+    // Routed experts: with at least kTransposedMinRows rows per expert the
+    // down projection (and the up projection of ReLU experts) runs on the
+    // transposed pair kernel, tokens on the MMA's N side so that a group's
+    // last tile pads at most 15 tokens; SwiGLU up projections run on the pair
+    // kernel for large groups and the single-CTA kernel otherwise;
+    // decode-sized batches split K on the single-CTA kernel.
     const bool pair_routed = pair_gemm((long long)T * K / E);
-    g1.tmB_pair = pair_routed ? &h->tmW13p[layer] : nullptr;
+    const bool relu = c.act != 1;
+    const bool transposed = (long long)T * K / E >= kTransposedMinRows;
+    g1.transposed = relu && transposed;
+    g1.tmB_pair = (g1.transposed || pair_routed) ? &h->tmW13p[layer] : nullptr;
     g1.goff = h->goff;
     g1.first_group = 0;
     g1.ngroups = E;
@@ -1027,7 +1042,8 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     GemmLaunch g2 = g1;
     g2.tmA = &h->tmAct;
     g2.tmB = &h->tmW2[layer];
-    g2.tmB_pair = pair_routed ? &h->tmW2p[layer] : nullptr;
+    g2.transposed = transposed;
+    g2.tmB_pair = (g2.transposed || pair_routed) ? &h->tmW2p[layer] : nullptr;
     g2.K = c.F;
     g2.n_tiles_n = d / 256;
     g2.b_rows_per_group = d;
@@ -1049,6 +1065,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (has_sh) {
         GemmLaunch s1 = g1;
         s1.ksplit = 1;
+        s1.transposed = 0;
         s1.tmB = &h->tmW13sh[layer];
         s1.tmB_pair = pair_gemm(T) ? &h->tmW13shp[layer] : nullptr;
         s1.first_group = E;

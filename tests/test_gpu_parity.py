@@ -281,6 +281,24 @@ def test_layer_parity_pair_gemm(name, kw):
     assert tot["exec"] > 0
 
 
+@pytest.mark.parametrize("name,kw", [
+    ("swiglu_E16_k2", dict(N=2, d=512, E=16, k=2, F=384, T=2300, M=10, H=3, zipf_s=1.0)),
+    ("relu_E8_k1", dict(N=2, d=768, E=8, k=1, F=512, C=64, act=W.ACT_RELU, T=2300, M=10, zipf_s=1.0)),
+])
+def test_layer_parity_transposed_pair_gemm(name, kw):
+    """Groups averaging >= 256 rows run the routed down projection (and the
+    ReLU up projection) on the transposed CTA-pair kernel: weights on the MMA's
+    M side, a group's tokens on its N side in tiles of up to 256 rounded up to
+    16.  With Zipf(1.0) routing the groups range from a few rows to well over
+    256, so token tiles of many sizes (N from 16 to 256, tails inside a
+    16-row step) occur."""
+    cfg = small_cfg(name=name, seed=99, **kw)
+    reports = _run_all_layers(cfg, theta=0.9, exit_bias=1.0 if cfg.C == 1 else 5.0)
+    tot = {k: sum(r[k] for r in reports) for k in ("exec", "skip", "exit")}
+    print(name, tot, [round(r["max_rel_err"], 5) for r in reports])
+    assert tot["exec"] > 0
+
+
 def test_layer_parity_decision_lane_groups_of_16():
     """8 < E <= 16 with more tokens than the resident warps (T >= 16 x SMs):
     the decision kernel runs two tokens per warp on 16-lane groups."""
