@@ -463,16 +463,16 @@ __global__ void __launch_bounds__(kWarps * 32, 6) decide_kernel(const DecidePara
     pdl_trigger();   // the next kernel may be scheduled once every block got here or exited
 }
 
-// The layer's look-ahead tables for Dbar = Dbar[0]: block (i, y) computes the
-// table of interval i (R = thr[i - 1], or -inf for i = 0) at depth dmin + y,
-// each entry by one thread with the same operation order as the per-token path
-// above.  A block has a thread per entry (up to 1024): each entry is a chain of
-// dependent loads and roundings, so the table is latency-bound and the blocks
-// (one per interval and depth) are too few to fill the SMs otherwise.
-__global__ void __launch_bounds__(1024) lookahead_shared_kernel(const DecideParams p) {
-    pdl_wait();      // results of the preceding kernel in the stream
+// One look-ahead table for Dbar = Dbar[0]: layer l, interval iv (R =
+// thr[iv - 1], or -inf for iv = 0), depth top (levels l + top .. l + 1), each
+// entry by one thread with the same operation order as the per-token path
+// above, written to out.  A block has a thread per entry (up to 1024): each
+// entry is a chain of dependent loads and roundings, so a table is
+// latency-bound.  Called by whole blocks.
+__device__ __forceinline__ void lookahead_table(const DecideParams& p, int l, const float* thr, int iv, int top,
+                                                float* out) {
     extern __shared__ float smem[];
-    const int E = p.E, M = p.M, l = p.layer;
+    const int E = p.E, M = p.M;
     const int ME = M * E;
     const int MC = p.tab.max_layer_cand;
     float* bufV = smem;
@@ -482,9 +482,7 @@ __global__ void __launch_bounds__(1024) lookahead_shared_kernel(const DecidePara
     uint8_t* cok = reinterpret_cast<uint8_t*>(cph + MC);
     uint8_t* cmv = cok + ((MC + 3) & ~3);
     const float Dbar = p.Dbar[0];
-    const int iv = blockIdx.x;
-    const float R = iv == 0 ? -kInf : p.thr[iv - 1];
-    const int top = p.dmin + blockIdx.y;
+    const float R = iv == 0 ? -kInf : thr[iv - 1];
     bool have_phi = false;
     for (int jj = top; jj >= 1; --jj) {
         const int lp = l + jj;
@@ -540,10 +538,32 @@ __global__ void __launch_bounds__(1024) lookahead_shared_kernel(const DecidePara
         __syncthreads();
         have_phi = true;
     }
-    float* out = p.phi_tabs_out + ((size_t)blockIdx.y * (p.n_thr + 1) + iv) * ME;
     for (int idx = threadIdx.x; idx < ME; idx += blockDim.x) out[idx] = have_phi ? bufPhi[idx] : 0.f;
-    if (threadIdx.x == 0 && iv == 0 && blockIdx.y == 0) *p.dbar_shared_out = Dbar;
+    if (threadIdx.x == 0 && iv == 0) *p.dbar_shared_out = Dbar;
+}
+
+// The tables of one layer: block (i, y) computes interval i at depth dmin + y.
+__global__ void __launch_bounds__(1024) lookahead_shared_kernel(const DecideParams p) {
+    pdl_wait();      // results of the preceding kernel in the stream
+    const int iv = blockIdx.x;
+    lookahead_table(p, p.layer, p.thr, iv, p.dmin + (int)blockIdx.y,
+                    p.phi_tabs_out + ((size_t)blockIdx.y * (p.n_thr + 1) + iv) * p.M * p.E);
     pdl_trigger();   // the next kernel may be scheduled once every block got here or exited
+}
+
+// The tables of every layer at once (they depend only on the tables, the
+// budget Dbar[0] and the cost weights): block (i, y, l) computes interval i at
+// depth dmin_l + y of layer l, for the layers whose tables pay off at p.T
+// tokens (the same test as the per-layer launch).
+__global__ void __launch_bounds__(1024) lookahead_all_kernel(const DecideParams p, const LaLayer* __restrict__ lay) {
+    const int l = blockIdx.z;
+    const LaLayer L = lay[l];
+    const int iv = blockIdx.x, y = blockIdx.y;
+    if (L.n_depth <= 0 || iv > L.n_thr || y >= L.n_depth) return;
+    if ((long long)(L.n_thr + 1) * L.n_depth * 4 > p.T) return;
+    const int top_full = min(p.H - 1, p.N - 1 - l);
+    lookahead_table(p, l, p.thr + L.thr_off, iv, top_full - L.n_depth + 1 + y,
+                    p.phi_tabs_out + L.tab_off + ((size_t)y * (L.n_thr + 1) + iv) * p.M * p.E);
 }
 
 }  // namespace
@@ -559,6 +579,17 @@ cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStre
     const int ME = p.M * p.E;
     const int threads = std::min(1024, std::max(256, (ME + 31) / 32 * 32));
     lookahead_shared_kernel<<<dim3(p.n_thr + 1, n_depth), threads, smem, st>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_lookahead_all(const DecideParams& p, const LaLayer* layers, int n_layers, int max_thr,
+                                 int max_depth, cudaStream_t st) {
+    if (p.T <= 0 || n_layers <= 0 || max_depth <= 0) return cudaSuccess;
+    const size_t MC = (size_t)p.tab.max_layer_cand;
+    const size_t smem = (2 * (size_t)p.M * p.E + 2 * MC) * sizeof(float) + ((MC + 3) / 4) * 2 * sizeof(float);
+    const int ME = p.M * p.E;
+    const int threads = std::min(1024, std::max(256, (ME + 31) / 32 * 32));
+    lookahead_all_kernel<<<dim3(max_thr + 1, max_depth, n_layers), threads, smem, st>>>(p, layers);
     return cudaGetLastError();
 }
 

@@ -24,6 +24,7 @@ constexpr int kMaxCand = 64;        // (1 + n_sub) * M with n_sub <= 3, M <= 16
 constexpr int kMaxME = 1024;        // look-ahead table entries per token
 constexpr size_t kMaxIntervals = 4096;            // shared look-ahead tables per depth and layer
 constexpr size_t kMaxTabFloats = (size_t)16 << 20; // 64 MB of shared look-ahead tables
+constexpr size_t kMaxAllTabFloats = (size_t)64 << 20; // every layer's tables at once: up to 256 MB
 constexpr int kGateUp = 128;        // W13 gate/up row interleave
 
 // Device error codes (first one wins); the public TRIMMOE_DEVERR_* values.
@@ -236,6 +237,14 @@ cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st);
 size_t decide_smem_bytes(int E, int C, int M, int max_layer_cand);
 size_t decide_la_scratch_floats(int E, int M, int max_layer_cand, int num_sms);
 cudaError_t launch_lookahead_shared(const DecideParams& p, int n_depth, cudaStream_t st);
+// Placement of one layer's shared look-ahead tables when every layer's tables
+// are computed in one launch: thresholds p.thr[thr_off .. thr_off + n_thr),
+// n_depth depths, tables from p.phi_tabs_out + tab_off.
+struct LaLayer {
+    int thr_off, n_thr, n_depth, tab_off;
+};
+cudaError_t launch_lookahead_all(const DecideParams& p, const LaLayer* layers, int n_layers, int max_thr,
+                                 int max_depth, cudaStream_t st);
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st);
 cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k, int d,
                           const __nv_bfloat16* h, const float* rnorm, const __nv_bfloat16* gamma,

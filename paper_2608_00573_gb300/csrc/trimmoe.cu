@@ -149,6 +149,12 @@ struct trimmoe {
     std::vector<int> tab_depths;      // [N] depths tabulated (0: none)
     float* thr = nullptr;
     float* phi_tabs = nullptr;
+    // Every layer's tables in one buffer (la_all): layer l's at tab_off, built
+    // by one launch at the start of a forward (tabs_ready while its layers run).
+    bool la_all = false, tabs_ready = false;
+    std::vector<LaLayer> h_la;
+    LaLayer* la_layers = nullptr;
+    int la_max_thr = 0, la_max_depth = 0;
     float* dbar_shared = nullptr;     // [1]
     float* cnorm = nullptr;           // [N][K_c] centroid norms
     int16_t* lhat = nullptr;          // [N][K_c] rounded average exit layers
@@ -524,6 +530,25 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         h->h_thr.insert(h->h_thr.end(), v.begin(), v.end());
         h->thr_off[l + 1] = (int)h->h_thr.size();
     }
+    // All layers' tables side by side when they fit in kMaxAllTabFloats.
+    {
+        size_t total = 0;
+        h->h_la.assign(N, LaLayer{0, 0, 0, 0});
+        for (int l = 0; l < N; ++l) {
+            LaLayer& L = h->h_la[l];
+            L.thr_off = h->thr_off[l];
+            L.n_thr = h->thr_off[l + 1] - h->thr_off[l];
+            L.n_depth = h->tab_depths[l];
+            L.tab_off = (int)total;
+            total += (size_t)L.n_depth * (L.n_thr + 1) * M * E;
+            if (L.n_depth > 0) {
+                h->la_max_thr = std::max(h->la_max_thr, L.n_thr);
+                h->la_max_depth = std::max(h->la_max_depth, L.n_depth);
+            }
+        }
+        h->la_all = total > 0 && total <= kMaxAllTabFloats;
+        if (h->la_all) tab_floats = total;
+    }
 
     // Router tables of kernel a0 (built from the borrowed device weights): per
     // layer, rows [0, E) hold gamma_l * W_r[l] split exactly into bf16 hi + lo
@@ -608,7 +633,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               h->dalloc(&h->Y, TK * d) && h->dalloc(&h->ctr, kCtrCopies) && h->dalloc(&h->dev_err, 1) &&
               h->dalloc(&h->fb_util, T) && h->dalloc(&h->fb_updated, T) && h->dalloc(&h->fb_result, 2) &&
               h->dalloc(&h->prev_target, T) && h->dalloc(&h->phi_tabs, std::max<size_t>(tab_floats, 1)) &&
-              h->dalloc(&h->thr, std::max<size_t>(h->h_thr.size(), 1)) && h->dalloc(&h->dbar_shared, 1);
+              h->dalloc(&h->thr, std::max<size_t>(h->h_thr.size(), 1)) && h->dalloc(&h->dbar_shared, 1) &&
+              (!h->la_all || h->dalloc(&h->la_layers, (size_t)N));
     h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
     ok = ok && h->dalloc(&h->c_counts, h->n_counts) &&
          h->dalloc(&h->splitk, (size_t)kSplitKMax * kSplitKRows * std::max<size_t>((size_t)h->n13 * c.F, (size_t)d));
@@ -631,6 +657,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     up(h->cand_k, ck.data(), ck.size());
     up(h->cand_Q, cq.data(), cq.size() * 4);
     if (!h->h_thr.empty()) up(h->thr, h->h_thr.data(), h->h_thr.size() * 4);
+    if (h->la_all) up(h->la_layers, h->h_la.data(), h->h_la.size() * sizeof(LaLayer));
     up(h->cand_off, coff.data(), coff.size() * 4);
     up(h->ctab, ctab.data(), ctab.size() * 4);
     up(h->rt_hi, rhi.data(), rhi.size() * 2);
@@ -898,12 +925,13 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     const int n_thr = h->thr_off[layer + 1] - h->thr_off[layer];
     const int n_depth = h->tab_depths[layer];
     const bool shared_tabs = n_depth > 0 && (size_t)(n_thr + 1) * n_depth * 4 <= (size_t)T;
-    dp.phi_tabs = shared_tabs ? h->phi_tabs : nullptr;
+    const size_t tab_off = h->la_all ? (size_t)h->h_la[layer].tab_off : 0;
+    dp.phi_tabs = shared_tabs ? h->phi_tabs + tab_off : nullptr;
     dp.dbar_shared = h->dbar_shared;
     dp.thr = h->thr + h->thr_off[layer];
     dp.n_thr = n_thr;
     dp.dmin = top_full - n_depth + 1;
-    dp.phi_tabs_out = h->phi_tabs;
+    dp.phi_tabs_out = h->phi_tabs + tab_off;
     dp.dbar_shared_out = h->dbar_shared;
     dp.la_scratch = shared_tabs ? h->la_scratch : nullptr;
     dp.calib = h->calib;
@@ -946,7 +974,9 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     // overlapping the router; heavy ones in line after it (run beside the
     // issue-bound router they slowed it more than they saved: Qwen-shaped,
     // M*E = 600, 23.5 -> 24.7 ms per forward; Switch-shaped 1.47 -> 1.40 ms).
-    const bool tabs_aside = shared_tabs && c.M * E <= 256;
+    // Already built for every layer at the start of the forward?
+    const bool tabs_here = shared_tabs && !h->tabs_ready;
+    const bool tabs_aside = tabs_here && c.M * E <= 256;
     if (tabs_aside) {
         e = cudaEventRecord(h->ev_fork, st);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(h->aux, h->ev_fork, 0);
@@ -971,7 +1001,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("look-ahead join: ") + cudaGetErrorString(e));
     }
     e = h->timed(K_DECIDE, st, [&] {
-        cudaError_t e2 = (shared_tabs && !tabs_aside) ? launch_lookahead_shared(dp, n_depth, st) : cudaSuccess;
+        cudaError_t e2 = (tabs_here && !tabs_aside) ? launch_lookahead_shared(dp, n_depth, st) : cudaSuccess;
         return e2 == cudaSuccess ? launch_decide(dp, h->num_sms, st) : e2;
     });
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("decide: ") + cudaGetErrorString(e));
@@ -1061,7 +1091,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     h->n_gemm_up++;
     h->n_gemm_down++;
     // router, decide, count, scatter, gather, gate/up GEMM, down GEMM (+ look-ahead tables, split-K finishes)
-    h->launches += 7 + (shared_tabs ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
+    h->launches += 7 + (tabs_here ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
     if (has_sh) {
         GemmLaunch s1 = g1;
         s1.ksplit = 1;
@@ -1141,12 +1171,52 @@ extern "C" trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T,
     return layer_step_impl(h, layer, T, tok, out, st);
 }
 
+// Every layer's shared look-ahead tables in one launch (they depend only on
+// the tables, the budget Dbar[0] and the cost weights, none of which change
+// within a forward); false if no layer uses them at T tokens.
+static bool build_all_tables(trimmoe_handle h, int T, const trimmoe_tokens* tok, cudaStream_t st, cudaError_t* err) {
+    *err = cudaSuccess;
+    if (!h->la_all || T <= 0) return false;
+    bool any = false;
+    for (const LaLayer& L : h->h_la) any |= L.n_depth > 0 && (size_t)(L.n_thr + 1) * L.n_depth * 4 <= (size_t)T;
+    if (!any) return false;
+    const trimmoe_config& c = h->cfg;
+    DecideParams dp{};
+    dp.T = T;
+    dp.N = c.N;
+    dp.E = c.E;
+    dp.M = c.M;
+    dp.H = c.H;
+    dp.omega_T = c.omega_T;
+    dp.omega_D = c.omega_D;
+    dp.Dbar = tok->Dbar;
+    dp.thr = h->thr;
+    dp.phi_tabs_out = h->phi_tabs;
+    dp.dbar_shared_out = h->dbar_shared;
+    dp.tab.cand_m = h->cand_m;
+    dp.tab.cand_k = h->cand_k;
+    dp.tab.cand_Q = h->cand_Q;
+    dp.tab.cand_off = h->cand_off;
+    dp.tab.ctab = h->ctab;
+    dp.tab.max_layer_cand = h->max_layer_cand;
+    dp.tab.P = h->P;
+    dp.tab.eps = h->eps;
+    *err = h->timed(K_DECIDE, st, [&] {
+        return launch_lookahead_all(dp, h->la_layers, c.N, h->la_max_thr, h->la_max_depth, st);
+    });
+    if (*err != cudaSuccess) return false;
+    h->launches += 1;
+    return true;
+}
+
 static trimmoe_status forward_layers(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st) {
-    for (int l = 0; l < h->cfg.N; ++l) {
-        trimmoe_status s = layer_step_impl(h, l, T, tok, nullptr, st);
-        if (s != TRIMMOE_OK) return s;
-    }
-    return TRIMMOE_OK;
+    cudaError_t e;
+    h->tabs_ready = build_all_tables(h, T, tok, st, &e);
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("look-ahead tables: ") + cudaGetErrorString(e));
+    trimmoe_status s = TRIMMOE_OK;
+    for (int l = 0; l < h->cfg.N && s == TRIMMOE_OK; ++l) s = layer_step_impl(h, l, T, tok, nullptr, st);
+    h->tabs_ready = false;
+    return s;
 }
 
 static bool same_tokens(const trimmoe_tokens& a, const trimmoe_tokens& b) {
