@@ -557,14 +557,12 @@ __global__ void __launch_bounds__(1024) lookahead_shared_kernel(const DecidePara
 
 // The tables of every layer at once (they depend only on the tables, the
 // budget Dbar[0] and the cost weights): block (i, y, l) computes interval i at
-// depth dmin_l + y of layer l, for the layers whose tables pay off at p.T
-// tokens (the same test as the per-layer launch).
+// depth dmin_l + y of layer l.
 __global__ void __launch_bounds__(1024) lookahead_all_kernel(const DecideParams p, const LaLayer* __restrict__ lay) {
     const int l = blockIdx.z;
     const LaLayer L = lay[l];
     const int iv = blockIdx.x, y = blockIdx.y;
     if (L.n_depth <= 0 || iv > L.n_thr || y >= L.n_depth) return;
-    if ((long long)(L.n_thr + 1) * L.n_depth * 4 > p.T) return;
     const int top_full = min(p.H - 1, p.N - 1 - l);
     lookahead_table(p, l, p.thr + L.thr_off, iv, top_full - L.n_depth + 1 + y,
                     p.phi_tabs_out + L.tab_off + ((size_t)y * (L.n_thr + 1) + iv) * p.M * p.E);

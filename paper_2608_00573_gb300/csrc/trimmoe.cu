@@ -920,11 +920,12 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     dp.cnorm = h->cnorm + (size_t)layer * Kc;
     dp.lhat_tab = h->lhat + (size_t)layer * Kc;
     dp.lhat_out = (out && out->lhat) ? out->lhat : nullptr;
-    // Shared tables pay off once the tokens outnumber the tables severalfold.
     const int top_full = std::min(c.H - 1, c.N - 1 - layer);
     const int n_thr = h->thr_off[layer + 1] - h->thr_off[layer];
     const int n_depth = h->tab_depths[layer];
-    const bool shared_tabs = n_depth > 0 && (size_t)(n_thr + 1) * n_depth * 4 <= (size_t)T;
+    // Tables built for every layer at the start of the forward serve any T;
+    // a layer that builds its own pays off once the tokens outnumber them.
+    const bool shared_tabs = n_depth > 0 && (h->tabs_ready || (size_t)(n_thr + 1) * n_depth * 4 <= (size_t)T);
     const size_t tab_off = h->la_all ? (size_t)h->h_la[layer].tab_off : 0;
     dp.phi_tabs = shared_tabs ? h->phi_tabs + tab_off : nullptr;
     dp.dbar_shared = h->dbar_shared;
@@ -1173,12 +1174,14 @@ extern "C" trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T,
 
 // Every layer's shared look-ahead tables in one launch (they depend only on
 // the tables, the budget Dbar[0] and the cost weights, none of which change
-// within a forward); false if no layer uses them at T tokens.
+// within a forward).  One launch per forward costs less than the tokens'
+// own tables at any T (at one token: a table chain per layer on the critical
+// path).  False if no layer has tables.
 static bool build_all_tables(trimmoe_handle h, int T, const trimmoe_tokens* tok, cudaStream_t st, cudaError_t* err) {
     *err = cudaSuccess;
     if (!h->la_all || T <= 0) return false;
     bool any = false;
-    for (const LaLayer& L : h->h_la) any |= L.n_depth > 0 && (size_t)(L.n_thr + 1) * L.n_depth * 4 <= (size_t)T;
+    for (const LaLayer& L : h->h_la) any |= L.n_depth > 0;
     if (!any) return false;
     const trimmoe_config& c = h->cfg;
     DecideParams dp{};
