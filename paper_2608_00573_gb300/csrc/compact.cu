@@ -10,7 +10,7 @@
 // Two passes over chunks of kChunk tokens: per-chunk bucket counts, then a
 // scatter in which each chunk's block derives its base and the group offsets
 // from all chunks' counts and each of its warps walks its 32 tokens in order,
-// ranking equal buckets with __match_any_sync.
+// ranking equal buckets with __match_any_sync (one pass for a single chunk).
 #include <mutex>
 #include <string>
 
@@ -48,9 +48,12 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const CompactParams p) {
 // positions (group offset + chunk base + the earlier warps' counts), and each
 // warp then walks its pairs in (t, j) order, 32 at a time, ranking equal
 // buckets with __match_any_sync.  Integer sums: the result does not depend on
-// the order of the additions.
+// the order of the additions.  With a single chunk (T <= kChunk) the block
+// counts its own pairs: no count kernel, and the bucket totals are the sums of
+// the warps' counts.
 constexpr int kScatWarps = kChunk / 32;
 
+template <bool kSingle>
 __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) {
     pdl_wait();      // results of the preceding kernel in the stream
     pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
@@ -60,7 +63,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) 
     const int nb = p.E + 1;
     for (int i = threadIdx.x; i < kScatWarps * nb; i += blockDim.x) run[i / nb][i % nb] = 0;
     // Chunk base and total per bucket: a warp per bucket, lanes over chunks.
-    for (int e = warp; e < nb; e += kScatWarps) {
+    for (int e = warp; e < (kSingle ? 0 : nb); e += kScatWarps) {
         int pre = 0, all = 0;
         for (int b0 = 0; b0 < p.nblk; b0 += 32) {
             const int b = b0 + lane;
@@ -75,6 +78,36 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) 
         }
         if (lane == 0) {
             cbase[e] = pre;
+            total[e] = all;
+        }
+    }
+    __syncthreads();
+    const int t0 = blockIdx.x * kChunk + warp * 32;
+    const int tn = max(0, min(32, p.T - t0));
+    const unsigned lt_mask = (1u << lane) - 1u;
+    const int npairs = tn * p.k;
+    // Pass 1: this warp's count per bucket.
+    for (int q0 = 0; q0 < npairs; q0 += 32) {
+        const int q = q0 + lane;
+        int key = -1;
+        if (q < npairs) {
+            const int t = t0 + q / p.k;
+            if (p.action[t] == 0) key = p.exp_sel[t * p.k + (q - (q / p.k) * p.k)];
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, key);
+        if (key >= 0 && (peers & lt_mask) == 0) run[warp][key] += __popc(peers);
+    }
+    if (p.has_shared) {
+        const bool take = lane < tn && (p.action[t0 + lane] == 0 || p.action[t0 + lane] == 1);
+        const unsigned ball = __ballot_sync(0xffffffffu, take);
+        if (lane == 0) run[warp][p.E] = __popc(ball);
+    }
+    __syncthreads();
+    if (kSingle) {
+        for (int e = threadIdx.x; e < nb; e += blockDim.x) {
+            int all = 0;
+            for (int w = 0; w < kScatWarps; ++w) all += run[w][e];
+            cbase[e] = 0;
             total[e] = all;
         }
     }
@@ -107,27 +140,6 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(const CompactParams p) 
                 if (total[p.E] > 0) atomicAdd(&p.ctr->shared_touched, 1ull);
             }
         }
-    }
-    __syncthreads();
-    const int t0 = blockIdx.x * kChunk + warp * 32;
-    const int tn = max(0, min(32, p.T - t0));
-    const unsigned lt_mask = (1u << lane) - 1u;
-    const int npairs = tn * p.k;
-    // Pass 1: this warp's count per bucket.
-    for (int q0 = 0; q0 < npairs; q0 += 32) {
-        const int q = q0 + lane;
-        int key = -1;
-        if (q < npairs) {
-            const int t = t0 + q / p.k;
-            if (p.action[t] == 0) key = p.exp_sel[t * p.k + (q - (q / p.k) * p.k)];
-        }
-        const unsigned peers = __match_any_sync(0xffffffffu, key);
-        if (key >= 0 && (peers & lt_mask) == 0) run[warp][key] += __popc(peers);
-    }
-    if (p.has_shared) {
-        const bool take = lane < tn && (p.action[t0 + lane] == 0 || p.action[t0 + lane] == 1);
-        const unsigned ball = __ballot_sync(0xffffffffu, take);
-        if (lane == 0) run[warp][p.E] = __popc(ball);
     }
     __syncthreads();
     // Per-warp starting positions: exclusive prefix over the warps, per bucket.
@@ -239,8 +251,13 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
 
 cudaError_t launch_compact(const CompactParams& p, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    cudaError_t e = launch_pdl(count_kernel, dim3(p.nblk), dim3(kChunk), 0, st, p);
-    if (e == cudaSuccess) e = launch_pdl(scatter_kernel, dim3(p.nblk), dim3(kChunk), 0, st, p);
+    cudaError_t e;
+    if (p.nblk == 1) {
+        e = launch_pdl(scatter_kernel<true>, dim3(1), dim3(kChunk), 0, st, p);
+    } else {
+        e = launch_pdl(count_kernel, dim3(p.nblk), dim3(kChunk), 0, st, p);
+        if (e == cudaSuccess) e = launch_pdl(scatter_kernel<false>, dim3(p.nblk), dim3(kChunk), 0, st, p);
+    }
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -1091,8 +1091,9 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("gemm down: ") + cudaGetErrorString(e));
     h->n_gemm_up++;
     h->n_gemm_down++;
-    // router, decide, count, scatter, gather, gate/up GEMM, down GEMM (+ look-ahead tables, split-K finishes)
-    h->launches += 7 + (tabs_here ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
+    // router, decide, count (more than 256 tokens), scatter, gather, gate/up GEMM, down GEMM
+    // (+ look-ahead tables, split-K finishes)
+    h->launches += (T > 256 ? 7 : 6) + (tabs_here ? 1 : 0) + (g1.ksplit > 1 ? 1 : 0) + (g2.ksplit > 1 ? 1 : 0);
     if (has_sh) {
         GemmLaunch s1 = g1;
         s1.ksplit = 1;
