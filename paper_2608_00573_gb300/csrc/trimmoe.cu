@@ -14,6 +14,8 @@
 #include <utility>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "internal.cuh"
 
 using namespace tmoe;
@@ -71,6 +73,22 @@ inline bool pair_gemm(long long rows_per_group) { return rows_per_group >= kPair
 constexpr int kTransposedMinRows = 256;
 
 enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
+
+// NVTX range names per kernel family, nested in "trimmoe.layer_step" (itself
+// inside "trimmoe.forward" for a forward): a profiler can select a family's
+// kernels by the host ranges they were launched in, e.g. ncu --nvtx
+// --nvtx-include "trimmoe.layer_step/gemm_down/".  Host-side markers only: a
+// replayed forward graph is launched by one call, so its kernels carry only
+// the range open at that call ("trimmoe.forward").
+const char* const kKindName[K_NUM] = {"decide", "compact", "gather", "gemm_up", "gemm_down",
+                                      "combine", "router", "attn", "attn_gemm"};
+
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange&) = delete;
+    NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 inline float bf16_to_float(uint16_t b) {
     uint32_t u = (uint32_t)b << 16;
@@ -266,6 +284,7 @@ struct trimmoe {
     // Launch helper: records profile events around fn() when enabled.
     template <class Fn>
     cudaError_t timed(int kind, cudaStream_t st, Fn fn) {
+        NvtxRange range(kKindName[kind]);
         cudaEvent_t a = nullptr, b = nullptr;
         // Inside a stream capture the events become event-record nodes of the
         // graph (cudaEventRecordExternal), recorded at every replay.
@@ -765,6 +784,7 @@ static trimmoe_status check_tokens(trimmoe_handle h, const trimmoe_tokens* tok) 
 
 static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmoe_tokens* tok,
                                       trimmoe_layer_out* out, cudaStream_t st) {
+    NvtxRange range("trimmoe.layer_step");
     // Launch errors are read with cudaGetLastError after each launch; clear a
     // non-sticky error left behind by other code in this thread first.
     cudaGetLastError();
@@ -1266,6 +1286,7 @@ static trimmoe_status capture_forward(trimmoe_handle h, int T, trimmoe_tokens* t
 }
 
 static trimmoe_status run_forward(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st) {
+    NvtxRange range("trimmoe.forward");
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     const bool capturable = h->cfg.graphs && st != nullptr && st != cudaStreamLegacy && st != cudaStreamPerThread &&
                             cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone;
