@@ -224,6 +224,30 @@ def test_device_wait_timeout_is_reported_and_context_survives():
     eng.close()
 
 
+def test_create_out_of_memory_returns_status_and_recovers():
+    """Workspaces for 100 million tokens (terabytes) cannot be allocated:
+    trimmoe_create returns ERR_OOM with a message, frees what it had already
+    allocated, and a create that fits works afterwards on the same device."""
+    import torch
+    cfg = small_cfg(name="oom", N=2, d=4096, E=8, k=2, F=256, T=64, M=6, H=2, seed=71)
+    small = W.make_small_weights(cfg)
+    tables = W.make_tables(cfg, small["W_r"])
+    experts = W.make_expert_weights_host(cfg)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    with pytest.raises(B.TrimmoeError) as ei:
+        B.Engine(cfg, tables, small, experts, T_max=100_000_000)
+    assert ei.value.status == -3 and "allocation" in str(ei.value)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] >= free0 - (512 << 20)
+    eng = B.Engine(cfg, tables, small, experts, T_max=64)
+    dev = eng.tokens_to_device(W.make_tokens(cfg))
+    eng.layer_step(0, dev)
+    torch.cuda.synchronize()
+    assert eng.stats()["status"] == 0
+    eng.close()
+
+
 def test_create_rejects_bad_input():
     cfg = SMALL["swiglu_k2_renorm_h2"]
     small = W.make_small_weights(cfg)
