@@ -179,6 +179,27 @@ def make_workload(cfg, device):
     return small, tables, experts, tok
 
 
+def cpu_model() -> str:
+    """The host CPU's model string (x86 "model name", or the Arm implementer and
+    part numbers), with the machine type; never raises."""
+    import platform
+    name = ""
+    try:
+        info = {}
+        with open("/proc/cpuinfo") as fh:
+            for line in fh:
+                if ":" in line:
+                    k, v = line.split(":", 1)
+                    info.setdefault(k.strip(), v.strip())
+        if info.get("model name"):
+            name = info["model name"]
+        elif info.get("CPU part"):
+            name = f"implementer {info.get('CPU implementer', '?')} part {info['CPU part']}"
+    except OSError:
+        pass
+    return f"{name} ({platform.machine()})" if name else platform.machine()
+
+
 def cpu_baseline(cfg, small, tables, experts, tok, n_tok, n_layers, steps=1):
     """Time the oracle (all host cores) on n_tok tokens through layers 0..n_layers-1."""
     import numpy as np
@@ -233,7 +254,8 @@ def run_reference(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": cfg.name, "T": cfg.T, "N": cfg.N, "d": cfg.d, "E": cfg.E, "k": cfg.k,
                        "F": cfg.F, "F_sh": cfg.F_sh, "H": cfg.H, "budget": cfg.budget},
-            "cpu_baseline": {"value": v, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
+                             "cpu": cpu_model()},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -398,7 +420,7 @@ def run_ours(args):
         n_tok, n_layers = CPU_SAMPLE.get(cfg.name, (64, 2))
         vals, threads, sample = cpu_baseline(cfg, small, tables, experts, tok, n_tok, n_layers)
         line["cpu_baseline"] = {"value": vals[0], "unit": UNIT, "cores": threads, "kind": "oracle",
-                                "sample": sample}
+                                "sample": sample, "cpu": cpu_model()}
     eng.close()
     if rank == 0:
         print(json.dumps(line), flush=True)

@@ -60,3 +60,9 @@ def test_clock_sampler_without_nvidia_smi_reports_nothing(bench_mod, monkeypatch
     s = bench_mod.ClockSampler(0)
     s.start()
     assert s.stop() is None
+
+
+def test_cpu_model_names_the_host(bench_mod):
+    import platform
+    name = bench_mod.cpu_model()
+    assert isinstance(name, str) and platform.machine() in name
