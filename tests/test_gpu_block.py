@@ -12,7 +12,7 @@ import pytest
 from oracle import oracle as O
 from paper_2608_00573_gb300 import binding as B
 from paper_2608_00573_gb300 import workload as W
-from tests.gpu_helpers import compare_layer, make_engine
+from tests.gpu_helpers import compare_layer, make_engine, targeted_rows
 from tests.oracle_helpers import small_cfg
 
 pytestmark = pytest.mark.gpu
@@ -78,18 +78,27 @@ def test_full_block_single_token_sequences_and_tiny_batches():
 
 def test_full_block_mixtral_shape_sampled():
     """Mixtral-shaped full block (32 query / 8 key-value heads of 128, d = 4096,
-    user sequences of 128) on the benchmark's launch path: every decision is
-    compared; attention and hidden rows on a seeded sample from three
-    sequences."""
+    user sequences of 128) over 4200 tokens, so that the attention projections
+    run on CTA pairs with a ragged last tile and the last sequence is ragged.
+    Every decision is compared; the attention output and the hidden state on
+    rows aimed at the tile structure: the first and last token of every
+    128-token block (every row tile of the q/k/v and output projections, both
+    CTAs of each pair tile, and the first and last position of every
+    sequence), plus the MoE GEMMs' group edges and every 128-row block of every
+    expert group in the compacted order."""
     import torch
     base = W.with_attention(W.CONFIGS["mixtral"])
-    cfg = base.replace(N=2, T=1024)
+    T = 4200
+    cfg = base.replace(N=2, T=T)
     eng, om, tables, small, experts = make_engine(cfg, device_experts=True)
     dev = eng.tokens_to_device(W.make_tokens(cfg))
-    rng = np.random.default_rng(5)
-    sample = np.concatenate([s * 128 + np.sort(rng.choice(128, 12, replace=False)) for s in (0, 3, 7)])
+    edges = np.unique(np.concatenate([np.arange(0, T, 128), np.minimum(np.arange(127, T + 127, 128), T - 1)]))
+
+    def rows(g):
+        return np.union1d(edges, targeted_rows(g, T, cfg.k, cfg.E, tiles=True, extra=16, seed=5))
+
     for l in range(cfg.N):
-        r = compare_layer(cfg, om, eng, l, dev, experts, row_sample=sample)
-        print(l, r["exec"], r["skip"], r["exit"], r["attn_rel_err"], r["max_rel_err"])
+        r = compare_layer(cfg, om, eng, l, dev, experts, row_sample=rows)
+        print(l, r["exec"], r["skip"], r["exit"], r["attn_rel_err"], r["max_rel_err"], r["rows_checked"])
     eng.close()
     torch.cuda.synchronize()
