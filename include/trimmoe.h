@@ -134,8 +134,9 @@ typedef struct {
  *       (attn_heads > 0): RMSNorm weights of the attention sublayer, the fused
  *       query/key/value projection (query heads, then key heads, then value
  *       heads, Dh rows each) and the output projection.  Layer l then computes
- *       a = bf16(h r' gamma'), q|k|v = bf16(a W_qkv^T), rotary embedding on q
- *       and k, causal softmax attention (query head j reads key/value head
+ *       a = bf16(h r' gamma'); v = bf16(a W_v^T); q and k are rotated (rotary
+ *       embedding) in fp32 on the unrounded projection a W_q^T, a W_k^T and
+ *       rounded to bf16 once, after the rotation; causal softmax attention (query head j reads key/value head
  *       j / (Hq/Hkv)), h_mid = bf16(h + o W_o^T); the router, experts and
  *       residual read h_mid, the exit head of layer l-1 and the exit prediction
  *       read h (the state entering the layer), and a token that exits at layer
@@ -261,6 +262,11 @@ typedef struct {
      * 4*Dh*Hq*(causal query-key pairs)). */
     double ms_attn, ms_attn_gemm;
     double flops_attn, flops_attn_gemm;
+    /* Executed (token, slot) pairs, and the bytes of the expert weights that
+     * received work (each such expert's up and down projections once per
+     * layer call, plus the shared expert's when it ran). */
+    uint64_t pairs_executed;
+    double bytes_expert_weights;
 } trimmoe_stats_t;
 
 /* Validate, copy the tables, derive the candidate lists V_{l,r} and losses Q,

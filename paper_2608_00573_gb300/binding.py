@@ -73,7 +73,8 @@ class trimmoe_stats_t(C.Structure):
                 ("bytes_gemm_up", C.c_double), ("bytes_gemm_down", C.c_double),
                 ("lookahead_shared", C.c_uint64),
                 ("ms_attn", C.c_double), ("ms_attn_gemm", C.c_double), ("flops_attn", C.c_double),
-                ("flops_attn_gemm", C.c_double)]
+                ("flops_attn_gemm", C.c_double), ("pairs_executed", C.c_uint64),
+                ("bytes_expert_weights", C.c_double)]
 
     def as_dict(self):
         return {n: getattr(self, n) for n, _ in self._fields_}

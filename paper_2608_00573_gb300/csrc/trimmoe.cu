@@ -1465,6 +1465,9 @@ extern "C" trimmoe_status trimmoe_stats(trimmoe_handle h, trimmoe_stats_t* out) 
     out->flops_attn_gemm = h->flops_attn_gemm;
     out->n_gemm_up = h->n_gemm_up;
     out->n_gemm_down = h->n_gemm_down;
+    out->pairs_executed = dc.pairs_total;
+    out->bytes_expert_weights = 2.0 * ((double)dc.experts_touched * (n13F + FF) * dd +
+                                       (double)dc.shared_touched * 3.0 * Fs * dd);
     if (derr) return h->fail(TRIMMOE_ERR_DEVICE_TIMEOUT, "stats: a kernel timed out waiting");
     return TRIMMOE_OK;
 }
