@@ -399,10 +399,15 @@ trimmoe_status trimmoe_replicate(int N, int E, int M, const float* lambda, const
  * array of about 132 KB held by every GPU that loads the library until exit;
  * hence T <= 65536 and E <= 128 (ERR_ARG beyond, with a message in
  * trimmoe_last_error(NULL)).  It calls no cudaMalloc/cudaFree.  The first call on
- * each device looks up the array's device address once; make that first call
- * before any stream capture.  All calls share the array: calls whose work
- * overlaps on the GPU (other streams, other host threads) race and must be
- * serialised by the caller.  Asynchronous on stream. */
+ * each device looks up the array's device address once (cudaGetSymbolAddress)
+ * and keeps it; make that first call before any stream capture.  After
+ * cudaDeviceReset the device gets a new context in which the array may sit
+ * elsewhere: the next call notices the new context and looks the address up
+ * again, so the first call after a reset must also come before any capture.
+ * All calls share the array and it keeps the previous call's contents (the
+ * call clears what must start at zero): calls whose work overlaps on the GPU
+ * (other streams, other host threads) race and must be serialised by the
+ * caller.  Asynchronous on stream. */
 trimmoe_status trimmoe_compact_noalloc(const uint8_t* action, const uint8_t* exp_sel, int T, int k, int E,
                                        int has_shared, int32_t* perm, int32_t* group_off,
                                        int32_t* pos_pair, int32_t* pos_sh, void* stream);

@@ -400,16 +400,16 @@ cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st) 
 cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int head_dim, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
     if (p.S < 1 || p.S > kSeqMax || p.Hkv < 1 || p.Hq % p.Hkv || !tm_qkv) return cudaErrorInvalidValue;
-    static bool attr_set = false;
-    if (!attr_set) {
+    static PerDevice attr;
+    const cudaError_t ea = (cudaError_t)attr.get([] {
         cudaError_t e = cudaFuncSetAttribute(attention_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)attn_smem<64>());
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(attention_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)attn_smem<128>());
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+        return (int)e;
+    }, true);
+    if (ea != cudaSuccess) return ea;
     const dim3 grid(p.Hkv, (p.T + p.S - 1) / p.S);
     cudaError_t e;
     if (head_dim == 64) e = launch_pdl(attention_kernel<64>, grid, dim3(kAttnThreads), attn_smem<64>(), st, *tm_qkv, p);

@@ -103,13 +103,13 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
 
 template <int KT>
 int combine_grid(int T, int num_sms) {
-    static int per_sm = 0;
-    if (per_sm == 0) {
+    static PerDevice occ;
+    const int per_sm = occ.get([] {
         int n = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, combine_kernel<KT>, 256, 0) != cudaSuccess || n < 1)
             n = 1;
-        per_sm = n;
-    }
+        return n;
+    });
     const int want = (T + 7) / 8;
     const int cap = num_sms * per_sm;
     return want < cap ? want : cap;

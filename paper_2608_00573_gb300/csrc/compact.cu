@@ -268,14 +268,14 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
     if (max_rows <= 0) return cudaSuccess;
     if (d > kMaxGatherD) return cudaErrorInvalidValue;
     const size_t smem = gamma ? (size_t)d * 2 : 0;
-    static int per_sm = 0;
-    if (per_sm == 0) {
+    static PerDevice occ;
+    const int per_sm = occ.get([] {
         int n = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gather_kernel, 256, (size_t)kMaxGatherD * 2) !=
                 cudaSuccess || n < 1)
             n = 1;
-        per_sm = n;
-    }
+        return n;
+    });
     int blocks = (max_rows + 7) / 8;
     blocks = blocks < num_sms * per_sm ? blocks : num_sms * per_sm;
     const cudaError_t e = launch_pdl(gather_kernel, dim3(blocks), dim3(256), smem, st, perm, goff, E, k, d, h, rnorm,
@@ -317,9 +317,44 @@ namespace {
 constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mu;
 void* g_noalloc_ptr[kMaxDevices] = {nullptr};
+unsigned long long g_noalloc_ctx[kMaxDevices] = {0};
 
-// Device address of the scratch array on the current device, looked up once
-// per device (the host-side symbol is only a stand-in, never a device address).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Identity of the calling thread's current CUDA context (0 if the driver
+// entry points are unavailable or no context is current).  A context made
+// after cudaDeviceReset has a new identity, and the module holding the array
+// is loaded again there, possibly at another address.
+unsigned long long current_context_id(bool* available) {
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        void* q = nullptr;
+        cudaDriverEntryPointQueryResult r1, r2;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &r1) == cudaSuccess &&
+            r1 == cudaDriverEntryPointSuccess &&
+            cudaGetDriverEntryPointByVersion("cuCtxGetId", &q, 12000, cudaEnableDefault, &r2) == cudaSuccess &&
+            r2 == cudaDriverEntryPointSuccess) {
+            get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+            get_id = reinterpret_cast<CtxGetIdFn>(q);
+        }
+    });
+    *available = get_current && get_id;
+    if (!*available) return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+// Device address of the scratch array on the current device.  The host-side
+// symbol is only a stand-in, never a device address, so the address is looked
+// up with cudaGetSymbolAddress at set-up: on the first call on each device,
+// with that device current, and again only if the device's context has been
+// replaced since (cudaDeviceReset), never on other calls.
 trimmoe_status noalloc_scratch(tmoe::NoAllocScratch** out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
@@ -327,7 +362,10 @@ trimmoe_status noalloc_scratch(tmoe::NoAllocScratch** out) {
         return TRIMMOE_ERR_CUDA;
     }
     std::lock_guard<std::mutex> g(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
+    bool have_ids = false;
+    const unsigned long long ctx = current_context_id(&have_ids);
+    const bool stale = have_ids && (ctx == 0 || ctx != g_noalloc_ctx[dev]);
+    if (!g_noalloc_ptr[dev] || stale) {
         void* p = nullptr;
         const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
         if (e != cudaSuccess || !p) {
@@ -336,6 +374,8 @@ trimmoe_status noalloc_scratch(tmoe::NoAllocScratch** out) {
             return TRIMMOE_ERR_CUDA;
         }
         g_noalloc_ptr[dev] = p;
+        // The lookup makes the device's primary context current if none was.
+        g_noalloc_ctx[dev] = have_ids ? current_context_id(&have_ids) : 0;
     }
     *out = static_cast<tmoe::NoAllocScratch*>(g_noalloc_ptr[dev]);
     return TRIMMOE_OK;

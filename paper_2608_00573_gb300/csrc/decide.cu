@@ -629,16 +629,16 @@ cudaError_t launch_decide(const DecideParams& p, int num_sms, cudaStream_t st) {
     const int G = p.T >= num_sms * 16 ? decide_group(p.E) : 32;
     const bool la_global = p.la_scratch != nullptr;
     const size_t smem = decide_smem_for(p.E, p.C, p.M, p.tab.max_layer_cand, G, la_global);
-    static bool attr_set = false;
-    if (!attr_set) {
+    static PerDevice attr;
+    const cudaError_t ea = (cudaError_t)attr.get([] {
         cudaError_t e = cudaFuncSetAttribute(decide_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(decide_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(decide_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+        return (int)e;
+    }, true);
+    if (ea != cudaSuccess) return ea;
     if (smem > 200 * 1024) return cudaErrorInvalidValue;
     const int per_block = kWarps * (32 / G);
     int blocks = (p.T + per_block - 1) / per_block;

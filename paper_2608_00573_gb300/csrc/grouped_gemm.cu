@@ -851,45 +851,31 @@ namespace {
 
 // Clusters of two that fit on the device at once (the pair kernel is
 // persistent, so it launches no more than that); 0 if none.
-int pair_clusters(int num_sms) {
-    static int n = -1;
-    if (n >= 0) return n;
-    n = 0;
-    if (cudaFuncSetAttribute(grouped_gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kPairSmemBytes) != cudaSuccess)
-        return n;
+template <typename Kernel>
+int clusters_of_two(Kernel kernel, size_t smem, int num_sms) {
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+        return 0;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(num_sms & ~1), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kPairSmemBytes;
+    cfg.dynamicSmemBytes = smem;
     int ncl = 0;
-    if (cudaOccupancyMaxActiveClusters(&ncl, grouped_gemm_pair_kernel, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&ncl, kernel, &cfg) != cudaSuccess) {
         cudaGetLastError();
-        return n;
+        return 0;
     }
-    n = std::min(ncl, num_sms / 2);
-    return n;
+    return std::min(ncl, num_sms / 2);
+}
+
+int pair_clusters(int num_sms) {
+    static PerDevice n;
+    return n.get([num_sms] { return clusters_of_two(grouped_gemm_pair_kernel, kPairSmemBytes, num_sms); });
 }
 
 // The same for the transposed pair kernel (a little more shared memory).
 int pair_t_clusters(int num_sms) {
-    static int n = -1;
-    if (n >= 0) return n;
-    n = 0;
-    if (cudaFuncSetAttribute(grouped_gemm_pair_t_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kPairTSmemBytes) != cudaSuccess)
-        return n;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(num_sms & ~1), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kPairTSmemBytes;
-    int ncl = 0;
-    if (cudaOccupancyMaxActiveClusters(&ncl, grouped_gemm_pair_t_kernel, &cfg) != cudaSuccess) {
-        cudaGetLastError();
-        return n;
-    }
-    n = std::min(ncl, num_sms / 2);
-    return n;
+    static PerDevice n;
+    return n.get([num_sms] { return clusters_of_two(grouped_gemm_pair_t_kernel, kPairTSmemBytes, num_sms); });
 }
 
 }  // namespace
@@ -897,13 +883,12 @@ int pair_t_clusters(int num_sms) {
 int grouped_gemm_pair_clusters(int num_sms) { return pair_clusters(num_sms); }
 
 cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t st) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)kSmemBytes);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static PerDevice attr;
+    const cudaError_t ea = (cudaError_t)attr.get([] {
+        return (int)cudaFuncSetAttribute(grouped_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    }, true);
+    if (ea != cudaSuccess) return ea;
     if (g.ngroups <= 0 || g.ngroups > kMaxGroups || g.K % BK != 0) return cudaErrorInvalidValue;
     // Row tiles per block: about 48 MB of activations (a third of L2), so that
     // a block stays resident while the weight tiles stream past it.

@@ -8,6 +8,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
 #include <string>
 #include <utility>
 
@@ -288,6 +290,36 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
+
+// Launch set-up kept per device: function attributes (dynamic shared memory
+// limits) belong to a device's context and occupancy figures are per device,
+// so one process-wide flag would skip the set-up on a second device.  get()
+// runs f once for the current device under a lock and caches its result; with
+// only_zero the result is cached only when it is 0 (cudaSuccess), so a failed
+// set-up is tried again on the next call.
+class PerDevice {
+  public:
+    static constexpr int kMaxDevices = 64;
+    template <class F>
+    int get(F&& f, bool only_zero = false) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return f();
+        if (done_[dev].load(std::memory_order_acquire)) return val_[dev];
+        std::lock_guard<std::mutex> g(mu_);
+        if (done_[dev].load(std::memory_order_relaxed)) return val_[dev];
+        const int v = f();
+        if (!only_zero || v == 0) {
+            val_[dev] = v;
+            done_[dev].store(true, std::memory_order_release);
+        }
+        return v;
+    }
+
+  private:
+    std::mutex mu_;
+    std::atomic<bool> done_[kMaxDevices] = {};
+    int val_[kMaxDevices] = {};
+};
 
 // Error text for calls made without a handle (read by trimmoe_last_error(NULL)).
 void set_global_error(const std::string& msg);

@@ -280,14 +280,14 @@ cudaError_t launch_router(const CUtensorMap* tmA, const CUtensorMap* tmBhi, cons
     if (p.d % kKS || p.ksplit < 1 || (p.d / kKS) % p.ksplit || p.ng < 8 || p.ng > kNG || p.ng % 8 ||
         p.nl < 0 || p.nl > p.ng || p.nl % 8 || !tmA || !tmBhi || (p.nl > 0 && !tmBlo))
         return cudaErrorInvalidValue;
-    static bool attr_set = false;
-    if (!attr_set) {
+    static PerDevice attr;
+    const cudaError_t ea = (cudaError_t)attr.get([] {
         cudaError_t e = cudaSuccess;
         for (const void* f : {(const void*)router_kernel<1>, (const void*)router_kernel<2>, (const void*)router_kernel<4>})
             if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBudget);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+        return (int)e;
+    }, true);
+    if (ea != cudaSuccess) return ea;
     const int nt = p.ng / 8;
     if (nt != 1 && nt != 2 && nt != 4) return cudaErrorInvalidValue;
     const int stages = stages_for(p.ng, p.nl);

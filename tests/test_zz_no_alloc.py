@@ -11,7 +11,7 @@ import pytest
 
 from paper_2608_00573_gb300 import binding as B
 from paper_2608_00573_gb300 import workload as W
-from tests.gpu_helpers import make_engine
+from tests.gpu_helpers import expected_compaction, make_engine
 from tests.oracle_helpers import small_cfg
 
 pytestmark = pytest.mark.gpu
@@ -68,3 +68,49 @@ def test_compact_noalloc_rejects_oversized_input():
     assert "65536" in str(ei.value)
     with pytest.raises(B.TrimmoeError):
         B.trimmoe_compact_noalloc(a, a, 8, 1, 129, 0, i32, i32, i32, None)
+
+
+@pytest.mark.parametrize("has_shared", [0, 1])
+@pytest.mark.parametrize("T", [0, 1, 200, 1000, 65536])
+def test_compact_noalloc_matches_stable_sort_and_allocates_nothing(T, has_shared):
+    """Synthetic decisions (all four actions, every expert) at the single-chunk
+    size (T <= 256), several chunks, the 65536-token limit and T = 0: the
+    output equals the stable sort by (expert, t, j) that defines the
+    compaction, twice in a row, and after a first call the device's free
+    memory does not change across a call."""
+    import torch
+    K, E = 2, 8
+    rng = np.random.default_rng(T + 7 * has_shared)
+    action_h = rng.choice(4, size=max(T, 1), p=[0.7, 0.15, 0.1, 0.05]).astype(np.uint8)[:T]
+    exp_h = rng.integers(0, E, size=T * K).astype(np.uint8)
+    exp_h[np.repeat(action_h != 0, K)] = 255          # as the layer step writes it
+    action = torch.from_numpy(np.concatenate([action_h, np.zeros(1, np.uint8)])).cuda()
+    exp_sel = torch.from_numpy(np.concatenate([exp_h, np.zeros(1, np.uint8)])).cuda()
+    perm = torch.full((T * K + T + 1,), -7, dtype=torch.int32, device="cuda")
+    goff = torch.full((E + 2,), -7, dtype=torch.int32, device="cuda")
+    pos_pair = torch.full((T * K + 1,), -7, dtype=torch.int32, device="cuda")
+    pos_sh = torch.full((T + 1,), -7, dtype=torch.int32, device="cuda") if has_shared else None
+    stream = torch.cuda.current_stream().cuda_stream
+    want_perm, want_goff = expected_compaction(action_h, exp_h, T, K, E, bool(has_shared))
+
+    def call():
+        B.trimmoe_compact_noalloc(action, exp_sel, T, K, E, has_shared, perm, goff, pos_pair, pos_sh, stream)
+        torch.cuda.synchronize()
+
+    call()                                           # first call: set-up on this device
+    torch.cuda.synchronize()
+    free_before = torch.cuda.mem_get_info()[0]
+    for _ in range(2):
+        perm.fill_(-7)
+        call()
+        assert np.array_equal(goff.cpu().numpy(), want_goff)
+        got = perm.cpu().numpy()
+        n = len(want_perm)
+        assert np.array_equal(got[:n], want_perm)
+        assert np.all(got[n:] == -7)                  # nothing written past the rows
+        if T:
+            pp = pos_pair.cpu().numpy()[:T * K]
+            ex = np.repeat(action_h == 0, K)
+            assert np.all(pp[~ex] == -1)
+            assert np.array_equal(got[pp[ex]], np.nonzero(ex)[0])
+    assert torch.cuda.mem_get_info()[0] == free_before
