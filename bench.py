@@ -283,14 +283,17 @@ def cpu_baseline(cfg, small, tables, ex_l, tok):
     """The oracle on the host cores: a bounded sample on every core (the
     headline), a smaller one on one thread, and the tiny workload's full
     forward both ways."""
+    from oracle import oracle as O
     n_tok, n_layers = CPU_SAMPLE.get(cfg.name, (64, 2))
-    vals, secs, threads, sample = cpu_sample(cfg, small, tables, ex_l, tok, n_tok, n_layers)
+    cores = O.max_threads()          # before any single-thread run changes the OpenMP default
+    vals, secs, threads, sample = cpu_sample(cfg, small, tables, ex_l, tok, n_tok, n_layers, nthreads=cores)
+    tiny = cpu_tiny_forward(cores)
     n1 = max(1, n_tok // 32)
     v1, s1, _, sample1 = cpu_sample(cfg, small, tables, ex_l, tok, n1, n_layers, nthreads=1)
     return {"value": vals[0], "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
             "cpu": cpu_model(),
             "single_thread": {"value": v1[0], "unit": UNIT, "cores": 1, "sample": sample1},
-            "tiny_forward": cpu_tiny_forward(), "tiny_forward_single_thread": cpu_tiny_forward(1)}
+            "tiny_forward": tiny, "tiny_forward_single_thread": cpu_tiny_forward(1)}
 
 
 def run_reference(args):
