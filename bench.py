@@ -330,7 +330,7 @@ def run_reference(args):
 STATE_BYTES_PER_TOKEN_LAYER = 19 + 13
 
 
-def rooflines(cfg, st, steps, ms_step, peaks, traffic):
+def rooflines(cfg, st, steps, ms_step, peaks, traffic, st_k=None):
     """The dominant GEMM launch kind's roofline and the whole forward's.
 
     Forward: F_alg = executed expert GEMM FLOPs + router/exit-head/centroid dot
@@ -338,10 +338,12 @@ def rooflines(cfg, st, steps, ms_step, peaks, traffic):
     work (once per layer), the router/exit-head/norm rows of every layer run,
     and per live token-layer its hidden row in and out plus its state.  Roofline
     time = max(F_alg / bf16 peak, B_alg / HBM peak); frac = roofline / measured,
-    against the dense burst peak, with the sustained peak beside it."""
-    kinds = {"grouped_gemm_gate_up": (st["ms_gemm_up"], st["flops_gemm_up"], st["n_gemm_up"], st["bytes_gemm_up"]),
-             "grouped_gemm_down": (st["ms_gemm_down"], st["flops_gemm_down"], st["n_gemm_down"],
-                                   st["bytes_gemm_down"])}
+    against the dense burst peak, with the sustained peak beside it.  st_k:
+    the counters of the pass whose events timed the GEMM launches (default st)."""
+    sk = st if st_k is None else st_k
+    kinds = {"grouped_gemm_gate_up": (sk["ms_gemm_up"], sk["flops_gemm_up"], sk["n_gemm_up"], sk["bytes_gemm_up"]),
+             "grouped_gemm_down": (sk["ms_gemm_down"], sk["flops_gemm_down"], sk["n_gemm_down"],
+                                   sk["bytes_gemm_down"])}
     dom = max(kinds, key=lambda k: kinds[k][0])
     ms_k, fl_k, n_k, by_k = kinds[dom]
     achieved = fl_k / (ms_k / 1e3) / 1e12 if ms_k > 0 else 0.0
@@ -356,7 +358,7 @@ def rooflines(cfg, st, steps, ms_step, peaks, traffic):
         roof = {"bound": "hbm", "kernel": dom, "achieved": achieved_bw, "peak": peaks["hbm"], "unit": "GB/s",
                 "frac": achieved_bw / peaks["hbm"], "traffic": traffic, "peak_source": f"{peaks['source']} HBM copy"}
     roof.update(flops_per_launch=fl_k / max(n_k, 1), bytes_per_launch=by_k / max(n_k, 1),
-                ms_per_launch=ms_k / max(n_k, 1), launches_per_step=n_k / max(steps, 1))
+                ms_per_launch=ms_k / max(n_k, 1), launches_per_step=n_k / max(steps, 1) if st_k is None else None)
     rows = cfg.E + cfg.C + cfg.n_centroids
     live = st["layer_tokens"] / steps
     layers_run = st["layer_calls"] / steps
@@ -468,19 +470,28 @@ def extra_workloads(args, device, local, peaks, mixtral_experts):
     forwards and the Mixtral-shaped decode stress case (T in {1, 8, 64, 256} at
     budget 0.02, and T = 64 at budgets 0.005 and 0.05), each step on a fresh
     initial state drawn from a pool of 16.  The decode case reuses the resident
-    Mixtral-shaped expert weights."""
+    Mixtral-shaped expert weights.  The step time comes from a pass without
+    per-kernel events (at these sizes the event nodes inside the graph cost a
+    noticeable share of the step); the dominant GEMM's launch time from a
+    second pass of the same steps with events around the GEMM launches."""
     import torch
     from paper_2608_00573_gb300 import workload as W
     out = {}
 
-    def record(name, cfg, timed, steps, warmup):
+    def record(name, cfg, tables, small, experts, pool, steps, warmup):
+        timed = Timed(cfg, tables, small, experts, pool, device, profile=0)
         ms, clk, st = timed.run(steps, warmup, clock_index=local)
-        roof, fwd = rooflines(cfg, st, steps, ms, peaks, stored_traffic(cfg, "grouped_gemm_gate_up"))
+        timed.close()
+        ksteps = min(steps, 200)
+        timed = Timed(cfg, tables, small, experts, pool, device, profile=2)
+        _, _, st_k = timed.run(ksteps, warmup)
+        timed.close()
+        roof, fwd = rooflines(cfg, st, steps, ms, peaks, stored_traffic(cfg, "grouped_gemm_gate_up"), st_k=st_k)
+        roof["timing"] = f"events around the GEMM launches in a second pass of {ksteps} steps"
         out[name] = {"workload": cfg.name, "T": cfg.T, "N": cfg.N, "budget": cfg.budget, "steps": steps,
                      "warmup": warmup, "ms_per_step": ms, "tokens_per_s": cfg.T / (ms / 1e3),
                      "roofline": roof, "forward_roofline": fwd, "decisions": decisions_block(st, steps, cfg.T),
                      "gpu_launches": st["launches"], "clocks": clk}
-        timed.close()
 
     dec = W.CONFIGS["mixtral_decode"]
     runs = [(T, dec.budget) for T in (1, 8, 64, 256)] + [(64, 0.005), (64, 0.05)]
@@ -490,12 +501,11 @@ def extra_workloads(args, device, local, peaks, mixtral_experts):
         tables = W.make_tables(cfg, small["W_r"])
         pool = [W.make_tokens(cfg, T=T, seed_offset=1000 * T + i) for i in range(16)]
         name = f"mixtral_decode_T{T}" + ("" if budget == dec.budget else f"_budget{budget:g}")
-        record(name, cfg, Timed(cfg, tables, small, mixtral_experts, pool, device), args.decode_steps,
-               max(args.warmup, 3))
+        record(name, cfg, tables, small, mixtral_experts, pool, args.decode_steps, max(args.warmup, 3))
     for wl, steps in (("qwen", max(args.steps, 50)), ("switch", max(args.steps, 400))):
         cfg = W.CONFIGS[wl]
         small, tables, experts, tok = make_workload(cfg, device)
-        record(wl, cfg, Timed(cfg, tables, small, experts, [tok], device), steps, max(args.warmup, 3))
+        record(wl, cfg, tables, small, experts, [tok], steps, max(args.warmup, 3))
         del experts
         torch.cuda.empty_cache()
     return out
