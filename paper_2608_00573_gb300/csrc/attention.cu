@@ -7,7 +7,8 @@
 //
 //   a       = bf16(h * r * gamma_attn),  r = 1/sqrt(mean(h^2) + eps)   (attn_norm_kernel)
 //   q, k    = bf16(rope(a W_q^T)), bf16(rope(a W_k^T)), v = bf16(a W_v^T)
-//                                  (grouped GEMM, one group, rotary epilogue)
+//                                  (grouped GEMM, one group, rotary epilogue;
+//                                  v is stored transposed per sequence)
 //   o       = softmax(q k^T / sqrt(Dh), causal) v                      (attention_kernel)
 //   h_mid   = bf16(h + o W_o^T)                                       (grouped GEMM, residual epilogue)
 //
@@ -19,26 +20,20 @@
 //
 // The rotary embedding (pairs i, i + Dh/2, angle pos * theta^(-2i/Dh) from a
 // host-made cos/sin table) is applied by the projection GEMM's epilogue to the
-// fp32 accumulators before their bf16 rounding.
+// fp32 accumulators before their bf16 rounding.  The same epilogue writes the
+// value heads as V^T[sequence][value dim][key slot] (128 slots per sequence),
+// the K-major operand of O = P V.
 //
-// attention_kernel: one CTA per (key/value head, sequence), 320 threads, on
-// the 5th-generation tensor cores.  S <= 128 keys fit one tile, so there is no
-// running maximum: per query head of the group
-//   S = Q K^T          tcgen05.mma M = 128 (queries), N = 128 (keys), K = Dh -> TMEM
-//   P = exp(scale (S - max))   causal mask, fp32 (exp as one ex2.approx per
-//                      key), rounded to bf16 into shared memory by the 256
-//                      softmax threads (two per query row, one per key half;
-//                      a warp skips the 32-key chunks above its rows' diagonal)
-//   O = P V            tcgen05.mma M = 128, N = Dh, K = 128 keys -> TMEM
-//   out = bf16(O / l)  l = the fp32 row sum of the unrounded probabilities
-// warp 0 loads K and V of the group once and the query heads one after another
-// (TMA, 128-byte swizzle); warp 1 issues the MMAs; warps 2-9 transpose V once
-// into a K-major tile (keys contiguous, so that every operand is K-major), then
-// run the softmax and the epilogue of each head (two warps per 32 query rows,
-// one per half of the keys) while the tensor core computes the next head's
-// scores.  Rows past the sequence are loaded (the next
-// sequence's rows, or zero fill) but masked as keys and never stored as
-// queries.  Every wait is bounded (2 s) and records an error word on expiry.
+// attention_kernel: one CTA per (query head, sequence), 192 threads, two
+// CTAs per SM (three at head_dim 64), on the 5th-generation tensor cores.
+// S <= 128 keys fit one tile, so there is no running maximum:
+//   S = Q K^T   tcgen05.mma M = 128 (queries), N = 128 (keys), K = Dh -> TMEM
+//   P = exp(scale (S - max))   causal mask, fp32 (one ex2.approx per key),
+//               rounded to bf16 into shared memory over Q by four warps, one
+//               query row per thread
+//   O = P V     tcgen05.mma M = 128, N = Dh, K = 128 keys -> the same TMEM columns
+//   out = bf16(O / l)   l = the fp32 row sum of the unrounded probabilities
+// Several CTAs per SM overlap one CTA's loads with another's softmax.
 #include "internal.cuh"
 
 namespace tmoe {
@@ -101,26 +96,23 @@ __global__ void __launch_bounds__(256) attn_norm_kernel(const AttnParams p) {
     }
 }
 
-constexpr int kAttnThreads = 320;            // load warp, MMA warp, 8 softmax / epilogue warps
+constexpr int kAttnThreads = 192;            // load warp, MMA warp, 4 softmax / epilogue warps
 
 // Shared-memory layout (byte offsets from a 1024-aligned base).  A box is 128
-// rows x 64 bf16 columns (16 KB, 128-byte rows, 128-byte swizzle).
+// rows x 64 bf16 columns (16 KB, 128-byte rows, 128-byte swizzle).  P is
+// written over Q once S = Q K^T has been computed.
 template <int DH>
 struct AttnLayout {
     static constexpr int KB = DH / 64;                    // 64-column blocks of a head
     static constexpr int BOX = 128 * 128;
-    static constexpr int Q = 0;                           // [KB][128 query rows][128 B]
-    static constexpr int K = Q + KB * BOX;                // [KB][128 key rows][128 B]
-    static constexpr int V = K + KB * BOX;                // as loaded: [KB][128 key rows][64 dims]
-    static constexpr int VT = V + KB * BOX;               // [2 key blocks][DH dim rows][64 keys]
-    static constexpr int P = VT + 2 * DH * 128;           // [2 key blocks][128 query rows][64 keys]
-    static constexpr int X = P + 2 * BOX;                 // row maxima and sums of the two key halves
-    static constexpr int BYTES = X + 4 * 128 * 4;
+    static constexpr int QP = 0;                          // Q: [KB][128 query rows][128 B]; P: [2][128][128 B]
+    static constexpr int K = QP + 2 * BOX;                // [KB][128 key rows][128 B]
+    static constexpr int VT = K + KB * BOX;               // [2 key blocks][DH dim rows][64 keys]
+    static constexpr int BYTES = VT + 2 * DH * 128;
 };
 
 struct __align__(8) AttnBars {
-    uint64_t kv, q, vt, s, sfree, pfull, pfree, o, ofree, qfree;
-    uint64_t pair[4];          // the two softmax warps of a TMEM lane quarter
+    uint64_t ld, s, p, o;
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -130,10 +122,29 @@ constexpr size_t attn_smem() {
     return 1024 + (size_t)AttnLayout<DH>::BYTES + sizeof(AttnBars);
 }
 
+// One CTA per (query head, sequence), 192 threads, two or three CTAs per SM:
+//   warp 0     TMA: Q of the head, K of its key/value head (rows of the q/k/v
+//              projection) and V^T of the key/value head (the projection's
+//              epilogue stores V transposed per sequence, keys contiguous);
+//              owns the TMEM allocation (128 columns)
+//   warp 1     S = Q K^T (M = 128 queries, N = 128 keys, K = Dh) into TMEM,
+//              then O = P V (M = 128, N = Dh, K = 128 keys) into the same
+//              columns once every row of S has been read
+//   warps 2-5  one query row per thread (TMEM lane quarter warp % 4): the row
+//              maximum over its causal keys from a first read of S, then
+//              p = 2^((s - max) scale log2 e) (one ex2.approx per key; keys
+//              past the diagonal or the sequence are 0) from a second read,
+//              rounded to bf16 into shared memory over Q, l = the fp32 sum of
+//              the unrounded p; finally out = bf16(O / l) for rows of the
+//              sequence
+// Rows past the sequence are loaded (the next sequence's rows, or zero fill)
+// and masked as keys, never stored as queries; their V^T slots hold zeros or
+// values of an earlier call, which the zero probabilities cancel.  Every wait
+// is bounded (2 s) and records an error word on expiry.
 template <int DH>
-__global__ void __launch_bounds__(kAttnThreads, 1)
-attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
-    pdl_wait();      // results of the preceding kernel in the stream
+__global__ void __launch_bounds__(kAttnThreads, 2)
+attention_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tm_vt,
+                 const AttnParams p) {
     using L = AttnLayout<DH>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -141,247 +152,167 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
     const uint32_t sb = smem_u32(smem);
     AttnBars* bars = reinterpret_cast<AttnBars*>(smem + L::BYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = blockIdx.x, b = blockIdx.y;
-    const int G = p.Hq / p.Hkv;                          // query heads per key/value head
+    const int hq = blockIdx.x, b = blockIdx.y;
+    const int g = hq / (p.Hq / p.Hkv);                   // key/value head of this query head
     const int t0 = b * p.S;
     const int n = min(p.S, p.T - t0);
-    const int kcol = (p.Hq + g) * DH, vcol = (p.Hq + p.Hkv + g) * DH;
 
     if (threadIdx.x == 0) {
-        mbar_init(smem_u32(&bars->kv), 1);
-        mbar_init(smem_u32(&bars->q), 1);
-        mbar_init(smem_u32(&bars->vt), 8);
+        mbar_init(smem_u32(&bars->ld), 1);
         mbar_init(smem_u32(&bars->s), 1);
-        mbar_init(smem_u32(&bars->sfree), 8);
-        mbar_init(smem_u32(&bars->pfull), 8);
-        mbar_init(smem_u32(&bars->pfree), 1);
+        mbar_init(smem_u32(&bars->p), 4);
         mbar_init(smem_u32(&bars->o), 1);
-        mbar_init(smem_u32(&bars->ofree), 8);
-        for (int j = 0; j < 4; ++j) mbar_init(smem_u32(&bars->pair[j]), 2);
-        mbar_init(smem_u32(&bars->qfree), 1);
         bars->abort_flag = 0;
         fence_barrier_init();
         prefetch_tmap(&tm);
+        prefetch_tmap(&tm_vt);
     }
-    if (warp == 0) tmem_alloc(smem_u32(&bars->tmem_base), 256);
+    if (warp == 0) tmem_alloc(smem_u32(&bars->tmem_base), 128);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tS = bars->tmem_base, tO = bars->tmem_base + 128;
+    const uint32_t tS = bars->tmem_base;                 // S, then O in the same columns
     volatile int* abort_flag = &bars->abort_flag;
+    pdl_wait();      // q/k/v and V^T written by the projection
 
     if (warp == 0) {
         if (lane == 0) {
             // ------------------------------------------------------- loads
-            const uint32_t kvb = smem_u32(&bars->kv);
-            mbar_arrive_expect_tx(kvb, 2 * L::KB * L::BOX);
+            const uint32_t lb = smem_u32(&bars->ld);
+            mbar_arrive_expect_tx(lb, 2 * L::KB * L::BOX + 2 * DH * 128);
+            const int qcol = hq * DH, kcol = (p.Hq + g) * DH;
             for (int kb = 0; kb < L::KB; ++kb) {
-                tma_load_2d(sb + L::K + kb * L::BOX, &tm, kcol + kb * 64, t0, kvb);
-                tma_load_2d(sb + L::V + kb * L::BOX, &tm, vcol + kb * 64, t0, kvb);
+                tma_load_2d(sb + L::QP + kb * L::BOX, &tm, qcol + kb * 64, t0, lb);
+                tma_load_2d(sb + L::K + kb * L::BOX, &tm, kcol + kb * 64, t0, lb);
             }
-            for (int i = 0; i < G; ++i) {
-                if (i > 0 && !mbar_wait_bounded(smem_u32(&bars->qfree), (i - 1) & 1, abort_flag, p.err,
-                                                ERR_TIMEOUT_ATTN))
-                    break;
-                const uint32_t qb = smem_u32(&bars->q);
-                mbar_arrive_expect_tx(qb, L::KB * L::BOX);
-                const int qcol = (g * G + i) * DH;
-                for (int kb = 0; kb < L::KB; ++kb) tma_load_2d(sb + L::Q + kb * L::BOX, &tm, qcol + kb * 64, t0, qb);
-            }
+            const int vrow = (b * p.Hkv + g) * DH;
+            for (int kb = 0; kb < 2; ++kb) tma_load_2d(sb + L::VT + kb * DH * 128, &tm_vt, kb * 64, vrow, lb);
         }
     } else if (warp == 1) {
         if (lane == 0) {
             // ------------------------------------------------------- MMAs
             constexpr uint32_t idS = idesc_bf16_f32(128, 128);
             constexpr uint32_t idO = idesc_bf16_f32(128, DH);
-            bool ok = mbar_wait_bounded(smem_u32(&bars->kv), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
-                      mbar_wait_bounded(smem_u32(&bars->vt), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
-            for (int i = 0; i < G && ok; ++i) {
-                const uint32_t ph = i & 1, pph = (i - 1) & 1;
-                ok = mbar_wait_bounded(smem_u32(&bars->q), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
-                     (i == 0 || mbar_wait_bounded(smem_u32(&bars->sfree), pph, abort_flag, p.err, ERR_TIMEOUT_ATTN));
-                if (!ok) break;
+            if (mbar_wait_bounded(smem_u32(&bars->ld), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN)) {
                 tc_fence_after();
 #pragma unroll
                 for (int kb = 0; kb < L::KB; ++kb)
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
-                        tc_mma_bf16(tS, smem_desc_sw128(sb + L::Q + kb * L::BOX + kk * 32),
+                        tc_mma_bf16(tS, smem_desc_sw128(sb + L::QP + kb * L::BOX + kk * 32),
                                     smem_desc_sw128(sb + L::K + kb * L::BOX + kk * 32), idS, (kb | kk) ? 1u : 0u);
                 tc_commit(smem_u32(&bars->s));
-                tc_commit(smem_u32(&bars->qfree));
-                ok = mbar_wait_bounded(smem_u32(&bars->pfull), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
-                     (i == 0 || mbar_wait_bounded(smem_u32(&bars->ofree), pph, abort_flag, p.err, ERR_TIMEOUT_ATTN));
-                if (!ok) break;
-                tc_fence_after();
+                if (mbar_wait_bounded(smem_u32(&bars->p), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN)) {
+                    tc_fence_after();
 #pragma unroll
-                for (int kb = 0; kb < 2; ++kb)
+                    for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        tc_mma_bf16(tO, smem_desc_sw128(sb + L::P + kb * L::BOX + kk * 32),
-                                    smem_desc_sw128(sb + L::VT + kb * DH * 128 + kk * 32), idO, (kb | kk) ? 1u : 0u);
-                tc_commit(smem_u32(&bars->o));
-                tc_commit(smem_u32(&bars->pfree));
+                        for (int kk = 0; kk < 4; ++kk)
+                            tc_mma_bf16(tS, smem_desc_sw128(sb + L::QP + kb * L::BOX + kk * 32),
+                                        smem_desc_sw128(sb + L::VT + kb * DH * 128 + kk * 32), idO,
+                                        (kb | kk) ? 1u : 0u);
+                    tc_commit(smem_u32(&bars->o));
+                }
             }
         }
     } else {
         // ----------------------------------------------- softmax and epilogue
-        // Eight warps: warps w and w + 4 share TMEM lane quarter qw = w & 3 (32
-        // query rows) and take the key halves hk = 0 and 1; a row's maximum
-        // and sum combine the halves through shared memory (a two-arrival
-        // mbarrier per quarter, bounded waits), and the epilogue splits O's
-        // columns the same way.
-        const int qw = warp & 3;
-        const int hk = (warp - 2) >> 2;
+        const int qw = warp & 3;                         // TMEM lane quarter of this warp
         const int r = qw * 32 + lane;
         const uint32_t loff = (uint32_t)(qw * 32) << 16;
-        const int tid = threadIdx.x - 64;              // 0..255
-        float* xmax = reinterpret_cast<float*>(smem + L::X);     // [2][128]
-        float* xsum = xmax + 256;                                // [2][128]
-        const uint32_t pbar = smem_u32(&bars->pair[qw]);
-        int ok = 1;
-        // Both warps of the pair write, then wait for the pair (phase u of use k).
-        auto pair_sync = [&](uint32_t parity) -> int {
-            __syncwarp();
-            if (lane == 0) mbar_arrive(pbar);
-            int w = 1;
-            if (lane == 0) w = mbar_wait_bounded(pbar, parity, abort_flag, p.err, ERR_TIMEOUT_ATTN);
-            w = __shfl_sync(0xffffffffu, w, 0);
-            __syncwarp();
-            return w;
-        };
-        if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->kv), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (ok) {
-            // V^T: chunk (8 keys) kc of dimension row dim, from V[key][dim].
-            for (int idx = tid; idx < DH * 16; idx += 256) {
-                const int kc = idx / DH, dim = idx - (idx / DH) * DH;
-                const int db = dim >> 6, dc = (dim & 63) >> 3, de = (dim & 7) * 2;
-                uint32_t w[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int k0 = kc * 8 + 2 * e;
-                    const uint16_t v0 = *reinterpret_cast<const uint16_t*>(
-                        smem + L::V + db * L::BOX + k0 * 128 + ((dc ^ (k0 & 7)) << 4) + de);
-                    const uint16_t v1 = *reinterpret_cast<const uint16_t*>(
-                        smem + L::V + db * L::BOX + (k0 + 1) * 128 + ((dc ^ ((k0 + 1) & 7)) << 4) + de);
-                    w[e] = (uint32_t)v0 | ((uint32_t)v1 << 16);
-                }
-                *reinterpret_cast<uint4*>(smem + L::VT + (kc >> 3) * DH * 128 + dim * 128 +
-                                          (((kc & 7) ^ (dim & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
-            }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars->vt));
-        }
+        const int kmax = min(r, n - 1);                  // causal keys of this row
+        const int kq = min(qw * 32 + 31, n - 1);         // largest key any row of the quarter needs
         const float sl2 = p.scale * 1.4426950408889634f;
-        const int kmax = min(r, n - 1);
-        // 32-key chunks of this warp's half that some row of the quarter needs.
-        const int kq = min(qw * 32 + 31, n - 1);
-        for (int i = 0; i < G && ok; ++i) {
-            const uint32_t ph = i & 1, pph = (i - 1) & 1;
-            if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->s), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) break;
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->s), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        float l = 0.f;
+        if (ok) {
             tc_fence_after();
-            float sv[64];
+            float m = -INFINITY;
+#pragma unroll 1
+            for (int cc = 0; cc < 4; ++cc) {
+                if (cc * 32 > kq) break;
+                uint32_t u[32];
+                tmem_ld_32x32(tS + loff + cc * 32, u);
+                tmem_ld_wait();
 #pragma unroll
-            for (int cc = 0; cc < 2; ++cc) {
-                if ((2 * hk + cc) * 32 <= kq) {
+                for (int j = 0; j < 32; ++j)
+                    if (cc * 32 + j <= kmax) m = fmaxf(m, __uint_as_float(u[j]));
+            }
+            const float ms = m * sl2;
+#pragma unroll 1
+            for (int cc = 0; cc < 4; ++cc) {
+                uint4 w[4];
+                if (cc * 32 <= kq) {
                     uint32_t u[32];
-                    tmem_ld_32x32(tS + loff + (2 * hk + cc) * 32, u);
+                    tmem_ld_32x32(tS + loff + cc * 32, u);
                     tmem_ld_wait();
+                    float e[32];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) sv[cc * 32 + j] = __uint_as_float(u[j]);
+                    for (int j = 0; j < 32; ++j) {
+                        float x;
+                        asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(x) : "f"(fmaf(__uint_as_float(u[j]), sl2, -ms)));
+                        e[j] = (cc * 32 + j <= kmax) ? x : 0.f;
+                        l += e[j];
+                    }
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4)
+                        w[q4] = make_uint4(pack_bf16x2(e[8 * q4 + 0], e[8 * q4 + 1]),
+                                           pack_bf16x2(e[8 * q4 + 2], e[8 * q4 + 3]),
+                                           pack_bf16x2(e[8 * q4 + 4], e[8 * q4 + 5]),
+                                           pack_bf16x2(e[8 * q4 + 6], e[8 * q4 + 7]));
+                } else {
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) w[q4] = make_uint4(0u, 0u, 0u, 0u);
+                }
+                // keys [32 cc, 32 cc + 32): key block cc / 2, 16-byte chunks (cc & 1) * 4 + q4
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const int c16 = (cc & 1) * 4 + q4;
+                    *reinterpret_cast<uint4*>(smem + L::QP + (cc >> 1) * L::BOX + r * 128 + ((c16 ^ (r & 7)) << 4)) =
+                        w[q4];
                 }
             }
             tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars->sfree));
-            // Causal softmax over keys 0..kmax; exp(x) as 2^(x log2 e), one
-            // ex2.approx per key (P is rounded to bf16 next).
-            float m = -INFINITY;
-#pragma unroll
-            for (int cc = 0; cc < 2; ++cc)
-                if ((2 * hk + cc) * 32 <= kq)
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (64 * hk + cc * 32 + j <= kmax) m = fmaxf(m, sv[cc * 32 + j]);
-            xmax[hk * 128 + r] = m;
-            ok = pair_sync(0);
-            if (!ok) break;
-            m = fmaxf(xmax[r], xmax[128 + r]);
-            const float ms = m * sl2;
-            float l = 0.f;
-#pragma unroll
-            for (int cc = 0; cc < 2; ++cc) {
-                if ((2 * hk + cc) * 32 <= kq) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        float e;
-                        asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(fmaf(sv[cc * 32 + j], sl2, -ms)));
-                        sv[cc * 32 + j] = (64 * hk + cc * 32 + j <= kmax) ? e : 0.f;
-                        l += sv[cc * 32 + j];
-                    }
-                }
-            }
-            if (i > 0) {
-                if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->pfree), pph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
-                ok = __shfl_sync(0xffffffffu, ok, 0);
-                if (!ok) break;
-            }
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                uint4 w = make_uint4(0u, 0u, 0u, 0u);
-                if ((2 * hk + (c >> 2)) * 32 <= kq) {
-                    w.x = pack_bf16x2(sv[c * 8 + 0], sv[c * 8 + 1]);
-                    w.y = pack_bf16x2(sv[c * 8 + 2], sv[c * 8 + 3]);
-                    w.z = pack_bf16x2(sv[c * 8 + 4], sv[c * 8 + 5]);
-                    w.w = pack_bf16x2(sv[c * 8 + 6], sv[c * 8 + 7]);
-                }
-                *reinterpret_cast<uint4*>(smem + L::P + hk * L::BOX + r * 128 + ((c ^ (r & 7)) << 4)) = w;
-            }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars->pfull));
-            xsum[hk * 128 + r] = l;
-            // Epilogue: O / l as bf16, this half's columns, rows of the sequence only.
-            if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->o), ph, abort_flag, p.err, ERR_TIMEOUT_ATTN);
+            if (lane == 0) mbar_arrive(smem_u32(&bars->p));
+            if (lane == 0) ok = mbar_wait_bounded(smem_u32(&bars->o), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN);
             ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) break;
-            ok = pair_sync(1);
-            if (!ok) break;
+        }
+        if (ok) {
+            // Epilogue: out = bf16(O / l), rows of the sequence only.
             tc_fence_after();
-            const float il = 1.f / (xsum[r] + xsum[128 + r]);
-            __nv_bfloat16* orow = p.out + (size_t)(t0 + min(r, n - 1)) * p.Hq * DH + (size_t)(g * G + i) * DH;
-#pragma unroll
-            for (int c = hk * (DH / 2); c < (hk + 1) * (DH / 2); c += 32) {
+            const float il = 1.f / l;
+            __nv_bfloat16* orow = p.out + (size_t)(t0 + min(r, n - 1)) * p.Hq * DH + (size_t)hq * DH;
+#pragma unroll 1
+            for (int c = 0; c < DH; c += 32) {
                 uint32_t u[32];
-                tmem_ld_32x32(tO + loff + c, u);
+                tmem_ld_32x32(tS + loff + c, u);
                 tmem_ld_wait();
                 if (r < n) {
                     uint4* d4 = reinterpret_cast<uint4*>(orow + c);
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        uint4 w;
-                        w.x = pack_bf16x2(__uint_as_float(u[8 * q4 + 0]) * il, __uint_as_float(u[8 * q4 + 1]) * il);
-                        w.y = pack_bf16x2(__uint_as_float(u[8 * q4 + 2]) * il, __uint_as_float(u[8 * q4 + 3]) * il);
-                        w.z = pack_bf16x2(__uint_as_float(u[8 * q4 + 4]) * il, __uint_as_float(u[8 * q4 + 5]) * il);
-                        w.w = pack_bf16x2(__uint_as_float(u[8 * q4 + 6]) * il, __uint_as_float(u[8 * q4 + 7]) * il);
-                        d4[q4] = w;
-                    }
+                    for (int q4 = 0; q4 < 4; ++q4)
+                        d4[q4] = make_uint4(pack_bf16x2(__uint_as_float(u[8 * q4 + 0]) * il,
+                                                        __uint_as_float(u[8 * q4 + 1]) * il),
+                                            pack_bf16x2(__uint_as_float(u[8 * q4 + 2]) * il,
+                                                        __uint_as_float(u[8 * q4 + 3]) * il),
+                                            pack_bf16x2(__uint_as_float(u[8 * q4 + 4]) * il,
+                                                        __uint_as_float(u[8 * q4 + 5]) * il),
+                                            pack_bf16x2(__uint_as_float(u[8 * q4 + 6]) * il,
+                                                        __uint_as_float(u[8 * q4 + 7]) * il));
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(smem_u32(&bars->ofree));
         }
+        tc_fence_before();
     }
     __syncthreads();
     if (warp == 0) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(bars->tmem_base, 256);
+        tmem_dealloc(bars->tmem_base, 128);
     }
     pdl_trigger();   // the next kernel may be scheduled once every block got here or exited
 }
@@ -397,9 +328,10 @@ cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st) 
     return cudaGetLastError();
 }
 
-cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int head_dim, cudaStream_t st) {
+cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, const CUtensorMap* tm_vt, int head_dim,
+                             cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
-    if (p.S < 1 || p.S > kSeqMax || p.Hkv < 1 || p.Hq % p.Hkv || !tm_qkv) return cudaErrorInvalidValue;
+    if (p.S < 1 || p.S > kSeqMax || p.Hkv < 1 || p.Hq % p.Hkv || !tm_qkv || !tm_vt) return cudaErrorInvalidValue;
     static PerDevice attr;
     const cudaError_t ea = (cudaError_t)attr.get([] {
         cudaError_t e = cudaFuncSetAttribute(attention_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -410,11 +342,12 @@ cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int
         return (int)e;
     }, true);
     if (ea != cudaSuccess) return ea;
-    const dim3 grid(p.Hkv, (p.T + p.S - 1) / p.S);
+    const dim3 grid(p.Hq, (p.T + p.S - 1) / p.S);
     cudaError_t e;
-    if (head_dim == 64) e = launch_pdl(attention_kernel<64>, grid, dim3(kAttnThreads), attn_smem<64>(), st, *tm_qkv, p);
+    if (head_dim == 64)
+        e = launch_pdl(attention_kernel<64>, grid, dim3(kAttnThreads), attn_smem<64>(), st, *tm_qkv, *tm_vt, p);
     else if (head_dim == 128)
-        e = launch_pdl(attention_kernel<128>, grid, dim3(kAttnThreads), attn_smem<128>(), st, *tm_qkv, p);
+        e = launch_pdl(attention_kernel<128>, grid, dim3(kAttnThreads), attn_smem<128>(), st, *tm_qkv, *tm_vt, p);
     else return cudaErrorInvalidValue;
     if (e != cudaSuccess) return e;
     return cudaGetLastError();

@@ -69,12 +69,39 @@ __device__ __forceinline__ void grp_argmax(unsigned gmask, float& v, int& i) {
     }
 }
 
-// Execute cost f(m, k) of Eq. (31) from the delay table and the quality term.
-__device__ __forceinline__ float exec_cost(const DecideParams& p, const float* ct_row, int m, float Q,
-                                           float Dbar) {
-    float c = ct_row[m];
-    if (Q > 0.f) c = __fadd_rn(c, __fmul_rn(p.omega_D, __fdiv_rn(Q, Dbar)));
-    return c;
+// Sum of n partial sums base[0], base[stride], ... added in index order.  The
+// loads of a batch of eight are issued before the additions, so a token's
+// column ranges cost one memory latency per batch rather than one each (the
+// order of the additions, and so the result, is unchanged).
+__device__ __forceinline__ float sum_parts(const float* __restrict__ base, size_t stride, int n) {
+    float acc = 0.f;
+    int i = 0;
+    for (; i + 8 <= n; i += 8) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = base[(size_t)(i + u) * stride];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc = __fadd_rn(acc, v[u]);
+    }
+    for (; i < n; ++i) acc = __fadd_rn(acc, base[(size_t)i * stride]);
+    return acc;
+}
+
+// The same for up to kMS values at once: value u sums base[off + u * ustride]
+// over the n parts (u < nv), parts in index order.  Every load of one part is
+// issued before the additions.
+constexpr int kMS = 8;
+__device__ __forceinline__ void multi_sum(const float* __restrict__ base, size_t stride, int n, int off,
+                                          int ustride, int nv, float (&out)[kMS]) {
+#pragma unroll
+    for (int u = 0; u < kMS; ++u) out[u] = 0.f;
+    for (int i = 0; i < n; ++i) {
+        float v[kMS];
+#pragma unroll
+        for (int u = 0; u < kMS; ++u) v[u] = u < nv ? base[(size_t)i * stride + off + u * ustride] : 0.f;
+#pragma unroll
+        for (int u = 0; u < kMS; ++u) out[u] = __fadd_rn(out[u], v[u]);
+    }
 }
 
 struct WarpCounters {
@@ -132,7 +159,14 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
     WarpCounters wc = {};
     const int ngroups = gridDim.x * kGroups;
     for (int t = blockIdx.x * kGroups + slot; t < p.T; t += ngroups) {
-        if (!p.alive[t]) {
+        // The token's state is read before the liveness test: the loads overlap.
+        const int alive_t = p.alive[t];
+        const int s = p.s[t];
+        const float Dhat = p.Dhat[t];
+        const float Dbar = p.Dbar[t];
+        const float pJ = p.pJ[t];
+        const int last_exec = p.last_exec[t];
+        if (!alive_t) {
             if (lane == 0) {
                 p.action[t] = 3;
                 p.I_out[t] = 0.f;
@@ -147,27 +181,21 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
             }
             continue;
         }
-        const int s = p.s[t];
-        const float Dhat = p.Dhat[t];
-        const float Dbar = p.Dbar[t];
-        const float pJ = p.pJ[t];
-        const int last_exec = p.last_exec[t];
 
         // Router logits: partial dot products of kernel a0 summed over the column
         // ranges in order, times the RMS factor, plus the bias; softmax (Eq. 4),
         // top-k by logit (a NaN logit ranks as -infinity).
         float rn = 1.f;
+        const size_t kstride = (size_t)p.zs;      // the column ranges of a token are contiguous
+        const float* zrow = p.zpart + (size_t)t * p.ksplit * p.zs;
+        float zacc = lane < E ? sum_parts(zrow + lane, kstride, p.ksplit) : 0.f;
         if (p.use_norm) {
-            float sq = 0.f;
-            for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart[(size_t)t * p.ksplit + ks]);
+            const float sq = sum_parts(p.sqpart + (size_t)t * p.ksplit, 1, p.ksplit);
             rn = rsqrtf(sq / (float)p.d + p.norm_eps);
             if (lane == 0) p.rnorm[t] = rn;
         }
-        const size_t kstride = (size_t)p.zs;      // the column ranges of a token are contiguous
-        const float* zrow = p.zpart + (size_t)t * p.ksplit * p.zs;
         for (int e = lane; e < E; e += G) {
-            float acc = 0.f;
-            for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + e]);
+            const float acc = e == lane ? zacc : sum_parts(zrow + e, kstride, p.ksplit);
             const float v = __fadd_rn(__fmul_rn(acc, rn), p.bias[e]);
             zs[e] = (v != v) ? -kInf : v;
         }
@@ -208,14 +236,17 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
             // sublayer in front of the MoE step that state has its own RMS factor.
             float rx = rn;
             if (p.use_norm && p.sqpart_x) {
-                float sq = 0.f;
-                for (int ks = 0; ks < p.ksplit; ++ks) sq = __fadd_rn(sq, p.sqpart_x[(size_t)t * p.ksplit + ks]);
+                const float sq = sum_parts(p.sqpart_x + (size_t)t * p.ksplit, 1, p.ksplit);
                 rx = rsqrtf(sq / (float)p.d + p.norm_eps);
             }
-            for (int c = lane; c < C; c += G) {
-                float acc = 0.f;
-                for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + c]);
-                xs[c] = __fadd_rn(__fmul_rn(acc, rx), p.bias[E + c]);
+            // This lane's classes c = lane + G u, kMS at a time.
+            for (int c0 = lane; c0 < C; c0 += kMS * G) {
+                const int nv = min(kMS, (C - c0 + G - 1) / G);
+                float acc[kMS];
+                multi_sum(zrow, kstride, p.ksplit, E + c0, G, nv, acc);
+#pragma unroll
+                for (int u = 0; u < kMS; ++u)
+                    if (u < nv) xs[c0 + u * G] = __fadd_rn(__fmul_rn(acc[u], rx), p.bias[E + c0 + u * G]);
             }
             __syncwarp(gmask);
             if (C == 1) {
@@ -239,12 +270,18 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
         if (p.n_cent > 0) {
             float bsc = -kInf;
             int bj = 0x7fffffff;
-            for (int j = lane; j < p.n_cent; j += G) {
-                float acc = 0.f;
-                for (int ks = 0; ks < p.ksplit; ++ks) acc = __fadd_rn(acc, zrow[ks * kstride + E + C + j]);
-                const float cn = p.cnorm[j];
-                const float sc = cn > 0.f ? __fdiv_rn(acc, cn) : -kInf;
-                if (sc > bsc || (sc == bsc && j < bj)) { bsc = sc; bj = j; }
+            for (int j0 = lane; j0 < p.n_cent; j0 += kMS * G) {
+                const int nv = min(kMS, (p.n_cent - j0 + G - 1) / G);
+                float acc[kMS];
+                multi_sum(zrow, kstride, p.ksplit, E + C + j0, G, nv, acc);
+#pragma unroll
+                for (int u = 0; u < kMS; ++u) {
+                    if (u >= nv) continue;
+                    const int j = j0 + u * G;
+                    const float cn = p.cnorm[j];
+                    const float sc = cn > 0.f ? __fdiv_rn(acc[u], cn) : -kInf;
+                    if (sc > bsc || (sc == bsc && j < bj)) { bsc = sc; bj = j; }
+                }
             }
             grp_argmax<G>(gmask, bsc, bj);
             Lhat = p.lhat_tab[bj];
@@ -256,6 +293,7 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
         for (int j = 0; j < K; ++j) {
             const int c0 = coff_l[topk[j]], c1 = coff_l[topk[j] + 1];
             float gmin = kInf;
+#pragma unroll 4
             for (int c = c0 + lane; c < c1; c += G) {
                 const float Q = p.tab.cand_Q[c];
                 if (__fadd_rn(Dhat, Q) <= Dbar) {
@@ -353,14 +391,19 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
             const int c0 = coff_l[topk[j]], c1 = coff_l[topk[j] + 1];
             float bv = kInf;
             int bi = 0x7fffffff;
+#pragma unroll 4
             for (int c = c0 + lane; c < c1; c += G) {
                 const float Q = p.tab.cand_Q[c];
+                const int m = p.tab.cand_m[c];
+                const float ct = ct_s[m];
+                // the cost-to-go is read before the budget tests decide whether it is used
+                const float ph = (j == 0 && have_phi) ? phiP[m * E + p.tab.cand_k[c]] : 0.f;
                 if (!(__fadd_rn(Dhat, Q) <= Dbar)) continue;
                 if (!(__fadd_rn(Drun, Q) <= Dbar)) continue;
-                const int m = p.tab.cand_m[c];
-                const float f = exec_cost(p, ct_s, m, Q, Dbar);
+                float f = ct;
+                if (Q > 0.f) f = __fadd_rn(f, __fmul_rn(p.omega_D, __fdiv_rn(Q, Dbar)));
                 float v = f;
-                if (j == 0) v = __fadd_rn(f, have_phi ? phiP[m * E + p.tab.cand_k[c]] : 0.f);
+                if (j == 0) v = __fadd_rn(f, ph);
                 if (v < bv) { bv = v; bi = c; }
             }
             grp_argmin<G>(gmask, bv, bi);
@@ -409,14 +452,18 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
                 Dnew = Drun;
                 p.Dhat[t] = Dnew;
                 p.last_exec[t] = 1;
-                for (int j = 0; j < K; ++j) {
+                float dl = 0.f;
+#pragma unroll
+                for (int j = 0; j < kMaxK; ++j) {
+                    if (j >= K) break;
                     const bool remote = msel[j] != s;
                     const bool sub = esel[j] != topk[j];
                     if (remote) { if (sub) ++wc.rs; else ++wc.re; ++wc.hops; }
                     else { if (sub) ++wc.ls; else ++wc.le; }
                     const float tr = remote ? p.tab.trans[s * M + msel[j]] : 0.f;
-                    wc.delay += (double)(tr + p.tab.comp[l * M + msel[j]]);
+                    dl += tr + p.tab.comp[l * M + msel[j]];
                 }
+                wc.delay += (double)dl;
                 ++wc.exec_tokens;
             } else if (action == 1) {
                 Dnew = __fadd_rn(Dhat, Lambda);

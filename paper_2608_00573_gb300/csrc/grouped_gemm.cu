@@ -171,8 +171,7 @@ __device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float (&v)
 __device__ __forceinline__ void epilogue_tile(uint32_t tb, int row, const Tile& ti, int kr, int ksplit,
                                               int epi_mode, __nv_bfloat16* __restrict__ out, int ldo,
                                               const __nv_bfloat16* __restrict__ res, int ldr,
-                                              const float2* __restrict__ rope, int rope_S, int rope_dh,
-                                              int n_rot, float* __restrict__ partial, int ldp,
+                                              const RopeEpi& rp, float* __restrict__ partial, int ldp,
                                               size_t pstride) {
     const bool valid = row < ti.rows;
     __nv_bfloat16* orow = out + (size_t)(ti.out_row + (valid ? row : 0)) * ldo;
@@ -215,12 +214,13 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tb, int row, const Tile& 
         // Rotary embedding of the query and key heads in the leading n_rot
         // columns (pairs i, i + Dh/2 of each head; position = row mod S),
         // the remaining (value) heads stored as they are.
-        const int pos = (ti.out_row + (valid ? row : 0)) % rope_S;
-        const int half = rope_dh >> 1;
+        const int tok = ti.out_row + (valid ? row : 0);
+        const int pos = tok % rp.S;
+        const int half = rp.dh >> 1;
 #pragma unroll 1
-        for (int h0 = 0; h0 < BN; h0 += rope_dh) {
+        for (int h0 = 0; h0 < BN; h0 += rp.dh) {
             const int col0 = ti.nt * BN + h0;
-            if (col0 < n_rot) {
+            if (col0 < rp.n_rot) {
 #pragma unroll 1
                 for (int c = 0; c < half; c += 32) {
                     uint32_t xa[32], xb[32];
@@ -228,7 +228,7 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tb, int row, const Tile& 
                     tmem_ld_32x32(tb + h0 + half + c, xb);
                     tmem_ld_wait();
                     if (valid) {
-                        const float2* cs = rope + (size_t)pos * half + c;
+                        const float2* cs = rp.cs + (size_t)pos * half + c;
                         float ya[32], yb[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
@@ -241,9 +241,26 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tb, int row, const Tile& 
                         store_row32(orow + col0 + half + c, yb);
                     }
                 }
+            } else if (rp.vt) {
+                // Value heads, transposed per sequence: for each feature the
+                // warp's 32 tokens are 32 consecutive key slots (64-byte stores).
+                const int seq = tok / rp.S;
+                __nv_bfloat16* vcol =
+                    rp.vt + ((size_t)seq * rp.vt_rows + (col0 - rp.n_rot)) * kVtSlots + (tok - seq * rp.S);
+#pragma unroll 1
+                for (int c = 0; c < rp.dh; c += 32) {
+                    uint32_t r[32];
+                    tmem_ld_32x32(tb + h0 + c, r);
+                    tmem_ld_wait();
+                    if (valid) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            vcol[(size_t)(c + i) * kVtSlots] = __float2bfloat16_rn(__uint_as_float(r[i]));
+                    }
+                }
             } else {
 #pragma unroll 1
-                for (int c = 0; c < rope_dh; c += 32) {
+                for (int c = 0; c < rp.dh; c += 32) {
                     uint32_t r[32];
                     tmem_ld_32x32(tb + h0 + c, r);
                     tmem_ld_wait();
@@ -295,8 +312,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
                     int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                     __nv_bfloat16* __restrict__ out, int ldo, int* err,
-                    const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
-                    int rope_S, int rope_dh, int n_rot, int mblk, int ksplit, float* __restrict__ partial,
+                    const __nv_bfloat16* __restrict__ res, int ldr, const RopeEpi rp,
+                    int mblk, int ksplit, float* __restrict__ partial,
                     int ldp, size_t pstride) {
     pdl_wait();      // results of the preceding kernel in the stream
     pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
@@ -416,8 +433,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             if (!ok) break;
             tc_fence_after();
             const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
-            epilogue_tile(tb, row, ti, t / ntiles, ksplit, epi_mode, out, ldo, res, ldr, rope, rope_S, rope_dh,
-                          n_rot, partial, ldp, pstride);
+            epilogue_tile(tb, row, ti, t / ntiles, ksplit, epi_mode, out, ldo, res, ldr, rp, partial, ldp,
+                          pstride);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&tl->tempty[buf]));
@@ -445,8 +462,7 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
                          const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
                          int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                          __nv_bfloat16* __restrict__ out, int ldo, int* err,
-                         const __nv_bfloat16* __restrict__ res, int ldr, const float2* __restrict__ rope,
-                         int rope_S, int rope_dh, int n_rot, int mblk) {
+                         const __nv_bfloat16* __restrict__ res, int ldr, const RopeEpi rp, int mblk) {
     pdl_wait();      // results of the preceding kernel in the stream
     pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint8_t smem_raw[];
@@ -564,8 +580,7 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
             if (!ok) break;
             tc_fence_after();
             const uint32_t tb = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
-            epilogue_tile(tb, row, ti, 0, 1, epi_mode, out, ldo, res, ldr, rope, rope_S, rope_dh, n_rot, nullptr,
-                          0, 0);
+            epilogue_tile(tb, row, ti, 0, 1, epi_mode, out, ldo, res, ldr, rp, nullptr, 0, 0);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
@@ -890,6 +905,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     }, true);
     if (ea != cudaSuccess) return ea;
     if (g.ngroups <= 0 || g.ngroups > kMaxGroups || g.K % BK != 0) return cudaErrorInvalidValue;
+    const RopeEpi rp{g.rope, g.rope_S, g.rope_dh, g.n_rot, g.vt, g.vt_rows};
     // Row tiles per block: about 48 MB of activations (a third of L2), so that
     // a block stays resident while the weight tiles stream past it.
     const long long a_tile_bytes = (long long)BM * g.K * 2;
@@ -912,8 +928,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
         const cudaError_t e = launch_pdl(
             grouped_gemm_pair_kernel, dim3(2 * pair_clusters(num_sms)), dim3(kThreads), kPairSmemBytes, st, *g.tmA,
             *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot,
-            mblk2);
+            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, rp, mblk2);
         if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }
@@ -921,8 +936,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     const cudaError_t e = launch_pdl(
         grouped_gemm_kernel, dim3(num_sms), dim3(kThreads), kSmemBytes, st, *g.tmA, *g.tmB, g.goff, g.first_group,
         g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n, g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err,
-        g.res, g.ldr, g.rope, g.rope_S, g.rope_dh, g.n_rot, mblk, g.ksplit > 1 ? g.ksplit : 1, g.partial, g.ldp,
-        g.pstride);
+        g.res, g.ldr, rp, mblk, g.ksplit > 1 ? g.ksplit : 1, g.partial, g.ldp, g.pstride);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

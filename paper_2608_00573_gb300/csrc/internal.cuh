@@ -177,6 +177,11 @@ struct GemmLaunch {
     int ldr;
     const float2* rope;         // EPI_ROPE: (cos, sin) [rope_S][rope_dh/2]
     int rope_S, rope_dh, n_rot; // sequence length, head dim, leading columns that rotate
+    // EPI_ROPE: the columns past n_rot (the value heads, vt_rows of them) are
+    // stored transposed per sequence instead: vt[(seq * vt_rows + col - n_rot)
+    // * kVtSlots + pos] for the token at position pos of sequence seq.
+    __nv_bfloat16* vt;
+    int vt_rows;
     // Split over K (ksplit > 1): each (tile, range) writes its fp32 partial
     // sums to partial[ks][row][col] (ldp columns, pstride floats per range) and
     // splitk_finish adds the ranges in order and applies the epilogue.
@@ -187,6 +192,17 @@ struct GemmLaunch {
 };
 
 enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2, EPI_RESID = 3, EPI_ROPE = 4 };
+
+// Key slots per sequence in the transposed value buffer (the longest sequence).
+constexpr int kVtSlots = 128;
+
+// Parameters of the rotary (q/k/v projection) epilogue, see GemmLaunch.
+struct RopeEpi {
+    const float2* cs;
+    int S, dh, n_rot;
+    __nv_bfloat16* vt;
+    int vt_rows;
+};
 
 // Attention sublayer of the full block (kernels e).
 struct AttnParams {
@@ -259,7 +275,8 @@ size_t grouped_gemm_smem_bytes();
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st);
 cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);
 // tm_qkv: the q/k/v rows [T][nqkv] in 128-row x 64-column boxes, 128-byte swizzle.
-cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, int head_dim, cudaStream_t st);
+cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, const CUtensorMap* tm_vt, int head_dim,
+                             cudaStream_t st);
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
 cudaError_t launch_watchdog_selftest(int* err, uint64_t limit_ns, cudaStream_t st);
 

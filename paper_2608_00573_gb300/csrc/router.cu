@@ -260,17 +260,21 @@ int router_pass_rows(int n_out) {
 }
 
 // Column ranges per launch: the smallest power of two dividing d/64 that gives
-// every SM at least one (tile, range, pass) unit.  More ranges only add
-// partial sums for the decision kernel to write and read back: on the
-// 8192-token layer with d = 2048 and 60 experts, 2 ranges took 27 us where 32
-// ranges (eight units per SM) took 50 us.
+// every SM at least one (tile, range, pass) unit, and at most kMaxSplit.  More
+// ranges only add partial sums for the decision kernel to write and read
+// back: on the 8192-token layer with d = 2048 and 60 experts, 2 ranges took
+// 27 us where 32 ranges (eight units per SM) took 50 us; and for a
+// decode-sized batch (one 128-token tile) the decision kernel's per-token
+// sums over 64 ranges cost more than the router saves with them.
+constexpr int kMaxSplit = 16;
+
 int router_ksplit(int T, int d, int n_out, int num_sms) {
     const int nslab = d / kKS;
     const int tiles = (T + kTok - 1) / kTok;
     const int ng = router_pass_rows(n_out);
     const long long units = (long long)tiles * ((n_out + ng - 1) / ng);
     int ks = 1;
-    while (ks < nslab && units * ks < num_sms && nslab % (ks * 2) == 0) ks *= 2;
+    while (ks < nslab && ks < kMaxSplit && units * ks < num_sms && nslab % (ks * 2) == 0) ks *= 2;
     return ks;
 }
 

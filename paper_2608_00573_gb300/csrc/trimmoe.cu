@@ -213,6 +213,10 @@ struct trimmoe {
     // attention sublayer of the full block
     int nqkv = 0;
     __nv_bfloat16 *qkv = nullptr, *attn_out = nullptr, *hm = nullptr;
+    // Value heads transposed per sequence [seq][Hkv * Dh][kVtSlots] (keys
+    // contiguous: the K-major operand of O = P V), zeroed at create.
+    __nv_bfloat16* vt = nullptr;
+    size_t vt_elems = 0;
     int* goff_attn = nullptr;
     float2* rope = nullptr;           // [attn_seq][head_dim/2] (cos, sin)
     float* sqbuf_x = nullptr;         // [rows_part] partial sums of squares of the layer input
@@ -666,6 +670,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
         ok = ok && h->dalloc(&h->qkv, T * h->nqkv) && h->dalloc(&h->attn_out, T * c.attn_heads * c.head_dim) &&
              h->dalloc(&h->hm, T * d) && h->dalloc(&h->goff_attn, 2) &&
              h->dalloc(&h->rope, (size_t)c.attn_seq * (c.head_dim / 2)) && h->dalloc(&h->sqbuf_x, h->rows_part);
+        h->vt_elems = ((T + c.attn_seq - 1) / c.attn_seq) * (size_t)c.attn_kv_heads * c.head_dim * kVtSlots;
+        ok = ok && h->dalloc(&h->vt, h->vt_elems);
     }
     if (!ok) return bail(TRIMMOE_ERR_OOM, "create: device allocation failed");
     cudaError_t ce = cudaSuccess;
@@ -700,6 +706,9 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
                 rt[(size_t)pos * half + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
             }
         up(h->rope, rt.data(), rt.size() * sizeof(float2));
+        // Key slots past a sequence's end are multiplied by zero probabilities:
+        // they must never hold NaN, so the buffer starts at zero.
+        if (ce == cudaSuccess) ce = cudaMemset(h->vt, 0, h->vt_elems * sizeof(__nv_bfloat16));
     }
     if (ce == cudaSuccess) ce = cudaStreamCreateWithFlags(&h->aux, cudaStreamNonBlocking);
     if (ce == cudaSuccess) ce = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
@@ -852,6 +861,8 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         qg.n_rot = (c.attn_heads + c.attn_kv_heads) * c.head_dim;
         qg.out = h->qkv;
         qg.ldo = h->nqkv;
+        qg.vt = h->vt;
+        qg.vt_rows = c.attn_kv_heads * c.head_dim;
         qg.err = h->dev_err;
         qg.tmB_pair = pair_gemm(T) ? &h->tmWqkvp[layer] : nullptr;
         e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(qg, h->num_sms, st); });
@@ -859,10 +870,12 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         // q/k/v rows of this call only: a sequence's 128-row box reads zeros past T
         // (never stale or uninitialised rows, which the masked products would
         // still multiply by zero).
-        CUtensorMap tm_qkv;
-        if (!make_tmap(&tm_qkv, h->qkv, h->nqkv, T, 128))
+        CUtensorMap tm_qkv, tm_vt;
+        const uint64_t vt_rows = (uint64_t)((T + c.attn_seq - 1) / c.attn_seq) * c.attn_kv_heads * c.head_dim;
+        if (!make_tmap(&tm_qkv, h->qkv, h->nqkv, T, 128) ||
+            !make_tmap(&tm_vt, h->vt, kVtSlots, vt_rows, (uint32_t)c.head_dim))
             return h->fail(TRIMMOE_ERR_CUDA, "attention: cuTensorMapEncodeTiled failed");
-        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, &tm_qkv, c.head_dim, st); });
+        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, &tm_qkv, &tm_vt, c.head_dim, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(e));
         GemmLaunch og = qg;
         og.rope = nullptr;
