@@ -95,6 +95,10 @@ __device__ __forceinline__ void multi_sum(const float* __restrict__ base, size_t
                                           int ustride, int nv, float (&out)[kMS]) {
 #pragma unroll
     for (int u = 0; u < kMS; ++u) out[u] = 0.f;
+    if (nv == 1) {
+        out[0] = sum_parts(base + off, stride, n);
+        return;
+    }
     for (int i = 0; i < n; ++i) {
         float v[kMS];
 #pragma unroll
@@ -107,7 +111,7 @@ __device__ __forceinline__ void multi_sum(const float* __restrict__ base, size_t
 struct WarpCounters {
     unsigned long long layer_tokens, exec_tokens, skipped, exited;
     unsigned long long le, ls, re, rs, hops, shared_phi;
-    double delay;
+    float delay;          // this warp's tokens (a handful): fp32 is enough for the statistic
     float max_ratio;
 };
 
@@ -463,7 +467,7 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
                     const float tr = remote ? p.tab.trans[s * M + msel[j]] : 0.f;
                     dl += tr + p.tab.comp[l * M + msel[j]];
                 }
-                wc.delay += (double)dl;
+                wc.delay += dl;
                 ++wc.exec_tokens;
             } else if (action == 1) {
                 Dnew = __fadd_rn(Dhat, Lambda);
@@ -492,7 +496,7 @@ __global__ void __launch_bounds__(kWarps * 32, 7) decide_kernel(const DecidePara
         atomicAdd(&blk_cnt[7], wc.rs);
         atomicAdd(&blk_cnt[8], wc.hops);
         atomicAdd(&blk_cnt[9], wc.shared_phi);
-        atomicAdd(&blk_delay, wc.delay);
+        atomicAdd(&blk_delay, (double)wc.delay);
         atomicMax(&blk_ratio, __float_as_uint(fmaxf(wc.max_ratio, 0.f)));
     }
     __syncthreads();
