@@ -112,7 +112,7 @@ struct AttnLayout {
 };
 
 struct __align__(8) AttnBars {
-    uint64_t ld, s, p, o;
+    uint64_t ldqk, ldv, s, p, o;
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -158,7 +158,8 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__
     const int n = min(p.S, p.T - t0);
 
     if (threadIdx.x == 0) {
-        mbar_init(smem_u32(&bars->ld), 1);
+        mbar_init(smem_u32(&bars->ldqk), 1);
+        mbar_init(smem_u32(&bars->ldv), 1);
         mbar_init(smem_u32(&bars->s), 1);
         mbar_init(smem_u32(&bars->p), 4);
         mbar_init(smem_u32(&bars->o), 1);
@@ -178,22 +179,24 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__
     if (warp == 0) {
         if (lane == 0) {
             // ------------------------------------------------------- loads
-            const uint32_t lb = smem_u32(&bars->ld);
-            mbar_arrive_expect_tx(lb, 2 * L::KB * L::BOX + 2 * DH * 128);
+            // Q and K first (S needs them), V^T behind them (only O needs it).
+            const uint32_t lb = smem_u32(&bars->ldqk), vb = smem_u32(&bars->ldv);
+            mbar_arrive_expect_tx(lb, 2 * L::KB * L::BOX);
             const int qcol = hq * DH, kcol = (p.Hq + g) * DH;
             for (int kb = 0; kb < L::KB; ++kb) {
                 tma_load_2d(sb + L::QP + kb * L::BOX, &tm, qcol + kb * 64, t0, lb);
                 tma_load_2d(sb + L::K + kb * L::BOX, &tm, kcol + kb * 64, t0, lb);
             }
+            mbar_arrive_expect_tx(vb, 2 * DH * 128);
             const int vrow = (b * p.Hkv + g) * DH;
-            for (int kb = 0; kb < 2; ++kb) tma_load_2d(sb + L::VT + kb * DH * 128, &tm_vt, kb * 64, vrow, lb);
+            for (int kb = 0; kb < 2; ++kb) tma_load_2d(sb + L::VT + kb * DH * 128, &tm_vt, kb * 64, vrow, vb);
         }
     } else if (warp == 1) {
         if (lane == 0) {
             // ------------------------------------------------------- MMAs
             constexpr uint32_t idS = idesc_bf16_f32(128, 128);
             constexpr uint32_t idO = idesc_bf16_f32(128, DH);
-            if (mbar_wait_bounded(smem_u32(&bars->ld), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN)) {
+            if (mbar_wait_bounded(smem_u32(&bars->ldqk), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN)) {
                 tc_fence_after();
 #pragma unroll
                 for (int kb = 0; kb < L::KB; ++kb)
@@ -202,7 +205,8 @@ attention_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__
                         tc_mma_bf16(tS, smem_desc_sw128(sb + L::QP + kb * L::BOX + kk * 32),
                                     smem_desc_sw128(sb + L::K + kb * L::BOX + kk * 32), idS, (kb | kk) ? 1u : 0u);
                 tc_commit(smem_u32(&bars->s));
-                if (mbar_wait_bounded(smem_u32(&bars->p), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN)) {
+                if (mbar_wait_bounded(smem_u32(&bars->p), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN) &&
+                    mbar_wait_bounded(smem_u32(&bars->ldv), 0, abort_flag, p.err, ERR_TIMEOUT_ATTN)) {
                     tc_fence_after();
 #pragma unroll
                     for (int kb = 0; kb < 2; ++kb)
