@@ -276,7 +276,7 @@ cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st)
 cudaError_t launch_attn_norm(const AttnParams& p, int num_sms, cudaStream_t st);
 // tm_qkv: the q/k/v rows [T][nqkv] in 128-row x 64-column boxes, 128-byte swizzle.
 cudaError_t launch_attention(const AttnParams& p, const CUtensorMap* tm_qkv, const CUtensorMap* tm_vt, int head_dim,
-                             cudaStream_t st);
+                             int num_sms, cudaStream_t st);
 cudaError_t launch_feedback(const FeedbackParams& p, cudaStream_t st);
 cudaError_t launch_watchdog_selftest(int* err, uint64_t limit_ns, cudaStream_t st);
 

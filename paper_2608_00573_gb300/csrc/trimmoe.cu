@@ -875,7 +875,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         if (!make_tmap(&tm_qkv, h->qkv, h->nqkv, T, 128) ||
             !make_tmap(&tm_vt, h->vt, kVtSlots, vt_rows, (uint32_t)c.head_dim))
             return h->fail(TRIMMOE_ERR_CUDA, "attention: cuTensorMapEncodeTiled failed");
-        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, &tm_qkv, &tm_vt, c.head_dim, st); });
+        e = h->timed(K_ATTN, st, [&] { return launch_attention(ap, &tm_qkv, &tm_vt, c.head_dim, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("attention: ") + cudaGetErrorString(e));
         GemmLaunch og = qg;
         og.rope = nullptr;
