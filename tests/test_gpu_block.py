@@ -40,12 +40,23 @@ BLOCKS = {
     # per group on average) run on CTA pairs, 256-row tiles with a ragged tail
     "gqa_pair_T4200": small_cfg(name="b5", N=2, d=512, E=4, k=2, F=256, T=4200, M=10, H=3, renorm_topk=1,
                                 attn_heads=8, attn_kv_heads=2, head_dim=64, attn_seq=128, seed=44),
+    # many (head, sequence) units per attention CTA: 1500 units of three query
+    # heads per key/value head, so groups straddle the CTAs' unit ranges and
+    # every Q slot and K/V buffer is reused; ragged last sequence
+    "gqa3_h64_s8_many_units": small_cfg(name="b6", N=2, d=512, E=8, k=2, F=256, T=1000, M=10, H=3,
+                                        renorm_topk=1, attn_heads=12, attn_kv_heads=4, head_dim=64, attn_seq=8,
+                                        seed=45),
+    # the same at head_dim 128: 978 units, ragged last sequence of 4 tokens
+    "gqa3_h128_s8_many_units": small_cfg(name="b7", N=2, d=512, E=8, k=2, F=256, T=1300, M=10, H=3,
+                                         renorm_topk=1, attn_heads=6, attn_kv_heads=2, head_dim=128, attn_seq=8,
+                                         seed=46),
 }
 
 
 # exit-head bias per configuration: the 64-class head's max-softmax confidence
 # needs a larger bias than the sigmoid head to reach p_J = 0.9
-EXIT_BIAS = {"gqa_h64_s128": 1.0, "mha_h128_s100_shared": 1.0, "relu_c64_s37_kc16": 5.0, "gqa_pair_T4200": 1.0}
+EXIT_BIAS = {"gqa_h64_s128": 1.0, "mha_h128_s100_shared": 1.0, "relu_c64_s37_kc16": 5.0, "gqa_pair_T4200": 1.0,
+             "gqa3_h64_s8_many_units": 1.0, "gqa3_h128_s8_many_units": 1.0}
 
 
 @pytest.mark.parametrize("name", list(BLOCKS))
