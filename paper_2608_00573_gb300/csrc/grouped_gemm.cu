@@ -911,8 +911,11 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
     const long long a_tile_bytes = (long long)BM * g.K * 2;
     if (g.transposed && g.tmB_pair && g.ksplit <= 1 && pair_t_clusters(num_sms) > 0) {
         if (g.epi_mode != EPI_STORE && g.epi_mode != EPI_RELU) return cudaErrorInvalidValue;
-        // Token-tile blocks of about 32 MB of activations, as for the pair kernel.
-        const int mblk2 = (int)std::max(1LL, (32LL << 20) / (2 * a_tile_bytes));
+        // Token-tile blocks of about 64 MB of activations: at K = 14336 eight
+        // token tiles, so a round of 76 tiles spans ~9.5 feature tiles x 8 token
+        // tiles, close to the square that streams the fewest operand slices
+        // (DRAM reads of the Mixtral-shaped down launch -9 % against 32 MB).
+        const int mblk2 = (int)std::max(1LL, (64LL << 20) / (2 * a_tile_bytes));
         const cudaError_t e = launch_pdl(
             grouped_gemm_pair_t_kernel, dim3(2 * pair_t_clusters(num_sms)), dim3(kThreads), kPairTSmemBytes, st,
             *g.tmA, *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
