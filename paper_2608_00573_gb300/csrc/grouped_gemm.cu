@@ -85,22 +85,38 @@ struct Tile {
 };
 
 // Per-group tile counts from the device-side group offsets (tile_rows rows per
-// row tile); one thread.
+// row tile); one warp: 32 groups' offsets loaded at once, tile counts
+// prefix-summed with shuffles (integer sums, the same table as a serial loop).
 template <class Tail>
 __device__ __forceinline__ void build_tile_table(Tail* tl, const int* goff, int first_group, int ngroups,
-                                                 int n_tiles_n, int tile_rows) {
-    int acc = 0;
-    for (int g = 0; g < ngroups; ++g) {
-        const int st = goff[first_group + g];
-        const int cnt = goff[first_group + g + 1] - st;
-        tl->gstart[g] = st;
-        tl->gcnt[g] = cnt;
-        tl->tile_start[g] = acc;
-        acc += ((cnt + tile_rows - 1) / tile_rows) * n_tiles_n;
+                                                 int n_tiles_n, int tile_rows, int lane) {
+    int carry = 0;
+    for (int g0 = 0; g0 < ngroups; g0 += 32) {
+        const int g = g0 + lane;
+        int st = 0, cnt = 0, nt = 0;
+        if (g < ngroups) {
+            st = goff[first_group + g];
+            cnt = goff[first_group + g + 1] - st;
+            nt = ((cnt + tile_rows - 1) / tile_rows) * n_tiles_n;
+        }
+        int incl = nt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (g < ngroups) {
+            tl->gstart[g] = st;
+            tl->gcnt[g] = cnt;
+            tl->tile_start[g] = carry + incl - nt;
+        }
+        carry += __shfl_sync(0xffffffffu, incl, 31);
     }
-    tl->tile_start[ngroups] = acc;
-    tl->total_tiles = acc;
-    tl->abort_flag = 0;
+    if (lane == 0) {
+        tl->tile_start[ngroups] = carry;
+        tl->total_tiles = carry;
+        tl->abort_flag = 0;
+    }
 }
 
 // Tile t -> (group, row tile, column tile).  Within a group the row tiles are
@@ -315,8 +331,6 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const __nv_bfloat16* __restrict__ res, int ldr, const RopeEpi rp,
                     int mblk, int ksplit, float* __restrict__ partial,
                     int ldp, size_t pstride) {
-    pdl_wait();      // results of the preceding kernel in the stream
-    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -328,16 +342,9 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
 
-    // Tile table from the device-side group offsets.
-    if (threadIdx.x == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, BM);
-    __syncthreads();
-    const int ntiles = tl->total_tiles;
-    const int total = ntiles * ksplit;    // unit u: tile u % ntiles, K range u / ntiles
-    if ((int)blockIdx.x >= total) return;
-    const int base0 = tl->gstart[0];
-    const int nkb = K / BK;
-    const int kbr = nkb / ksplit;         // k blocks per range
-
+    // Set-up that touches only this CTA's own resources (barriers, TMEM,
+    // descriptor prefetch) runs before the programmatic wait, under the
+    // preceding kernel's tail.
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(smem_u32(&tl->full[s]), 1);
@@ -356,6 +363,25 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = tl->tmem_base;
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
+
+    // Tile table from the device-side group offsets.
+    if (warp == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, BM, lane);
+    __syncthreads();
+    const int ntiles = tl->total_tiles;
+    const int total = ntiles * ksplit;    // unit u: tile u % ntiles, K range u / ntiles
+    if ((int)blockIdx.x >= total) {
+        if (warp == 0) {
+            __syncwarp();
+            tc_fence_after();
+            tmem_dealloc(tmem_base, TMEM_COLS);
+        }
+        return;
+    }
+    const int base0 = tl->gstart[0];
+    const int nkb = K / BK;
+    const int kbr = nkb / ksplit;         // k blocks per range
     volatile int* abort_flag = &tl->abort_flag;
 
     if (warp == 0) {
@@ -463,8 +489,6 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
                          int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                          __nv_bfloat16* __restrict__ out, int ldo, int* err,
                          const __nv_bfloat16* __restrict__ res, int ldr, const RopeEpi rp, int mblk) {
-    pdl_wait();      // results of the preceding kernel in the stream
-    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -479,13 +503,8 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
     const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
     const int sub = (int)rank * (BM);             // this CTA's rows / B rows within the tile
 
-    if (threadIdx.x == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, 2 * BM);
-    __syncthreads();
-    const int ntiles = tl->total_tiles;
-    if (cid >= ntiles) return;                    // both CTAs of the pair leave together
-    const int base0 = tl->gstart[0];
-    const int nkb = K / BK;
-
+    // Set-up that touches only the pair's own resources runs before the
+    // programmatic wait, under the preceding kernel's tail.
     if (threadIdx.x == 0) {
         for (int s = 0; s < P_STAGES; ++s) {
             mbar_init(smem_u32(&tl->full[s]), 1);
@@ -505,6 +524,23 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
     cluster_sync();                               // both CTAs' barriers are initialised
     tc_fence_after();
     const uint32_t tmem_base = tl->tmem_base;
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
+
+    if (warp == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, 2 * BM, lane);
+    __syncthreads();
+    const int ntiles = tl->total_tiles;
+    if (cid >= ntiles) {                          // both CTAs of the pair leave together
+        cluster_sync();
+        if (warp == 0) {
+            __syncwarp();
+            tc_fence_after();
+            tmem_dealloc_pair(tmem_base, TMEM_COLS);
+        }
+        return;
+    }
+    const int base0 = tl->gstart[0];
+    const int nkb = K / BK;
     volatile int* abort_flag = &tl->abort_flag;
 
     if (warp == 0) {
@@ -663,8 +699,6 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
                            int first_group, int ngroups, int x_rebase, int out_rebase, int K, int n_ft,
                            int w_rows_per_group, int epi_mode, __nv_bfloat16* __restrict__ out, int ldo,
                            int* err, int mblk, int staged) {
-    pdl_wait();      // results of the preceding kernel in the stream
-    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -679,13 +713,8 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
     const uint32_t rank = cluster_ctarank();      // 0: issues the MMAs, 1: peer
     const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
 
-    if (threadIdx.x == 0) build_tile_table(tl, goff, first_group, ngroups, n_ft, 2 * BM);
-    __syncthreads();
-    const int ntiles = tl->total_tiles;
-    if (cid >= ntiles) return;                    // both CTAs of the pair leave together
-    const int base0 = tl->gstart[0];
-    const int nkb = K / BK;
-
+    // Set-up that touches only the pair's own resources runs before the
+    // programmatic wait, under the preceding kernel's tail.
     if (threadIdx.x == 0) {
         for (int s = 0; s < P_STAGES; ++s) {
             mbar_init(smem_u32(&tl->full[s]), 1);
@@ -705,6 +734,23 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
     cluster_sync();                               // both CTAs' barriers are initialised
     tc_fence_after();
     const uint32_t tmem_base = tl->tmem_base;
+    pdl_wait();      // results of the preceding kernel in the stream
+    pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
+
+    if (warp == 0) build_tile_table(tl, goff, first_group, ngroups, n_ft, 2 * BM, lane);
+    __syncthreads();
+    const int ntiles = tl->total_tiles;
+    if (cid >= ntiles) {                          // both CTAs of the pair leave together
+        cluster_sync();
+        if (warp == 0) {
+            __syncwarp();
+            tc_fence_after();
+            tmem_dealloc_pair(tmem_base, TMEM_COLS);
+        }
+        return;
+    }
+    const int base0 = tl->gstart[0];
+    const int nkb = K / BK;
     volatile int* abort_flag = &tl->abort_flag;
 
     if (warp == 0) {
