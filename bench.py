@@ -593,7 +593,7 @@ def run_ours(args):
 
 # Revision tag of each timed GEMM launch kind; a stored ncu traffic figure is
 # used only when it was taken on that revision.
-KERNEL_REV = {"grouped_gemm_gate_up": "gemm-v9", "grouped_gemm_down": "gemm-v11"}
+KERNEL_REV = {"grouped_gemm_gate_up": "gemm-v10", "grouped_gemm_down": "gemm-v12"}
 
 
 def launch_ranks(args, argv):

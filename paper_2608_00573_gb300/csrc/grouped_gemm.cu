@@ -44,6 +44,8 @@
 // per tile, so a group's tail pads at most 15 tokens; described at the kernel.
 #include <algorithm>
 
+#include <climits>
+
 #include "internal.cuh"
 
 namespace tmoe {
@@ -61,12 +63,17 @@ constexpr int kThreads = 192;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int kMaxGroups = kMaxE + 1;
 
+constexpr int kTQ = 4;                            // tile queue depth (transposed pair kernel)
+
 template <int NST>
 struct __align__(8) SmemTail {
     uint64_t full[NST];
     uint64_t empty[NST];
     uint64_t tfull[2];
     uint64_t tempty[2];
+    uint64_t tq_full[kTQ];         // transposed pair kernel: tile index published (each CTA)
+    uint64_t tq_empty[kTQ];        // ... and taken by every role of both CTAs (even CTA)
+    int tq[kTQ];
     uint32_t tmem_base;
     int abort_flag;
     int total_tiles;
@@ -698,7 +705,7 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
                            const int* __restrict__ goff,
                            int first_group, int ngroups, int x_rebase, int out_rebase, int K, int n_ft,
                            int w_rows_per_group, int epi_mode, __nv_bfloat16* __restrict__ out, int ldo,
-                           int* err, int mblk, int staged) {
+                           int* err, int mblk, int staged, int* __restrict__ sched) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -724,6 +731,11 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
             mbar_init(smem_u32(&tl->tfull[b]), 1);
             mbar_init(smem_u32(&tl->tempty[b]), 8);
         }
+        for (int b = 0; b < kTQ; ++b) {
+            mbar_init(smem_u32(&tl->tq_full[b]), 1);
+            // takers: MMA issuer + 4 epilogue warps (even CTA), producer + 4 epilogue warps (odd CTA)
+            mbar_init(smem_u32(&tl->tq_empty[b]), 10);
+        }
         fence_barrier_init();
         prefetch_tmap(&tmX);
         prefetch_tmap(&tmW);
@@ -740,24 +752,59 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
     if (warp == 0) build_tile_table(tl, goff, first_group, ngroups, n_ft, 2 * BM, lane);
     __syncthreads();
     const int ntiles = tl->total_tiles;
-    if (cid >= ntiles) {                          // both CTAs of the pair leave together
-        cluster_sync();
-        if (warp == 0) {
-            __syncwarp();
-            tc_fence_after();
-            tmem_dealloc_pair(tmem_base, TMEM_COLS);
-        }
-        return;
-    }
     const int base0 = tl->gstart[0];
     const int nkb = K / BK;
     volatile int* abort_flag = &tl->abort_flag;
+
+    // Tile sequence of the pair.  Its first tile is cid; after that the even
+    // CTA's producer draws the next tile from the launch-wide counter (tiles
+    // in order, so the tiles in flight stay neighbours in the L2-blocked
+    // order, and a pair that drew short tiles takes more of them), one draw
+    // ahead so that the atomic's latency hides behind the current tile's
+    // loads, and publishes each tile to both CTAs through a queue of kTQ
+    // slots; every other role takes the same sequence from the queue.
+    // Without a counter every role walks the static order cid, cid + ncl, ...
+    // on its own.  A tile index >= ntiles ends the sequence.
+    auto draw = [&](int i) -> int {               // the pair's tile for step i >= 1
+        return sched ? ncl + atomicAdd(sched, 1) : cid + i * ncl;
+    };
+    auto publish = [&](int i, int t) -> int {
+        const int slot = i % kTQ;
+        if (i >= kTQ && !mbar_wait_bounded(smem_u32(&tl->tq_empty[slot]), ((i / kTQ) - 1) & 1, abort_flag, err,
+                                           ERR_TIMEOUT_PRODUCER))
+            return INT_MAX;
+        tl->tq[slot] = t;
+        st_shared_cluster_u32(mapa_shared(smem_u32(&tl->tq[slot]), 1), (uint32_t)t);
+        mbar_arrive(smem_u32(&tl->tq_full[slot]));
+        mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tq_full[slot]), 1));
+        return t;
+    };
+    auto take = [&](int i, int code) -> int {    // one thread per role
+        if (!sched) return cid + i * ncl;
+        const int slot = i % kTQ;
+        if (!mbar_wait_bounded(smem_u32(&tl->tq_full[slot]), (i / kTQ) & 1, abort_flag, err, code)) return INT_MAX;
+        const int t = *reinterpret_cast<volatile int*>(&tl->tq[slot]);
+        if (rank == 0) mbar_arrive(smem_u32(&tl->tq_empty[slot]));
+        else mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tq_empty[slot]), 0));
+        return t;
+    };
 
     if (warp == 0) {
         if (lane == 0) {
             // ---------------------------------------------------- producer (both CTAs)
             int it = 0;
-            for (int t = cid; t < ntiles && !*abort_flag; t += ncl) {
+            int t_next = cid;
+            for (int i = 0; !*abort_flag; ++i) {
+                int t;
+                if (!sched) {
+                    t = cid + i * ncl;
+                } else if (rank == 0) {
+                    t = publish(i, t_next);
+                    if (t < ntiles) t_next = draw(i + 1);
+                } else {
+                    t = take(i, ERR_TIMEOUT_PRODUCER);
+                }
+                if (t >= ntiles) break;
                 int g, mt, ft;
                 locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
                 const int half = ((tile_tokens(tl, g, mt) + 15) & ~15) >> 1;
@@ -781,7 +828,9 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
             // ---------------------------------------------------- MMA issuer (even CTA)
             int it = 0, tl_i = 0;
             bool ok = true;
-            for (int t = cid; t < ntiles && ok; t += ncl, ++tl_i) {
+            for (; ok; ++tl_i) {
+                const int t = take(tl_i, ERR_TIMEOUT_MMA);
+                if (t >= ntiles) break;
                 int g, mt, ft;
                 locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
                 const uint32_t idesc = idesc_bf16_f32(2 * BM, (tile_tokens(tl, g, mt) + 15) & ~15);
@@ -819,7 +868,13 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
         const int q = warp & 3;                   // TMEM lane quarter of this warp
         const int et = (warp - 2) * 32 + lane;    // epilogue thread 0..127
         int tl_i = 0, chunk = 0;
-        for (int t = cid; t < ntiles; t += ncl, ++tl_i) {
+        for (;; ++tl_i) {
+            int t = 0;
+            if (lane == 0) t = take(tl_i, ERR_TIMEOUT_EPI);
+            t = __shfl_sync(0xffffffffu, t, 0);
+            // The four warps leave together (a queue wait that gave up in one
+            // of them ends the others too): they meet at named barriers below.
+            if (sched ? !bar_and_named(kEpiBar, 128, t < ntiles) : t >= ntiles) break;
             int g, mt, ft;
             locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
             const int rows = tile_tokens(tl, g, mt);
@@ -966,7 +1021,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
             grouped_gemm_pair_t_kernel, dim3(2 * pair_t_clusters(num_sms)), dim3(kThreads), kPairTSmemBytes, st,
             *g.tmA, *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
             g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, mblk2,
-            g.K <= kStagedMaxK ? 1 : 0);
+            g.K <= kStagedMaxK ? 1 : 0, g.sched);
         if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }

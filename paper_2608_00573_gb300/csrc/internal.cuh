@@ -189,6 +189,10 @@ struct GemmLaunch {
     float* partial;
     int ldp;
     size_t pstride;
+    // Transposed pair kernel: launch-wide tile counter, zero when the launch
+    // starts (each launch of a forward has its own, zeroed at the forward's
+    // start).  Null: a static tile order.
+    int* sched;
 };
 
 enum : int { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RELU = 2, EPI_RESID = 3, EPI_ROPE = 4 };

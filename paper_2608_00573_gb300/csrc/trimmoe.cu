@@ -72,6 +72,14 @@ inline bool pair_gemm(long long rows_per_group) { return rows_per_group >= kPair
 // last round (Mixtral-shaped decode at 256 tokens: 15.2 -> 15.6 ms per step).
 constexpr int kTransposedMinRows = 256;
 
+// Transposed pair launches with at least this K draw their tiles from a
+// launch-wide counter (a pair that drew short tiles takes more of them); at
+// shorter K the per-tile hand-off costs more than the balance saves
+// (Switch-shaped forward 1.011 -> 1.034 ms, Mixtral-shaped 198.3 -> 196.5 ms).
+constexpr int kDynamicMinK = 4096;
+
+inline bool dynamic_tiles(int K) { return K >= kDynamicMinK; }
+
 enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
 
 // NVTX range names per kernel family, nested in "trimmoe.layer_step" (itself
@@ -198,6 +206,7 @@ struct trimmoe {
     DevCounters* ctr = nullptr;
     int* dev_err = nullptr;
     float* splitk = nullptr;          // [8][64][max(n13 F, d)] partial sums of split-K GEMMs
+    int* gemm_sched = nullptr;        // [N][2] tile counters of the transposed pair GEMM launches of a layer
     float* la_scratch = nullptr;      // per-token look-ahead scratch of the decision kernel (shared-table layers)
     // Side stream for the shared look-ahead tables: they depend only on the
     // tables and the budget, so they are computed while the router runs.
@@ -660,7 +669,8 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
               (!h->la_all || h->dalloc(&h->la_layers, (size_t)N));
     h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
     ok = ok && h->dalloc(&h->c_counts, h->n_counts) &&
-         h->dalloc(&h->splitk, (size_t)kSplitKMax * kSplitKRows * std::max<size_t>((size_t)h->n13 * c.F, (size_t)d));
+         h->dalloc(&h->splitk, (size_t)kSplitKMax * kSplitKRows * std::max<size_t>((size_t)h->n13 * c.F, (size_t)d)) &&
+         h->dalloc(&h->gemm_sched, (size_t)2 * N);
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
     if (ok && tab_floats > 0)
         ok = h->dalloc(&h->la_scratch, decide_la_scratch_floats(E, M, h->max_layer_cand, h->num_sms));
@@ -715,6 +725,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     if (ce == cudaSuccess) ce = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
     if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies);
     if (ce == cudaSuccess) ce = cudaMemset(h->dev_err, 0, sizeof(int));
+    if (ce == cudaSuccess) ce = cudaMemset(h->gemm_sched, 0, (size_t)2 * N * sizeof(int));
     if (ce == cudaSuccess) ce = cudaMemset(h->Xp, 0, (size_t)h->rows_xp * d * 2);
     if (ce != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, std::string("create: ") + cudaGetErrorString(ce));
 
@@ -1088,6 +1099,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     g1.out = h->act;
     g1.ldo = c.F;
     g1.err = h->dev_err;
+    g1.sched = dynamic_tiles(d) ? h->gemm_sched + 2 * layer : nullptr;
     // Few executed pairs (decode-sized batches): few tiles would leave most
     // CTAs idle, so the K range is split and a finish kernel adds the parts.
     const bool small = (long long)T * K <= kSplitKRows;
@@ -1107,6 +1119,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     g2.tmA = &h->tmAct;
     g2.tmB = &h->tmW2[layer];
     g2.transposed = transposed;
+    g2.sched = dynamic_tiles(c.F) ? h->gemm_sched + 2 * layer + 1 : nullptr;
     g2.tmB_pair = (g2.transposed || pair_routed) ? &h->tmW2p[layer] : nullptr;
     g2.K = c.F;
     g2.n_tiles_n = d / 256;
@@ -1203,6 +1216,9 @@ extern "C" trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T,
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     h->last_stream = st;
     if (T == 0) return TRIMMOE_OK;
+    if ((dynamic_tiles(h->cfg.d) || dynamic_tiles(h->cfg.F)) &&
+        cudaMemsetAsync(h->gemm_sched + 2 * layer, 0, 2 * sizeof(int), st) != cudaSuccess)
+        return h->fail(TRIMMOE_ERR_CUDA, "layer_step: tile counter reset failed");
     return layer_step_impl(h, layer, T, tok, out, st);
 }
 
@@ -1247,7 +1263,11 @@ static bool build_all_tables(trimmoe_handle h, int T, const trimmoe_tokens* tok,
 }
 
 static trimmoe_status forward_layers(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st) {
-    cudaError_t e;
+    // Tile counters of the layers' transposed pair GEMM launches start at zero.
+    cudaError_t e = cudaSuccess;
+    if (dynamic_tiles(h->cfg.d) || dynamic_tiles(h->cfg.F))
+        e = cudaMemsetAsync(h->gemm_sched, 0, (size_t)2 * h->cfg.N * sizeof(int), st);
+    if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("forward: ") + cudaGetErrorString(e));
     h->tabs_ready = build_all_tables(h, T, tok, st, &e);
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("look-ahead tables: ") + cudaGetErrorString(e));
     trimmoe_status s = TRIMMOE_OK;
@@ -1492,6 +1512,7 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
     h->drain_events();
     if (cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies) != cudaSuccess ||
         cudaMemset(h->dev_err, 0, sizeof(int)) != cudaSuccess ||
+        cudaMemset(h->gemm_sched, 0, (size_t)2 * h->cfg.N * sizeof(int)) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "reset: memset failed");
     for (double& m : h->ms) m = 0.0;

@@ -50,11 +50,15 @@ SMALL = {
                              M=10, seed=23),
     "e60_k4_h3": small_cfg(name="s4", N=4, d=256, E=60, k=4, F=128, F_sh=128, T=300, M=10, H=3,
                            zipf_s=1.0, seed=24),
+    # ~300 rows per expert and K = F = 4096: the down projection runs on the
+    # transposed pair kernel with tiles drawn from the launch-wide counter
+    "dyn_tiles_f4096": small_cfg(name="s5", N=3, d=512, E=4, k=2, F=4096, T=600, M=10, H=3,
+                                 zipf_s=0.5, seed=25),
 }
 
 
 KNOBS = {"switch_tiny": (None, None), "swiglu_shared_k4": (0.9, 1.0), "swiglu_k2_renorm_h2": (0.9, 1.0),
-         "relu_k1_c64": (0.9, 5.0), "e60_k4_h3": (0.6, 1.0)}
+         "relu_k1_c64": (0.9, 5.0), "e60_k4_h3": (0.6, 1.0), "dyn_tiles_f4096": (0.9, 1.0)}
 
 
 @pytest.mark.parametrize("name", list(SMALL))
