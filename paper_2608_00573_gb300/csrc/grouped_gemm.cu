@@ -482,6 +482,68 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     }
 }
 
+// Tile sequence of a CTA pair.  Its first tile is cid; after that the even
+// CTA's producer draws the next tile index from a launch-wide counter (tiles
+// in order, so the tiles in flight stay neighbours in the L2-blocked order,
+// and a pair whose tiles ran short takes more of them), one draw ahead so that
+// the atomic's latency hides behind the current tile's loads, and publishes
+// each index to both CTAs through a queue of kTQ slots (tq_full in each CTA,
+// tq_empty in the even CTA counting the ten roles that take every entry: the
+// odd CTA's producer, the MMA issuer, and both CTAs' four epilogue warps).
+// Without a counter every role walks the static order cid, cid + ncl, ... on
+// its own.  An index >= the tile count ends the sequence.
+template <class Tail>
+struct PairTiles {
+    Tail* tl;
+    int* sched;
+    int cid, ncl;
+    uint32_t rank;
+    volatile int* abort_flag;
+    int* err;
+
+    __device__ __forceinline__ int draw(int i) const {       // the pair's tile for step i >= 1
+        return sched ? ncl + atomicAdd(sched, 1) : cid + i * ncl;
+    }
+    // Even CTA's producer: publish tile t as step i (INT_MAX if a wait gave up).
+    __device__ __forceinline__ int publish(int i, int t) const {
+        const int slot = i % kTQ;
+        if (i >= kTQ && !mbar_wait_bounded(smem_u32(&tl->tq_empty[slot]), ((i / kTQ) - 1) & 1, abort_flag, err,
+                                           ERR_TIMEOUT_PRODUCER))
+            return INT_MAX;
+        tl->tq[slot] = t;
+        st_shared_cluster_u32(mapa_shared(smem_u32(&tl->tq[slot]), 1), (uint32_t)t);
+        mbar_arrive(smem_u32(&tl->tq_full[slot]));
+        mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tq_full[slot]), 1));
+        return t;
+    }
+    // Every other role (one thread each): the tile of step i.
+    __device__ __forceinline__ int take(int i, int code) const {
+        if (!sched) return cid + i * ncl;
+        const int slot = i % kTQ;
+        if (!mbar_wait_bounded(smem_u32(&tl->tq_full[slot]), (i / kTQ) & 1, abort_flag, err, code)) return INT_MAX;
+        const int t = *reinterpret_cast<volatile int*>(&tl->tq[slot]);
+        if (rank == 0) mbar_arrive(smem_u32(&tl->tq_empty[slot]));
+        else mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tq_empty[slot]), 0));
+        return t;
+    }
+    // Producer of either CTA: the tile of step i; t_next carries the even
+    // CTA's draw for the next step.
+    __device__ __forceinline__ int producer_step(int i, int ntiles, int& t_next) const {
+        if (!sched) return cid + i * ncl;
+        if (rank != 0) return take(i, ERR_TIMEOUT_PRODUCER);
+        const int t = publish(i, t_next);
+        if (t < ntiles) t_next = draw(i + 1);
+        return t;
+    }
+};
+
+__device__ __forceinline__ void init_tile_queue_bars(uint64_t* tq_full, uint64_t* tq_empty) {
+    for (int b = 0; b < kTQ; ++b) {
+        mbar_init(smem_u32(&tq_full[b]), 1);
+        mbar_init(smem_u32(&tq_empty[b]), 10);
+    }
+}
+
 // Pair variant: one cluster of two CTAs per row-pair tile of 256 rows x 256
 // columns.  The tile sequence is shared by both CTAs; CTA rank r takes rows
 // [r * 128, r * 128 + 128) of the tile and B rows (output columns)
@@ -495,7 +557,8 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
                          const int* __restrict__ goff, int first_group, int ngroups, int a_rebase,
                          int out_rebase, int K, int n_tiles_n, int b_rows_per_group, int epi_mode,
                          __nv_bfloat16* __restrict__ out, int ldo, int* err,
-                         const __nv_bfloat16* __restrict__ res, int ldr, const RopeEpi rp, int mblk) {
+                         const __nv_bfloat16* __restrict__ res, int ldr, const RopeEpi rp, int mblk,
+                         int* __restrict__ sched) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     const uint32_t pad = ((raw_addr + 1023u) & ~1023u) - raw_addr;
@@ -521,6 +584,7 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
             mbar_init(smem_u32(&tl->tfull[b]), 1);
             mbar_init(smem_u32(&tl->tempty[b]), 8);
         }
+        init_tile_queue_bars(tl->tq_full, tl->tq_empty);
         fence_barrier_init();
         prefetch_tmap(&tmA);
         prefetch_tmap(&tmB);
@@ -537,24 +601,19 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
     if (warp == 0) build_tile_table(tl, goff, first_group, ngroups, n_tiles_n, 2 * BM, lane);
     __syncthreads();
     const int ntiles = tl->total_tiles;
-    if (cid >= ntiles) {                          // both CTAs of the pair leave together
-        cluster_sync();
-        if (warp == 0) {
-            __syncwarp();
-            tc_fence_after();
-            tmem_dealloc_pair(tmem_base, TMEM_COLS);
-        }
-        return;
-    }
     const int base0 = tl->gstart[0];
     const int nkb = K / BK;
     volatile int* abort_flag = &tl->abort_flag;
+    const PairTiles<PairSmemTail> tiles{tl, sched, cid, ncl, rank, abort_flag, err};
 
     if (warp == 0) {
         if (lane == 0) {
             // ---------------------------------------------------- producer (both CTAs)
             int it = 0;
-            for (int t = cid; t < ntiles && !*abort_flag; t += ncl) {
+            int t_next = cid;
+            for (int i = 0; !*abort_flag; ++i) {
+                const int t = tiles.producer_step(i, ntiles, t_next);
+                if (t >= ntiles) break;
                 const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
                                          b_rows_per_group, mblk, 2 * BM, sub, sub);
                 for (int kb = 0; kb < nkb; ++kb, ++it) {
@@ -576,7 +635,8 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
             constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
             int it = 0, tl_i = 0;
             bool ok = true;
-            for (int t = cid; t < ntiles && ok; t += ncl, ++tl_i) {
+            for (; ok; ++tl_i) {
+                if (tiles.take(tl_i, ERR_TIMEOUT_MMA) >= ntiles) break;
                 const int buf = tl_i & 1;
                 const uint32_t aph = (tl_i >> 1) & 1;
                 if (!mbar_wait_bounded(smem_u32(&tl->tempty[buf]), aph ^ 1, abort_flag, err,
@@ -611,7 +671,11 @@ grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_c
         const int q = warp & 3;
         const int row = q * 32 + lane;
         int tl_i = 0;
-        for (int t = cid; t < ntiles; t += ncl, ++tl_i) {
+        for (;; ++tl_i) {
+            int t = 0;
+            if (lane == 0) t = tiles.take(tl_i, ERR_TIMEOUT_EPI);
+            t = __shfl_sync(0xffffffffu, t, 0);
+            if (t >= ntiles) break;
             const Tile ti = map_tile(tl, t, ngroups, n_tiles_n, base0, a_rebase, out_rebase,
                                      b_rows_per_group, mblk, 2 * BM, sub, sub);
             const int buf = tl_i & 1;
@@ -731,11 +795,7 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
             mbar_init(smem_u32(&tl->tfull[b]), 1);
             mbar_init(smem_u32(&tl->tempty[b]), 8);
         }
-        for (int b = 0; b < kTQ; ++b) {
-            mbar_init(smem_u32(&tl->tq_full[b]), 1);
-            // takers: MMA issuer + 4 epilogue warps (even CTA), producer + 4 epilogue warps (odd CTA)
-            mbar_init(smem_u32(&tl->tq_empty[b]), 10);
-        }
+        init_tile_queue_bars(tl->tq_full, tl->tq_empty);
         fence_barrier_init();
         prefetch_tmap(&tmX);
         prefetch_tmap(&tmW);
@@ -756,38 +816,7 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
     const int nkb = K / BK;
     volatile int* abort_flag = &tl->abort_flag;
 
-    // Tile sequence of the pair.  Its first tile is cid; after that the even
-    // CTA's producer draws the next tile from the launch-wide counter (tiles
-    // in order, so the tiles in flight stay neighbours in the L2-blocked
-    // order, and a pair that drew short tiles takes more of them), one draw
-    // ahead so that the atomic's latency hides behind the current tile's
-    // loads, and publishes each tile to both CTAs through a queue of kTQ
-    // slots; every other role takes the same sequence from the queue.
-    // Without a counter every role walks the static order cid, cid + ncl, ...
-    // on its own.  A tile index >= ntiles ends the sequence.
-    auto draw = [&](int i) -> int {               // the pair's tile for step i >= 1
-        return sched ? ncl + atomicAdd(sched, 1) : cid + i * ncl;
-    };
-    auto publish = [&](int i, int t) -> int {
-        const int slot = i % kTQ;
-        if (i >= kTQ && !mbar_wait_bounded(smem_u32(&tl->tq_empty[slot]), ((i / kTQ) - 1) & 1, abort_flag, err,
-                                           ERR_TIMEOUT_PRODUCER))
-            return INT_MAX;
-        tl->tq[slot] = t;
-        st_shared_cluster_u32(mapa_shared(smem_u32(&tl->tq[slot]), 1), (uint32_t)t);
-        mbar_arrive(smem_u32(&tl->tq_full[slot]));
-        mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tq_full[slot]), 1));
-        return t;
-    };
-    auto take = [&](int i, int code) -> int {    // one thread per role
-        if (!sched) return cid + i * ncl;
-        const int slot = i % kTQ;
-        if (!mbar_wait_bounded(smem_u32(&tl->tq_full[slot]), (i / kTQ) & 1, abort_flag, err, code)) return INT_MAX;
-        const int t = *reinterpret_cast<volatile int*>(&tl->tq[slot]);
-        if (rank == 0) mbar_arrive(smem_u32(&tl->tq_empty[slot]));
-        else mbar_arrive_cluster(mapa_shared(smem_u32(&tl->tq_empty[slot]), 0));
-        return t;
-    };
+    const PairTiles<PairSmemTail> tiles{tl, sched, cid, ncl, rank, abort_flag, err};
 
     if (warp == 0) {
         if (lane == 0) {
@@ -795,15 +824,7 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
             int it = 0;
             int t_next = cid;
             for (int i = 0; !*abort_flag; ++i) {
-                int t;
-                if (!sched) {
-                    t = cid + i * ncl;
-                } else if (rank == 0) {
-                    t = publish(i, t_next);
-                    if (t < ntiles) t_next = draw(i + 1);
-                } else {
-                    t = take(i, ERR_TIMEOUT_PRODUCER);
-                }
+                const int t = tiles.producer_step(i, ntiles, t_next);
                 if (t >= ntiles) break;
                 int g, mt, ft;
                 locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
@@ -829,7 +850,7 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
             int it = 0, tl_i = 0;
             bool ok = true;
             for (; ok; ++tl_i) {
-                const int t = take(tl_i, ERR_TIMEOUT_MMA);
+                const int t = tiles.take(tl_i, ERR_TIMEOUT_MMA);
                 if (t >= ntiles) break;
                 int g, mt, ft;
                 locate_tile(tl, t, ngroups, n_ft, mblk, 2 * BM, g, mt, ft);
@@ -870,7 +891,7 @@ grouped_gemm_pair_t_kernel(const __grid_constant__ CUtensorMap tmX, const __grid
         int tl_i = 0, chunk = 0;
         for (;; ++tl_i) {
             int t = 0;
-            if (lane == 0) t = take(tl_i, ERR_TIMEOUT_EPI);
+            if (lane == 0) t = tiles.take(tl_i, ERR_TIMEOUT_EPI);
             t = __shfl_sync(0xffffffffu, t, 0);
             // The four warps leave together (a queue wait that gave up in one
             // of them ends the others too): they meet at named barriers below.
@@ -1032,7 +1053,7 @@ cudaError_t launch_grouped_gemm(const GemmLaunch& g, int num_sms, cudaStream_t s
         const cudaError_t e = launch_pdl(
             grouped_gemm_pair_kernel, dim3(2 * pair_clusters(num_sms)), dim3(kThreads), kPairSmemBytes, st, *g.tmA,
             *g.tmB_pair, g.goff, g.first_group, g.ngroups, g.a_rebase, g.out_rebase, g.K, g.n_tiles_n,
-            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, rp, mblk2);
+            g.b_rows_per_group, g.epi_mode, g.out, g.ldo, g.err, g.res, g.ldr, rp, mblk2, g.sched);
         if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }

@@ -72,13 +72,17 @@ inline bool pair_gemm(long long rows_per_group) { return rows_per_group >= kPair
 // last round (Mixtral-shaped decode at 256 tokens: 15.2 -> 15.6 ms per step).
 constexpr int kTransposedMinRows = 256;
 
-// Transposed pair launches with at least this K draw their tiles from a
-// launch-wide counter (a pair that drew short tiles takes more of them); at
-// shorter K the per-tile hand-off costs more than the balance saves
-// (Switch-shaped forward 1.011 -> 1.034 ms, Mixtral-shaped 198.3 -> 196.5 ms).
+// CTA-pair launches with at least this K draw their tiles from a launch-wide
+// counter (a pair whose tiles ran short takes more of them); at shorter K the
+// per-tile hand-off costs more than the balance saves (transposed launches:
+// Switch-shaped forward 1.011 -> 1.034 ms, Mixtral-shaped 198.3 -> 196.5 ms).
 constexpr int kDynamicMinK = 4096;
 
 inline bool dynamic_tiles(int K) { return K >= kDynamicMinK; }
+
+// Tile counters per layer, one per CTA-pair launch: routed up, routed down,
+// shared up, shared down, q/k/v projection, output projection.
+enum SchedSlot { SCHED_UP = 0, SCHED_DOWN, SCHED_SH_UP, SCHED_SH_DOWN, SCHED_QKV, SCHED_O, SCHED_SLOTS };
 
 enum Kind { K_DECIDE = 0, K_COMPACT, K_GATHER, K_GEMM_UP, K_GEMM_DOWN, K_COMBINE, K_ROUTER, K_ATTN, K_ATTN_GEMM, K_NUM };
 
@@ -206,7 +210,12 @@ struct trimmoe {
     DevCounters* ctr = nullptr;
     int* dev_err = nullptr;
     float* splitk = nullptr;          // [8][64][max(n13 F, d)] partial sums of split-K GEMMs
-    int* gemm_sched = nullptr;        // [N][2] tile counters of the transposed pair GEMM launches of a layer
+    int* gemm_sched = nullptr;        // [N][SCHED_SLOTS] tile counters of a layer's CTA-pair GEMM launches
+    bool sched_any = false;           // some launch draws its tiles from a counter
+    // Counter of a layer's launch of depth K, or null (static tile order).
+    int* sched_for(int layer, int slot, int K) const {
+        return dynamic_tiles(K) ? gemm_sched + (size_t)layer * SCHED_SLOTS + slot : nullptr;
+    }
     float* la_scratch = nullptr;      // per-token look-ahead scratch of the decision kernel (shared-table layers)
     // Side stream for the shared look-ahead tables: they depend only on the
     // tables and the budget, so they are computed while the router runs.
@@ -670,7 +679,7 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     h->n_counts = (size_t)std::max(N - 1, 1) * E * E + N + (size_t)N * M + 2 * (size_t)N * E;
     ok = ok && h->dalloc(&h->c_counts, h->n_counts) &&
          h->dalloc(&h->splitk, (size_t)kSplitKMax * kSplitKRows * std::max<size_t>((size_t)h->n13 * c.F, (size_t)d)) &&
-         h->dalloc(&h->gemm_sched, (size_t)2 * N);
+         h->dalloc(&h->gemm_sched, (size_t)SCHED_SLOTS * N);
     if (ok && has_sh) ok = h->dalloc(&h->act_sh, T * c.F_sh) && h->dalloc(&h->Ysh, T * d);
     if (ok && tab_floats > 0)
         ok = h->dalloc(&h->la_scratch, decide_la_scratch_floats(E, M, h->max_layer_cand, h->num_sms));
@@ -725,7 +734,9 @@ extern "C" trimmoe_status trimmoe_create(const trimmoe_config* cfg, const trimmo
     if (ce == cudaSuccess) ce = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
     if (ce == cudaSuccess) ce = cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies);
     if (ce == cudaSuccess) ce = cudaMemset(h->dev_err, 0, sizeof(int));
-    if (ce == cudaSuccess) ce = cudaMemset(h->gemm_sched, 0, (size_t)2 * N * sizeof(int));
+    if (ce == cudaSuccess) ce = cudaMemset(h->gemm_sched, 0, (size_t)SCHED_SLOTS * N * sizeof(int));
+    h->sched_any = dynamic_tiles(d) || dynamic_tiles(c.F) || (has_sh && dynamic_tiles(c.F_sh)) ||
+                   (c.attn_heads > 0 && dynamic_tiles(c.attn_heads * c.head_dim));
     if (ce == cudaSuccess) ce = cudaMemset(h->Xp, 0, (size_t)h->rows_xp * d * 2);
     if (ce != cudaSuccess) return bail(TRIMMOE_ERR_CUDA, std::string("create: ") + cudaGetErrorString(ce));
 
@@ -876,6 +887,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         qg.vt_rows = c.attn_kv_heads * c.head_dim;
         qg.err = h->dev_err;
         qg.tmB_pair = pair_gemm(T) ? &h->tmWqkvp[layer] : nullptr;
+        qg.sched = h->sched_for(layer, SCHED_QKV, d);
         e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(qg, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("qkv gemm: ") + cudaGetErrorString(e));
         // q/k/v rows of this call only: a sequence's 128-row box reads zeros past T
@@ -901,6 +913,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         og.ldo = d;
         og.res = hid_in;
         og.ldr = d;
+        og.sched = h->sched_for(layer, SCHED_O, hd);
         e = h->timed(K_ATTN_GEMM, st, [&] { return launch_grouped_gemm(og, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("output projection: ") + cudaGetErrorString(e));
         h->launches += 4;
@@ -1099,7 +1112,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     g1.out = h->act;
     g1.ldo = c.F;
     g1.err = h->dev_err;
-    g1.sched = dynamic_tiles(d) ? h->gemm_sched + 2 * layer : nullptr;
+    g1.sched = h->sched_for(layer, SCHED_UP, d);
     // Few executed pairs (decode-sized batches): few tiles would leave most
     // CTAs idle, so the K range is split and a finish kernel adds the parts.
     const bool small = (long long)T * K <= kSplitKRows;
@@ -1119,7 +1132,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
     g2.tmA = &h->tmAct;
     g2.tmB = &h->tmW2[layer];
     g2.transposed = transposed;
-    g2.sched = dynamic_tiles(c.F) ? h->gemm_sched + 2 * layer + 1 : nullptr;
+    g2.sched = h->sched_for(layer, SCHED_DOWN, c.F);
     g2.tmB_pair = (g2.transposed || pair_routed) ? &h->tmW2p[layer] : nullptr;
     g2.K = c.F;
     g2.n_tiles_n = d / 256;
@@ -1154,6 +1167,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         s1.epi_mode = EPI_SWIGLU;
         s1.out = h->act_sh;
         s1.ldo = c.F_sh;
+        s1.sched = h->sched_for(layer, SCHED_SH_UP, d);
         e = h->timed(K_GEMM_UP, st, [&] { return launch_grouped_gemm(s1, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("shared gemm up: ") + cudaGetErrorString(e));
         GemmLaunch s2 = s1;
@@ -1167,6 +1181,7 @@ static trimmoe_status layer_step_impl(trimmoe_handle h, int layer, int T, trimmo
         s2.epi_mode = EPI_STORE;
         s2.out = h->Ysh;
         s2.ldo = d;
+        s2.sched = h->sched_for(layer, SCHED_SH_DOWN, c.F_sh);
         e = h->timed(K_GEMM_DOWN, st, [&] { return launch_grouped_gemm(s2, h->num_sms, st); });
         if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("shared gemm down: ") + cudaGetErrorString(e));
         h->n_gemm_up++;
@@ -1216,8 +1231,8 @@ extern "C" trimmoe_status trimmoe_layer_step(trimmoe_handle h, int layer, int T,
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     h->last_stream = st;
     if (T == 0) return TRIMMOE_OK;
-    if ((dynamic_tiles(h->cfg.d) || dynamic_tiles(h->cfg.F)) &&
-        cudaMemsetAsync(h->gemm_sched + 2 * layer, 0, 2 * sizeof(int), st) != cudaSuccess)
+    if (h->sched_any &&
+        cudaMemsetAsync(h->gemm_sched + (size_t)layer * SCHED_SLOTS, 0, SCHED_SLOTS * sizeof(int), st) != cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "layer_step: tile counter reset failed");
     return layer_step_impl(h, layer, T, tok, out, st);
 }
@@ -1265,8 +1280,7 @@ static bool build_all_tables(trimmoe_handle h, int T, const trimmoe_tokens* tok,
 static trimmoe_status forward_layers(trimmoe_handle h, int T, trimmoe_tokens* tok, cudaStream_t st) {
     // Tile counters of the layers' transposed pair GEMM launches start at zero.
     cudaError_t e = cudaSuccess;
-    if (dynamic_tiles(h->cfg.d) || dynamic_tiles(h->cfg.F))
-        e = cudaMemsetAsync(h->gemm_sched, 0, (size_t)2 * h->cfg.N * sizeof(int), st);
+    if (h->sched_any) e = cudaMemsetAsync(h->gemm_sched, 0, (size_t)SCHED_SLOTS * h->cfg.N * sizeof(int), st);
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("forward: ") + cudaGetErrorString(e));
     h->tabs_ready = build_all_tables(h, T, tok, st, &e);
     if (e != cudaSuccess) return h->fail(TRIMMOE_ERR_CUDA, std::string("look-ahead tables: ") + cudaGetErrorString(e));
@@ -1512,7 +1526,7 @@ extern "C" trimmoe_status trimmoe_reset_stats(trimmoe_handle h) {
     h->drain_events();
     if (cudaMemset(h->ctr, 0, sizeof(DevCounters) * kCtrCopies) != cudaSuccess ||
         cudaMemset(h->dev_err, 0, sizeof(int)) != cudaSuccess ||
-        cudaMemset(h->gemm_sched, 0, (size_t)2 * h->cfg.N * sizeof(int)) != cudaSuccess ||
+        cudaMemset(h->gemm_sched, 0, (size_t)SCHED_SLOTS * h->cfg.N * sizeof(int)) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess)
         return h->fail(TRIMMOE_ERR_CUDA, "reset: memset failed");
     for (double& m : h->ms) m = 0.0;

@@ -54,11 +54,16 @@ SMALL = {
     # transposed pair kernel with tiles drawn from the launch-wide counter
     "dyn_tiles_f4096": small_cfg(name="s5", N=3, d=512, E=4, k=2, F=4096, T=600, M=10, H=3,
                                  zipf_s=0.5, seed=25),
+    # 2100 live tokens through a shared expert of F_sh = 4096: its down
+    # projection runs on the CTA-pair kernel with tiles drawn from the counter
+    "shared_f4096_pair_dyn": small_cfg(name="s6", N=3, d=512, E=4, k=2, F=256, F_sh=4096, T=2100, M=10,
+                                       H=3, zipf_s=0.5, seed=26),
 }
 
 
 KNOBS = {"switch_tiny": (None, None), "swiglu_shared_k4": (0.9, 1.0), "swiglu_k2_renorm_h2": (0.9, 1.0),
-         "relu_k1_c64": (0.9, 5.0), "e60_k4_h3": (0.6, 1.0), "dyn_tiles_f4096": (0.9, 1.0)}
+         "relu_k1_c64": (0.9, 5.0), "e60_k4_h3": (0.6, 1.0), "dyn_tiles_f4096": (0.9, 1.0),
+         "shared_f4096_pair_dyn": (0.9, 1.0)}
 
 
 @pytest.mark.parametrize("name", list(SMALL))
