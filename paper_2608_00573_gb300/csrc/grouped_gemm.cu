@@ -42,6 +42,11 @@
 // Transposed pair variant (routed down projections, ReLU up projections): the
 // weights on the MMA's M side and the tokens on its N side, N rounded up to 16
 // per tile, so a group's tail pads at most 15 tokens; described at the kernel.
+//
+// Both pair variants take their tiles in the order above; for long K they
+// draw them from a launch-wide counter (PairTiles) rather than each cluster
+// walking a fixed stride, so clusters that finish early take more tiles and
+// the tiles in flight stay neighbours in that order.
 #include <algorithm>
 
 #include <climits>
