@@ -21,16 +21,24 @@ namespace {
 
 // KT: slots held in registers (k <= KT).  All loads of one step (the residual
 // base, every slot's Y row and the shared expert's row, kU chunks of 16 bytes
-// per lane each) are issued before the first one is used.
+// per lane each) are issued before the first one is used.  A warp takes one
+// segment of nseg of a token's row: the whole row (nseg = 1) for large
+// batches, one step of it per warp for decode-sized ones, so that the row's
+// loads are in flight at once rather than one step after another.
 template <int KT>
-__global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
+__global__ void __launch_bounds__(256) combine_kernel(const CombineParams p, int nseg) {
     pdl_wait();      // results of the preceding kernel in the stream
     pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     constexpr int kU = KT <= 2 ? 4 : 2;
     const int lane = threadIdx.x & 31;
     const int nchunk = p.d >> 3;
-    for (int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; t < p.T;
-         t += (gridDim.x * blockDim.x) >> 5) {
+    const int seg_chunks = (nchunk + nseg - 1) / nseg;
+    const long long nunits = (long long)p.T * nseg;
+    for (long long unit = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; unit < nunits;
+         unit += (gridDim.x * blockDim.x) >> 5) {
+        const int t = (int)(unit / nseg);
+        const int cbeg = (int)(unit - (long long)t * nseg) * seg_chunks;
+        const int cend = min(nchunk, cbeg + seg_chunks);
         const int a = p.action[t];
         if (a > 1 || (a == 1 && !p.has_shared && p.h_src == p.h)) continue;
         float w[KT];
@@ -52,29 +60,29 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
         const uint4* srow = reinterpret_cast<const uint4*>(p.Ysh + (size_t)(psh >= 0 ? psh : 0) * p.d);
         uint4* hrow = reinterpret_cast<uint4*>(p.h + (size_t)t * p.d);
         const uint4* brow = reinterpret_cast<const uint4*>(p.h_src + (size_t)t * p.d);
-        for (int c0 = lane; c0 < nchunk; c0 += 32 * kU) {
+        for (int c0 = cbeg + lane; c0 < cend; c0 += 32 * kU) {
             uint4 hv[kU], yv[KT][kU], sv[kU];
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const int c = c0 + 32 * u;
-                hv[u] = c < nchunk ? brow[c] : make_uint4(0u, 0u, 0u, 0u);
+                hv[u] = c < cend ? brow[c] : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
             for (int j = 0; j < KT; ++j)
 #pragma unroll
                 for (int u = 0; u < kU; ++u) {
                     const int c = c0 + 32 * u;
-                    yv[j][u] = (j < nj && c < nchunk) ? __ldg(yrow[j] + c) : make_uint4(0u, 0u, 0u, 0u);
+                    yv[j][u] = (j < nj && c < cend) ? __ldg(yrow[j] + c) : make_uint4(0u, 0u, 0u, 0u);
                 }
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const int c = c0 + 32 * u;
-                sv[u] = (psh >= 0 && c < nchunk) ? __ldg(srow + c) : make_uint4(0u, 0u, 0u, 0u);
+                sv[u] = (psh >= 0 && c < cend) ? __ldg(srow + c) : make_uint4(0u, 0u, 0u, 0u);
             }
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
                 const int c = c0 + 32 * u;
-                if (c >= nchunk) continue;
+                if (c >= cend) continue;
                 const uint32_t hw[4] = {hv[u].x, hv[u].y, hv[u].z, hv[u].w};
                 uint32_t ow[4];
 #pragma unroll
@@ -101,6 +109,14 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineParams p) {
     }
 }
 
+// Row segments per token: one per warp step of kU chunks for decode-sized
+// batches (at most 256 tokens), the whole row otherwise.
+int combine_segments(int T, int d, int kU) {
+    if (T > 256) return 1;
+    const int steps = ((d >> 3) + 32 * kU - 1) / (32 * kU);
+    return steps > 1 ? steps : 1;
+}
+
 template <int KT>
 int combine_grid(int T, int num_sms) {
     static PerDevice occ;
@@ -120,10 +136,17 @@ int combine_grid(int T, int num_sms) {
 cudaError_t launch_combine(const CombineParams& p, int num_sms, cudaStream_t st) {
     if (p.T <= 0) return cudaSuccess;
     cudaError_t e;
-    if (p.k <= 1) e = launch_pdl(combine_kernel<1>, dim3(combine_grid<1>(p.T, num_sms)), dim3(256), 0, st, p);
-    else if (p.k <= 2) e = launch_pdl(combine_kernel<2>, dim3(combine_grid<2>(p.T, num_sms)), dim3(256), 0, st, p);
-    else if (p.k <= 4) e = launch_pdl(combine_kernel<4>, dim3(combine_grid<4>(p.T, num_sms)), dim3(256), 0, st, p);
-    else e = launch_pdl(combine_kernel<kMaxK>, dim3(combine_grid<kMaxK>(p.T, num_sms)), dim3(256), 0, st, p);
+    const int kU = p.k <= 2 ? 4 : 2;                  // combine_kernel's chunks per lane and step
+    const int nseg = combine_segments(p.T, p.d, kU);
+    const int units = p.T * nseg;
+    if (p.k <= 1)
+        e = launch_pdl(combine_kernel<1>, dim3(combine_grid<1>(units, num_sms)), dim3(256), 0, st, p, nseg);
+    else if (p.k <= 2)
+        e = launch_pdl(combine_kernel<2>, dim3(combine_grid<2>(units, num_sms)), dim3(256), 0, st, p, nseg);
+    else if (p.k <= 4)
+        e = launch_pdl(combine_kernel<4>, dim3(combine_grid<4>(units, num_sms)), dim3(256), 0, st, p, nseg);
+    else
+        e = launch_pdl(combine_kernel<kMaxK>, dim3(combine_grid<kMaxK>(units, num_sms)), dim3(256), 0, st, p, nseg);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

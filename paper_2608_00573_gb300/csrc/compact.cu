@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
                                                      int d, const __nv_bfloat16* __restrict__ h,
                                                      const float* __restrict__ rnorm,
                                                      const __nv_bfloat16* __restrict__ gamma,
-                                                     __nv_bfloat16* __restrict__ Xp) {
+                                                     __nv_bfloat16* __restrict__ Xp, int nseg) {
     pdl_wait();      // results of the preceding kernel in the stream
     pdl_trigger();   // single-wave grid: let the next kernel be scheduled now
     extern __shared__ uint4 sg[];      // gamma, d / 8 chunks
@@ -215,22 +215,29 @@ __global__ void __launch_bounds__(256) gather_kernel(const int32_t* __restrict__
         for (int c = threadIdx.x; c < nchunk; c += blockDim.x) sg[c] = __ldg(gv4 + c);
         __syncthreads();
     }
-    for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < nrows;
-         r += (gridDim.x * blockDim.x) >> 5) {
+    // A warp copies one of nseg segments of a row (nseg > 1 for decode-sized
+    // batches, so that a row's loads are in flight together).
+    const int seg_chunks = (nchunk + nseg - 1) / nseg;
+    const long long nunits = (long long)nrows * nseg;
+    for (long long unit = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; unit < nunits;
+         unit += (gridDim.x * blockDim.x) >> 5) {
+        const int r = (int)(unit / nseg);
+        const int cbeg = (int)(unit - (long long)r * nseg) * seg_chunks;
+        const int cend = min(nchunk, cbeg + seg_chunks);
         const int code = perm[r];
         const int t = r < routed ? code / k : code;
         const uint4* __restrict__ src = reinterpret_cast<const uint4*>(h + (size_t)t * d);
         uint4* __restrict__ dst = reinterpret_cast<uint4*>(Xp + (size_t)r * d);
         const float rn = gamma ? rnorm[t] : 1.f;
-        for (int c0 = lane; c0 < nchunk; c0 += 32 * kGU) {
+        for (int c0 = cbeg + lane; c0 < cend; c0 += 32 * kGU) {
             uint4 hv[kGU];
 #pragma unroll
             for (int u = 0; u < kGU; ++u)
-                if (c0 + 32 * u < nchunk) hv[u] = src[c0 + 32 * u];
+                if (c0 + 32 * u < cend) hv[u] = src[c0 + 32 * u];
 #pragma unroll
             for (int u = 0; u < kGU; ++u) {
                 const int c = c0 + 32 * u;
-                if (c >= nchunk) continue;
+                if (c >= cend) continue;
                 if (!gamma) {
                     dst[c] = hv[u];
                     continue;
@@ -276,10 +283,13 @@ cudaError_t launch_gather(const int32_t* perm, const int32_t* goff, int E, int k
             n = 1;
         return n;
     });
-    int blocks = (max_rows + 7) / 8;
-    blocks = blocks < num_sms * per_sm ? blocks : num_sms * per_sm;
+    // Decode-sized batches: one row segment (a step of kGU chunks per lane) per warp.
+    const int steps = ((d >> 3) + 32 * kGU - 1) / (32 * kGU);
+    const int nseg = max_rows <= 512 && steps > 1 ? steps : 1;
+    long long want = ((long long)max_rows * nseg + 7) / 8;
+    const int blocks = (int)(want < (long long)num_sms * per_sm ? want : (long long)num_sms * per_sm);
     const cudaError_t e = launch_pdl(gather_kernel, dim3(blocks), dim3(256), smem, st, perm, goff, E, k, d, h, rnorm,
-                                     gamma, Xp);
+                                     gamma, Xp, nseg);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
