@@ -68,7 +68,7 @@ constexpr int kThreads = 192;
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int kMaxGroups = kMaxE + 1;
 
-constexpr int kTQ = 4;                            // tile queue depth (transposed pair kernel)
+constexpr int kTQ = 4;                            // tile queue depth (CTA-pair kernels)
 
 template <int NST>
 struct __align__(8) SmemTail {
@@ -76,7 +76,7 @@ struct __align__(8) SmemTail {
     uint64_t empty[NST];
     uint64_t tfull[2];
     uint64_t tempty[2];
-    uint64_t tq_full[kTQ];         // transposed pair kernel: tile index published (each CTA)
+    uint64_t tq_full[kTQ];         // CTA-pair kernels: tile index published (each CTA)
     uint64_t tq_empty[kTQ];        // ... and taken by every role of both CTAs (even CTA)
     int tq[kTQ];
     uint32_t tmem_base;
