@@ -9,7 +9,6 @@ MoE step alone (teacher forcing inside the layer).
 import numpy as np
 import pytest
 
-from oracle import oracle as O
 from paper_2608_00573_gb300 import binding as B
 from paper_2608_00573_gb300 import workload as W
 from tests.gpu_helpers import compare_layer, make_engine, targeted_rows

@@ -11,7 +11,6 @@ every grouped GEMM launch of that layer (including its last persistent round)
 contributes a checked row.  Layers that are not checked still run on the GPU
 so that later checked layers see realistic state (skips, exits, budgets).
 """
-import numpy as np
 import pytest
 
 from paper_2608_00573_gb300 import workload as W
